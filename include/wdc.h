@@ -1,0 +1,280 @@
+/*
+ * wdc.h -- C ABI of libwdc.so: the WorldDynCache cached denoising rollout on
+ * one NVIDIA GB300 (sm_103a).
+ *
+ * The method (arxiv 2608.01845, "WorldDynCache: Risk-Controlled Latent Dynamics
+ * Approximation for Diffusion World Models") replaces some exact transitions
+ *     z_{t-1} = Psi_t(z_t, F_theta(z_t, t, c))                       (Eq. 1)
+ * of a diffusion world model's rollout by a surrogate
+ *     z_hat_{t-1} = G_t(z_t, H_t)                                   (Eq. 1-5)
+ * whenever a calibrated, accumulated transition risk allows it (Eq. 6-10).
+ *
+ * Conventions for every entry point:
+ *  - Errors are reported by return code only; nothing aborts or throws across
+ *    the ABI.  Argument errors are detected before any launch.  After an error
+ *    wdc_last_error(ctx) holds a one-line description.
+ *  - Pointers named "device" must point to memory of the context's device;
+ *    latents are fp32, contiguous [C, F, H, W] (flat N = C*F*H*W elements) and
+ *    16-byte aligned.  The caller owns every pointer it passes; the context
+ *    owns its weights, bank latents, workspace and controller state.
+ *  - Work is enqueued on the given stream (a cudaStream_t; NULL = the legacy
+ *    default stream).  Calls that must return a decision to the host
+ *    (wdc_surrogate_step, wdc_rollout) synchronise that stream.
+ *  - Step index convention: step k = 0..T-1 maps z_k to z_{k+1}; the paper's
+ *    t counts down (t = T - k).  Noise levels sigma_k = 1 - k/T (optionally
+ *    time-shifted), model timestep 1000*sigma_k, phase q_k = sigma_k.
+ *  - A context is not thread-safe; use one per host thread.
+ */
+#ifndef WDC_H
+#define WDC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum wdc_status {
+    WDC_OK = 0,
+    WDC_ERR_INVALID_ARG = 1,   /* bad pointer, size, alignment or config        */
+    WDC_ERR_CUDA = 2,          /* a CUDA runtime/driver call failed              */
+    WDC_ERR_UNSUPPORTED = 3,   /* valid request this build does not implement    */
+    WDC_ERR_TIMEOUT = 4,       /* a bounded device-side wait gave up             */
+    WDC_ERR_NONFINITE = 5,     /* reserved: non-finite data where it is an error */
+    WDC_ERR_STATE = 6,         /* call out of order for the context's state      */
+    WDC_ERR_OOM = 7            /* device allocation failed                       */
+} wdc_status;
+
+enum { WDC_F32 = 0, WDC_BF16 = 1 };
+
+#define WDC_MAX_BANK 8          /* largest supported bank capacity K           */
+#define WDC_SUMMARY_DIM 256     /* the fixed summary s(.) (section "Kernelized Nonlinear Observation") */
+#define WDC_SKETCH 120          /* buckets of each latent block of s(.)        */
+
+typedef struct wdc_ctx wdc_ctx;
+typedef void* wdc_stream;       /* a cudaStream_t */
+
+/* The denoiser F_theta: an adaLN DiT over video-latent tokens.  The paper
+ * takes F_theta from the backbone (Introduction, Eq. 1); layer layout:
+ *   x = [Linear(cond tokens); Linear(patchify(z)) + sinusoidal position]
+ *   per block: x += g1*(Wo Attn(LN(x)(1+s1)+b1) + bo);
+ *              x += g2*(W2 GELU_tanh(W1(LN(x)(1+s2)+b2) + b1') + b2')
+ *   v = unpatchify(Wf(LN(x_video)(1+sf)+bf) + bf')
+ * layers == 0 creates a context without a denoiser (controller and fused step
+ * kernels only); then the latent shape [in_ch, frames, height, width] is
+ * arbitrary. */
+typedef struct wdc_dit_config {
+    int layers, hidden, heads, head_dim, mlp, temb_dim, freq_dim;
+    int in_ch, frames, height, width, patch;
+    int cond_tokens, cond_dim;
+    int dual_stream;            /* 1: separate block weights for condition tokens */
+    int dtype;                  /* WDC_F32 (fp32 parity mode) or WDC_BF16          */
+} wdc_dit_config;
+
+/* Flow-matching Euler schedule: sigma_k = 1 - k/T, shifted by
+ * s*sigma/(1+(s-1)*sigma) when shift != 1. */
+typedef struct wdc_schedule {
+    int T;
+    double shift;
+} wdc_schedule;
+
+/* Constants of Eq. 3-10.  The paper defers their values to supplementary
+ * material; wdc_default_cache_params() fills the readings this library uses. */
+typedef struct wdc_cache_params {
+    int bank_capacity;          /* FIFO capacity K of the bank, 1..WDC_MAX_BANK  */
+    int min_support;            /* |N_t| needed for adequate support             */
+    double sim_min, q_gap_max;  /* compatibility (Eq. 3 text)                    */
+    double gamma_q, tau_in;     /* retrieval score and temperature (Eq. 3)       */
+    double tau_obs;             /* observation temperature tau (Eq. 5)           */
+    double alpha_min, alpha_max;/* clip of the scheduler scaling (Eq. 4)         */
+    double eps, eps_nu;         /* Eq. 4/7/8 epsilon; RMS-normalisation epsilon  */
+    uint32_t sketch_seed;       /* seed of the summary's sign hash               */
+    double w_z, w_age, w_phase, w_cam, w_depth;   /* proxy weights (Eq. 6)       */
+    double eta_init, eta_min, eta_max, beta_d;    /* calibration (Eq. 8)         */
+    double a_cam, a_depth, a_phase;               /* impact weight (Eq. 9)       */
+    double lambda_, tau_risk;                     /* decay and threshold (Eq. 9-10) */
+    int max_age;                /* pre-decision anchor age limit (Eq. 10 text)   */
+    int n_init_exact, n_final_exact;              /* mandatory-exact phases      */
+    int flags;                  /* reserved, must be 0                           */
+} wdc_cache_params;
+
+/* Model condition c of one step.  tokens: [cond_tokens, cond_dim] fp32, device
+ * or host memory (NULL only when layers == 0).  cam/depth: the camera/motion
+ * and depth/geometry descriptors of the lift (Eq. 2); zero when missing. */
+typedef struct wdc_cond {
+    const float* tokens;
+    double cam[4];
+    double depth[4];
+} wdc_cond;
+
+/* Per-step record filled by the step calls (host memory). */
+typedef struct wdc_step_info {
+    int k;
+    int decision;               /* 1 Surrogate, 0 Exact (Eq. 10)                 */
+    int finite, supported, n_compat, n_bank, age;
+    double q, alpha, p, d_hat, w, delta, R_cand, R, eta, d_cf, d_z, r;
+    double kappa[WDC_MAX_BANK], pi[WDC_MAX_BANK];
+} wdc_step_info;
+
+/* One bank record's small fields (section "Local Lifted Evolution"): the
+ * summaries of the lifted input and output and their increment, the phases,
+ * the relative RMS increment r of the transition and its descriptors. */
+typedef struct wdc_record_host {
+    double s_in[WDC_SUMMARY_DIM], s_out[WDC_SUMMARY_DIM], s_dphi[WDC_SUMMARY_DIM];
+    double q_in, q_out, r;
+    double cam[4], depth[4];
+} wdc_record_host;
+
+/* Host view of the controller and memory state.  In wdc_state_set the
+ * "derived" fields are ignored and recomputed on the device from the latents. */
+typedef struct wdc_state_host {
+    int n_bank;                 /* records rec[0..n_bank-1], oldest first        */
+    int age;                    /* surrogate steps since the latest exact step   */
+    double R, eta;              /* stored risk and calibration gain              */
+    double q_a_in, q_a_out;     /* latest exact interval                         */
+    double cam_a[4], depth_a[4];/* descriptors of the latest exact step          */
+    wdc_record_host rec[WDC_MAX_BANK];
+    /* derived (read back only) */
+    double cur_sketch[WDC_SKETCH], cur_sumsq, cur_sumsq_anchor;
+    double anchor_sketch[WDC_SKETCH], anchor_sumsq;
+    double s_phi[WDC_SUMMARY_DIM];
+    int cand_supported, cand_finite;
+    double cand_p;
+} wdc_state_host;
+
+/* Parameter tensors of the denoiser (wdc_set_tensor).  Shapes, [out, in] for
+ * Linear weights; D hidden, E temb_dim, M mlp, P = in_ch*patch*patch, Fd freq_dim. */
+enum wdc_tensor_id {
+    WDC_T_PATCH_W = 0,  /* [D, P]    */  WDC_T_PATCH_B = 1,  /* [D]   */
+    WDC_T_COND_W = 2,   /* [D, Dc]   */  WDC_T_COND_B = 3,   /* [D]   */
+    WDC_T_T1_W = 4,     /* [E, Fd]   */  WDC_T_T1_B = 5,     /* [E]   */
+    WDC_T_T2_W = 6,     /* [E, E]    */  WDC_T_T2_B = 7,     /* [E]   */
+    WDC_T_FMOD_W = 8,   /* [2D, E]   */  WDC_T_FMOD_B = 9,   /* [2D]  */
+    WDC_T_FINAL_W = 10, /* [P, D]    */  WDC_T_FINAL_B = 11, /* [P]   */
+    /* per (layer, stream) */
+    WDC_T_MOD_W = 12,   /* [6D, E]   */  WDC_T_MOD_B = 13,   /* [6D]  */
+    WDC_T_QKV_W = 14,   /* [3D, D]   */  WDC_T_QKV_B = 15,   /* [3D]  */
+    WDC_T_O_W = 16,     /* [D, D]    */  WDC_T_O_B = 17,     /* [D]   */
+    WDC_T_FC1_W = 18,   /* [M, D]    */  WDC_T_FC1_B = 19,   /* [M]   */
+    WDC_T_FC2_W = 20,   /* [D, M]    */  WDC_T_FC2_B = 21,   /* [D]   */
+    WDC_T_COUNT = 22
+};
+
+/* ------------------------------------------------------------------ lifetime */
+const char* wdc_status_string(wdc_status s);
+/* Fills the parameter readings used by default (see wdc_cache_params). */
+wdc_status wdc_default_cache_params(wdc_cache_params* out);
+/* Creates a context on CUDA device `device`: validates the configs, allocates
+ * the weights (when layers > 0), the K bank latents, two candidate buffers,
+ * the velocity buffer, the DiT workspace and the device controller state.
+ * WDC_ERR_OOM if device memory is short. */
+wdc_status wdc_create(const wdc_dit_config* cfg, const wdc_schedule* sched,
+                      const wdc_cache_params* params, int device, wdc_ctx** out);
+void wdc_destroy(wdc_ctx* ctx);
+const char* wdc_last_error(const wdc_ctx* ctx);
+size_t wdc_latent_numel(const wdc_ctx* ctx);
+/* Number of kernels this context has launched so far (all streams). */
+unsigned long long wdc_launch_count(const wdc_ctx* ctx);
+
+/* ------------------------------------------------------------------ weights */
+/* Copies one parameter tensor (host fp32, `count` elements, shape as listed in
+ * wdc_tensor_id) into the model, converting to the model dtype (bf16:
+ * round-to-nearest-even).  layer/stream are ignored for global tensors. */
+wdc_status wdc_set_tensor(wdc_ctx* ctx, int tensor_id, int layer, int stream,
+                          const float* host, size_t count);
+/* Initialises every matrix N(0, std^2) and every bias to 0 on the device from
+ * a counter-based Philox4x32-10 stream (Salmon et al., SC'11) keyed by seed. */
+wdc_status wdc_init_weights(wdc_ctx* ctx, unsigned long long seed, float std);
+
+/* ------------------------------------------------------------------ F_theta */
+/* v = F_theta(z_t, t, c) (Eq. 1): z_t device fp32 latent, t the model timestep,
+ * cond_tokens device fp32 [cond_tokens, cond_dim], v device fp32 latent-shaped
+ * output.  Asynchronous. */
+wdc_status wdc_dit_forward(wdc_ctx* ctx, const float* z_t, float t, const float* cond_tokens,
+                           float* v, wdc_stream stream);
+/* One DiT block in place on the token sequence x (device, model dtype,
+ * [cond_tokens + video_tokens, hidden]) with modulation mod6 (device fp32,
+ * [streams][6][hidden] = shift1, scale1, gate1, shift2, scale2, gate2). */
+wdc_status wdc_dit_block_forward(wdc_ctx* ctx, int layer, void* x, const float* mod6,
+                                 wdc_stream stream);
+/* Timestep conditioning: writes [layers][streams][6][hidden] block modulations
+ * followed by the final layer's [2][hidden] into mod_out (device fp32). */
+wdc_status wdc_dit_modulation(wdc_ctx* ctx, float t, float* mod_out, wdc_stream stream);
+
+/* ------------------------------------------------------------------ Psi_t */
+/* z_next = Psi_k(z_t, v) = z_t + (sigma_{k+1} - sigma_k) v (Eq. 1, flow-matching
+ * Euler), elementwise fp32 (one fused multiply-add).  z_next may equal z_t. */
+wdc_status wdc_scheduler_step(wdc_ctx* ctx, int k, const float* z_t, const float* v,
+                              float* z_next, wdc_stream stream);
+
+/* ------------------------------------------------------------------ cache state */
+/* Starts a rollout from z_T (device): empties the bank, R = 0,
+ * eta = eta_init, age = 0, anchor z_a := a copy of z_T, and computes the
+ * current latent's statistics. */
+wdc_status wdc_state_reset(wdc_ctx* ctx, const float* z_T, wdc_stream stream);
+/* Reads the controller/memory state back (synchronises the stream). */
+wdc_status wdc_state_get(wdc_ctx* ctx, wdc_state_host* out, wdc_stream stream);
+/* Installs a state: the small fields from `in`, bank latents copied from
+ * z_out[0..in->n_bank-1] (device), the anchor = the newest record's latent
+ * (or a copy of z_cur when the bank is empty), and recomputes the derived
+ * statistics from z_cur (device) and the anchor.  For tests and resume. */
+wdc_status wdc_state_set(wdc_ctx* ctx, const wdc_state_host* in, const float* const* z_out,
+                         const float* z_cur, wdc_stream stream);
+
+/* ------------------------------------------------------------------ steps */
+/* Surrogate candidate and decision of step k (Eq. 2-6, 9, 10) in one fused,
+ * HBM-bound pass: lifts the current state (its statistics are held by the
+ * context), retrieves and evolves in summary space, and when supported writes
+ * z_hat = sum_i kappa_i z_out_i (Eq. 5) to `z_hat` (device, N floats) while
+ * reducing the statistics the next step needs; then decides.  On Surrogate the
+ * state advances (R <- R_cand, age += 1) and z_hat becomes the current latent
+ * (keep the buffer alive until the next step).  On Exact the caller runs
+ * F_theta and wdc_risk_update.  Synchronises the stream; `info` (host) gets
+ * the step record. */
+wdc_status wdc_surrogate_step(wdc_ctx* ctx, int k, const wdc_cond* c, float* z_hat,
+                              wdc_step_info* info, wdc_stream stream);
+/* Exact branch of step k (Eq. 1, 7, 8; section "Reliability Decision"): one
+ * fused pass writes z_exact = Psi_k(z_t, v) straight into the bank's FIFO slot,
+ * reduces the counterfactual defect against z_cf (the candidate of the same
+ * step, or NULL), calibrates eta_d when that candidate was supported and
+ * finite, decays R <- lambda R and inserts the record lifted with the
+ * pre-insertion anchor and history.  *z_next receives the device address of
+ * z_exact (owned by the context, valid until that slot is recycled).
+ * `info` may be NULL; when given, the stream is synchronised and it is
+ * completed with d_cf, R, eta and r. */
+wdc_status wdc_risk_update(wdc_ctx* ctx, int k, const wdc_cond* c, const float* z_t,
+                           const float* v, const float* z_cf, const float** z_next,
+                           wdc_step_info* info, wdc_stream stream);
+
+/* ------------------------------------------------------------------ rollouts */
+/* The cached rollout (section "Inference and Complexity"): T steps from z_T,
+ * each a wdc_surrogate_step and, on Exact, wdc_dit_forward + wdc_risk_update.
+ * z_T and z_out may be device or host pointers (host ones are staged through
+ * the context's buffers).  conds: n_cond == 1 (used for every step) or T
+ * entries.  decisions (host int[T]) and trace (host wdc_step_info[T]) may be
+ * NULL.  Synchronises the stream once per step. */
+wdc_status wdc_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* conds, int n_cond,
+                       float* z_out, int* decisions, wdc_step_info* trace, wdc_stream stream);
+/* The uncached rollout: wdc_dit_forward + wdc_scheduler_step at every step. */
+wdc_status wdc_native_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* conds, int n_cond,
+                              float* z_out, wdc_stream stream);
+
+/* ------------------------------------------------------------------ operators
+ * The denoiser's hot kernels, exposed for parity tests and roofline timing.   */
+/* C = epilogue(A W^T): A [M, K], W [N, K] (model dtype, device, row-major);
+ * bias [N] fp32 or NULL; gelu != 0 applies GELU_tanh; when res != NULL
+ * C = res + gate * (.) with gate [N] fp32 (NULL = 1) and res/C [M, N] in the
+ * model dtype (res may equal C). */
+wdc_status wdc_op_gemm(wdc_ctx* ctx, const void* A, const void* W, const float* bias, void* C,
+                       int M, int N, int K, int gelu, const void* res, const float* gate,
+                       wdc_stream stream);
+/* O = softmax(Q K^T / sqrt(d)) V per head, non-causal: q, k [heads, L, d],
+ * vt [heads, d, L] (V transposed), o [L, heads*d]; model dtype, device. */
+wdc_status wdc_op_attention(wdc_ctx* ctx, const void* q, const void* k, const void* vt, void* o,
+                            int heads, int L, int d, wdc_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* WDC_H */

@@ -1,0 +1,672 @@
+// The exact denoiser F_theta (Eq. 1): an adaLN-modulated DiT over video-latent
+// tokens, and its orchestration on one GPU.
+//
+// Layer layout (the paper takes F_theta from its backbone; this is the DiT
+// reading shared with the CPU checker):
+//   x = [Linear(cond tokens); Linear(patchify(z)) + sinusoidal position]
+//   per block: x += gate1 * (W_o Attn(LN(x)(1+scale1)+shift1) + b_o)
+//              x += gate2 * (W_2 GELU_tanh(W_1 (LN(x)(1+scale2)+shift2) + b_1) + b_2)
+//   v = unpatchify(W_f (LN(x_video)(1+scale_f)+shift_f) + b_f)
+//   modulations = W_mod SiLU(temb), temb = W_t2 SiLU(W_t1 f(t) + b_t1) + b_t2.
+//
+// fp32 mode (parity) runs every kernel in fp32 SIMT form.  bf16 mode keeps
+// activations and weights in bf16 with fp32 accumulation; its GEMMs and
+// attention are the tcgen05/TMEM kernels of gemm_tc.cu and attn_tc.cu.
+#include "dit_kernels.cuh"
+
+#include <cmath>
+#include <cstring>
+#include <vector>
+
+namespace wdc {
+
+// tcgen05 paths (gemm_tc.cu, attn_tc.cu); return false when the shape is not
+// supported so the caller can report it.
+bool tc_gemm_supported(int M, int N, int K);
+wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, const Epi& e, cudaStream_t s);
+bool tc_attention_supported(int L, int d);
+wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
+                        cudaStream_t s);
+
+struct Lin {
+    void* w = nullptr;
+    float* b = nullptr;
+    int out = 0, in = 0;
+};
+
+struct DiT {
+    int dtype = WDC_F32;
+    size_t esz = 4;
+    int S = 1;                            // weight streams (2 with dual_stream)
+    int D = 0, H = 0, d = 0, M = 0, E = 0, Fd = 0, P = 0, Lc = 0, Lv = 0, L = 0, Dc = 0, layers = 0;
+    Lin patch, cond, t1, t2, fin;
+    void* modW = nullptr;                 // [(layers*S*6 + 2) * D, E]
+    float* modB = nullptr;
+    size_t mod_rows = 0;
+    std::vector<Lin> qkv, o, fc1, fc2;    // index layer * S + stream
+    // activations / workspace
+    void *x = nullptr, *h = nullptr, *q = nullptr, *k = nullptr, *vt = nullptr, *ao = nullptr, *m = nullptr;
+    void *tok = nullptr, *condx = nullptr, *pe = nullptr;
+    float *feat = nullptr, *h1 = nullptr, *temb = nullptr, *mods = nullptr;
+    std::vector<void*> allocs;
+};
+
+namespace {
+
+// ---------------------------------------------------------------- small kernels
+__global__ void features_kernel(float t, int half, float* out) {
+    const int j = threadIdx.x + blockIdx.x * blockDim.x;
+    if (j >= half) return;
+    const double w = exp(-log(10000.0) * (double)j / (double)half);
+    const double a = (double)t * w;
+    out[j] = (float)cos(a);
+    out[half + j] = (float)sin(a);
+}
+
+// y[r] = act(W[r,:] . x + b[r]); one warp per row.  act: 0 none, 1 SiLU.
+template <typename T>
+__global__ void gemv_kernel(const T* __restrict__ W, const float* __restrict__ x, const float* __restrict__ b,
+                            float* __restrict__ y, int rows, int cols, int act) {
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+    if (warp >= rows) return;
+    const T* w = W + (size_t)warp * cols;
+    float s = 0.f;
+    for (int c = lane; c < cols; c += 32) s = fmaf(ld_act<T>(w + c), x[c], s);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) {
+        float v = s + (b ? b[warp] : 0.f);
+        if (act == 1) v = v / (1.0f + expf(-v));
+        y[warp] = v;
+    }
+}
+
+// h[r] = LN(x[r]) * (1 + scale) + shift, one warp per row, rows [r0, r1).
+template <typename T, int VPT>
+__global__ void ln_mod_kernel(const T* __restrict__ x, T* __restrict__ h, int r0, int r1, int D,
+                              const float* __restrict__ shift, const float* __restrict__ scale, int h_row_off) {
+    const int row = r0 + ((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    if (row >= r1) return;
+    const T* xr = x + (size_t)row * D;
+    float v[VPT];
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < VPT; ++i) {
+        const int c = lane + 32 * i;
+        v[i] = (c < D) ? ld_act<T>(xr + c) : 0.f;
+        s += v[i];
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const float mean = s / (float)D;
+    float q = 0.f;
+#pragma unroll
+    for (int i = 0; i < VPT; ++i) {
+        const int c = lane + 32 * i;
+        const float dlt = (c < D) ? v[i] - mean : 0.f;
+        q += dlt * dlt;
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+    const float rstd = 1.0f / sqrtf(q / (float)D + 1e-6f);
+    T* hr = h + (size_t)(row - h_row_off) * D;
+#pragma unroll
+    for (int i = 0; i < VPT; ++i) {
+        const int c = lane + 32 * i;
+        if (c < D) hr[c] = to_act<T>(fmaf((v[i] - mean) * rstd, 1.0f + scale[c], shift[c]));
+    }
+}
+
+// tok[(f, h', w'), (c, ph, pw)] = z[c, f, h'*p+ph, w'*p+pw]
+template <typename T>
+__global__ void patchify_kernel(const float* __restrict__ z, T* __restrict__ tok, int C, int F, int Hh, int Ww, int p) {
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const int P = C * p * p, hp = Hh / p, wp = Ww / p;
+    const long long total = (long long)F * hp * wp * P;
+    if (i >= total) return;
+    const int col = (int)(i % P);
+    const long long m = i / P;
+    const int f = (int)(m / (hp * wp)), rem = (int)(m % (hp * wp)), h2 = rem / wp, w2 = rem % wp;
+    const int c = col / (p * p), r2 = col % (p * p), ph = r2 / p, pw = r2 % p;
+    tok[i] = to_act<T>(z[(((size_t)c * F + f) * Hh + h2 * p + ph) * Ww + w2 * p + pw]);
+}
+
+template <typename T>
+__global__ void convert_kernel(const float* __restrict__ src, T* __restrict__ dst, long long n) {
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) dst[i] = to_act<T>(src[i]);
+}
+
+template <typename T>
+__global__ void posemb_kernel(T* __restrict__ pe, int n, int D) {
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (long long)n * D) return;
+    const int row = (int)(i / D), col = (int)(i % D), j = col / 2;
+    const double w = pow(10000.0, -2.0 * (double)j / (double)D);
+    const double a = (double)row * w;
+    pe[i] = to_act<T>((float)((col & 1) ? cos(a) : sin(a)));
+}
+
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) + Box-Muller.
+__device__ __forceinline__ void philox(uint32_t c[4], uint32_t k0, uint32_t k1) {
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        const uint32_t hi0 = __umulhi(0xD2511F53u, c[0]), lo0 = 0xD2511F53u * c[0];
+        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c[2]), lo1 = 0xCD9E8D57u * c[2];
+        const uint32_t n0 = hi1 ^ c[1] ^ k0, n2 = hi0 ^ c[3] ^ k1;
+        c[0] = n0; c[1] = lo1; c[2] = n2; c[3] = lo0;
+        k0 += 0x9E3779B9u;
+        k1 += 0xBB67AE85u;
+    }
+}
+
+template <typename T>
+__global__ void normal_init_kernel(T* __restrict__ dst, long long n, unsigned long long seed, uint32_t stream_id,
+                                   float std) {
+    const long long i4 = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i4 * 4 >= n) return;
+    uint32_t c[4] = {(uint32_t)i4, (uint32_t)(i4 >> 32), stream_id, 0x57444331u};
+    philox(c, (uint32_t)seed, (uint32_t)(seed >> 32));
+    const float u0 = ((float)c[0] + 0.5f) * 2.3283064365386963e-10f;
+    const float u1 = ((float)c[1] + 0.5f) * 2.3283064365386963e-10f;
+    const float u2 = ((float)c[2] + 0.5f) * 2.3283064365386963e-10f;
+    const float u3 = ((float)c[3] + 0.5f) * 2.3283064365386963e-10f;
+    const float r0 = sqrtf(-2.0f * logf(u0)), r1 = sqrtf(-2.0f * logf(u2));
+    float s0, c0, s1, c1;
+    sincospif(2.0f * u1, &s0, &c0);
+    sincospif(2.0f * u3, &s1, &c1);
+    const float v[4] = {r0 * c0, r0 * s0, r1 * c1, r1 * s1};
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+        if (i4 * 4 + j < n) dst[i4 * 4 + j] = to_act<T>(std * v[j]);
+}
+
+// ---------------------------------------------------------------- SIMT GEMM
+// C = epilogue(A W^T), A [M, K], W [N, K]; 64x64 tiles, 4x4 per thread,
+// sequential-k fp32 accumulation.
+template <typename T>
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ W, int M,
+                                                         int N, int K, const Epi e) {
+    __shared__ float As[16][68];
+    __shared__ float Ws[16][68];
+    const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+    const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+    float acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+    for (int k0 = 0; k0 < K; k0 += 16) {
+        for (int i = threadIdx.x; i < 1024; i += 256) {
+            const int r = i / 16, kk = i % 16, gk = k0 + kk;
+            const int gm = m0 + r, gn = n0 + r;
+            As[kk][r] = (gm < M && gk < K) ? ld_act<T>(A + (size_t)gm * K + gk) : 0.f;
+            Ws[kk][r] = (gn < N && gk < K) ? ld_act<T>(W + (size_t)gn * K + gk) : 0.f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < 16; ++kk) {
+            float a[4], b[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) b[j] = Ws[kk][tx * 4 + j];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int m = m0 + ty * 4 + i, n = n0 + tx * 4 + j;
+            if (m < M && n < N) epi_apply<T>(e, m, n, acc[i][j]);
+        }
+}
+
+// ---------------------------------------------------------------- SIMT attention
+// One thread per query row, online softmax over key tiles staged in shared memory.
+template <typename T, int HD>
+__global__ void __launch_bounds__(128) attn_simt_kernel(const T* __restrict__ q, const T* __restrict__ k,
+                                                         const T* __restrict__ vt, T* __restrict__ o, int H, int L,
+                                                         float scale) {
+    constexpr int KT = HD <= 64 ? 64 : 32;
+    __shared__ float Ks[KT][HD + 1];
+    __shared__ float Vs[KT][HD + 1];
+    const int h = blockIdx.y;
+    const int qi = blockIdx.x * 128 + threadIdx.x;
+    float qr[HD], acc[HD];
+#pragma unroll
+    for (int dd = 0; dd < HD; ++dd) {
+        qr[dd] = (qi < L) ? ld_act<T>(q + ((size_t)h * L + qi) * HD + dd) : 0.f;
+        acc[dd] = 0.f;
+    }
+    float mx = -INFINITY, l = 0.f;
+    for (int j0 = 0; j0 < L; j0 += KT) {
+        for (int i = threadIdx.x; i < KT * HD; i += 128) {
+            const int jj = i / HD, dd = i % HD;
+            Ks[jj][dd] = (j0 + jj < L) ? ld_act<T>(k + ((size_t)h * L + j0 + jj) * HD + dd) : 0.f;
+            const int dv = i / KT, jv = i % KT;
+            Vs[jv][dv] = (j0 + jv < L) ? ld_act<T>(vt + ((size_t)h * HD + dv) * L + j0 + jv) : 0.f;
+        }
+        __syncthreads();
+        const int nk = min(KT, L - j0);
+        for (int jj = 0; jj < nk; ++jj) {
+            float s = 0.f;
+#pragma unroll
+            for (int dd = 0; dd < HD; ++dd) s = fmaf(qr[dd], Ks[jj][dd], s);
+            s *= scale;
+            if (s > mx) {
+                const float corr = expf(mx - s);
+                l *= corr;
+#pragma unroll
+                for (int dd = 0; dd < HD; ++dd) acc[dd] *= corr;
+                mx = s;
+            }
+            const float pj = expf(s - mx);
+            l += pj;
+#pragma unroll
+            for (int dd = 0; dd < HD; ++dd) acc[dd] = fmaf(pj, Vs[jj][dd], acc[dd]);
+        }
+        __syncthreads();
+    }
+    if (qi < L) {
+        const float inv = 1.0f / l;
+#pragma unroll
+        for (int dd = 0; dd < HD; ++dd) o[(size_t)qi * H * HD + h * HD + dd] = to_act<T>(acc[dd] * inv);
+    }
+}
+
+inline unsigned blocks_for(long long n, int per) { return (unsigned)((n + per - 1) / per); }
+
+template <typename T>
+void launch_ln_mod(const void* x, void* h, int r0, int r1, int D, const float* shift, const float* scale,
+                   int h_row_off, cudaStream_t s) {
+    const int rows = r1 - r0;
+    if (rows <= 0) return;
+    const unsigned grid = blocks_for((long long)rows * 32, 256);
+    const T* xp = reinterpret_cast<const T*>(x);
+    T* hp = reinterpret_cast<T*>(h);
+    if (D <= 256) ln_mod_kernel<T, 8><<<grid, 256, 0, s>>>(xp, hp, r0, r1, D, shift, scale, h_row_off);
+    else if (D <= 1024) ln_mod_kernel<T, 32><<<grid, 256, 0, s>>>(xp, hp, r0, r1, D, shift, scale, h_row_off);
+    else ln_mod_kernel<T, 128><<<grid, 256, 0, s>>>(xp, hp, r0, r1, D, shift, scale, h_row_off);
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------- dispatch
+static wdc_status gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, const Epi& e, cudaStream_t s) {
+    if (M <= 0 || N <= 0) return WDC_OK;
+    if (c->cfg.dtype == WDC_BF16 && tc_gemm_supported(M, N, K)) return tc_gemm(c, A, W, M, N, K, e, s);
+    dim3 grid(blocks_for(N, 64), blocks_for(M, 64));
+    if (c->cfg.dtype == WDC_BF16)
+        gemm_simt_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(reinterpret_cast<const __nv_bfloat16*>(A),
+                                                             reinterpret_cast<const __nv_bfloat16*>(W), M, N, K, e);
+    else
+        gemm_simt_kernel<float><<<grid, 256, 0, s>>>(reinterpret_cast<const float*>(A),
+                                                     reinterpret_cast<const float*>(W), M, N, K, e);
+    c->launches++;
+    return WDC_OK;
+}
+
+static wdc_status attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
+                            cudaStream_t s) {
+    if (c->cfg.dtype == WDC_BF16 && tc_attention_supported(L, d)) return tc_attention(c, q, k, vt, o, H, L, d, s);
+    dim3 grid(blocks_for(L, 128), H);
+    const float scale = 1.0f / sqrtf((float)d);
+    if (c->cfg.dtype == WDC_BF16) {
+        using T = __nv_bfloat16;
+        if (d == 64)
+            attn_simt_kernel<T, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+        else
+            attn_simt_kernel<T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+    } else {
+        using T = float;
+        if (d == 64)
+            attn_simt_kernel<T, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+        else
+            attn_simt_kernel<T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+    }
+    c->launches++;
+    return WDC_OK;
+}
+
+static void ln_mod(Ctx* c, const void* x, void* h, int r0, int r1, const float* shift, const float* scale,
+                   int h_row_off, cudaStream_t s) {
+    if (r1 <= r0) return;
+    if (c->cfg.dtype == WDC_BF16)
+        launch_ln_mod<__nv_bfloat16>(x, h, r0, r1, c->cfg.hidden, shift, scale, h_row_off, s);
+    else
+        launch_ln_mod<float>(x, h, r0, r1, c->cfg.hidden, shift, scale, h_row_off, s);
+    c->launches++;
+}
+
+// ---------------------------------------------------------------- lifetime
+static wdc_status dalloc(Ctx* c, void** p, size_t bytes) {
+    DiT* t = c->dit;
+    cudaError_t e = cudaMalloc(p, bytes ? bytes : 16);
+    if (e != cudaSuccess) return fail(c, WDC_ERR_OOM, std::string("cudaMalloc: ") + cudaGetErrorString(e));
+    t->allocs.push_back(*p);
+    cudaMemset(*p, 0, bytes ? bytes : 16);
+    return WDC_OK;
+}
+
+static wdc_status alloc_lin(Ctx* c, Lin& l, int out, int in) {
+    l.out = out;
+    l.in = in;
+    wdc_status s = dalloc(c, &l.w, (size_t)out * in * c->dit->esz);
+    if (s) return s;
+    return dalloc(c, (void**)&l.b, (size_t)out * sizeof(float));
+}
+
+wdc_status dit_create(Ctx* c) {
+    const wdc_dit_config& g = c->cfg;
+    DiT* t = new DiT();
+    c->dit = t;
+    t->dtype = g.dtype;
+    t->esz = g.dtype == WDC_BF16 ? 2 : 4;
+    t->S = g.dual_stream ? 2 : 1;
+    t->D = g.hidden;
+    t->H = g.heads;
+    t->d = g.head_dim;
+    t->M = g.mlp;
+    t->E = g.temb_dim;
+    t->Fd = g.freq_dim;
+    t->P = g.in_ch * g.patch * g.patch;
+    t->Lc = g.cond_tokens;
+    t->Lv = g.frames * (g.height / g.patch) * (g.width / g.patch);
+    t->L = t->Lc + t->Lv;
+    t->Dc = g.cond_dim;
+    t->layers = g.layers;
+    wdc_status s;
+    if ((s = alloc_lin(c, t->patch, t->D, t->P))) return s;
+    if ((s = alloc_lin(c, t->cond, t->D, t->Dc > 0 ? t->Dc : 1))) return s;
+    if ((s = alloc_lin(c, t->t1, t->E, t->Fd))) return s;
+    if ((s = alloc_lin(c, t->t2, t->E, t->E))) return s;
+    if ((s = alloc_lin(c, t->fin, t->P, t->D))) return s;
+    t->mod_rows = ((size_t)t->layers * t->S * 6 + 2) * t->D;
+    if ((s = dalloc(c, &t->modW, t->mod_rows * t->E * t->esz))) return s;
+    if ((s = dalloc(c, (void**)&t->modB, t->mod_rows * sizeof(float)))) return s;
+    const int n = t->layers * t->S;
+    t->qkv.resize(n);
+    t->o.resize(n);
+    t->fc1.resize(n);
+    t->fc2.resize(n);
+    for (int i = 0; i < n; ++i) {
+        if ((s = alloc_lin(c, t->qkv[i], 3 * t->D, t->D))) return s;
+        if ((s = alloc_lin(c, t->o[i], t->D, t->D))) return s;
+        if ((s = alloc_lin(c, t->fc1[i], t->M, t->D))) return s;
+        if ((s = alloc_lin(c, t->fc2[i], t->D, t->M))) return s;
+    }
+    const size_t LD = (size_t)t->L * t->D * t->esz;
+    if ((s = dalloc(c, &t->x, LD))) return s;
+    if ((s = dalloc(c, &t->h, LD))) return s;
+    if ((s = dalloc(c, &t->q, LD))) return s;
+    if ((s = dalloc(c, &t->k, LD))) return s;
+    if ((s = dalloc(c, &t->vt, LD))) return s;
+    if ((s = dalloc(c, &t->ao, LD))) return s;
+    if ((s = dalloc(c, &t->m, (size_t)t->L * t->M * t->esz))) return s;
+    if ((s = dalloc(c, &t->tok, (size_t)t->Lv * t->P * t->esz))) return s;
+    if ((s = dalloc(c, &t->condx, (size_t)(t->Lc > 0 ? t->Lc : 1) * (t->Dc > 0 ? t->Dc : 1) * t->esz))) return s;
+    if ((s = dalloc(c, &t->pe, (size_t)t->Lv * t->D * t->esz))) return s;
+    if ((s = dalloc(c, (void**)&t->feat, (size_t)t->Fd * sizeof(float)))) return s;
+    if ((s = dalloc(c, (void**)&t->h1, (size_t)t->E * sizeof(float)))) return s;
+    if ((s = dalloc(c, (void**)&t->temb, (size_t)t->E * sizeof(float)))) return s;
+    if ((s = dalloc(c, (void**)&t->mods, t->mod_rows * sizeof(float)))) return s;
+    const long long npe = (long long)t->Lv * t->D;
+    if (t->dtype == WDC_BF16)
+        posemb_kernel<__nv_bfloat16><<<blocks_for(npe, 256), 256>>>((__nv_bfloat16*)t->pe, t->Lv, t->D);
+    else
+        posemb_kernel<float><<<blocks_for(npe, 256), 256>>>((float*)t->pe, t->Lv, t->D);
+    c->launches++;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("DiT init: ") + cudaGetErrorString(e));
+    return WDC_OK;
+}
+
+void dit_destroy(Ctx* c) {
+    if (!c->dit) return;
+    for (void* p : c->dit->allocs) cudaFree(p);
+    delete c->dit;
+    c->dit = nullptr;
+}
+
+static uint16_t f32_to_bf16_bits(float f) {
+    uint32_t u;
+    std::memcpy(&u, &f, 4);
+    if ((u & 0x7f800000u) == 0x7f800000u) return (uint16_t)((u >> 16) | ((u & 0xffff) ? 0x40 : 0));
+    u += 0x7fffu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+static wdc_status upload(Ctx* c, void* dst, const float* host, size_t count, bool model_dtype) {
+    if (!model_dtype || c->dit->dtype == WDC_F32) {
+        WDC_CUDA_TRY(c, cudaMemcpy(dst, host, count * sizeof(float), cudaMemcpyHostToDevice));
+        return WDC_OK;
+    }
+    std::vector<uint16_t> tmp(count);
+    for (size_t i = 0; i < count; ++i) tmp[i] = f32_to_bf16_bits(host[i]);
+    WDC_CUDA_TRY(c, cudaMemcpy(dst, tmp.data(), count * 2, cudaMemcpyHostToDevice));
+    return WDC_OK;
+}
+
+wdc_status dit_set_tensor(Ctx* c, int id, int layer, int stream, const float* host, size_t count) {
+    DiT* t = c->dit;
+    if (!t) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
+    if (!host) return fail(c, WDC_ERR_INVALID_ARG, "null host pointer");
+    const bool per_layer = id >= WDC_T_MOD_W;
+    if (per_layer && (layer < 0 || layer >= t->layers || stream < 0 || stream >= t->S))
+        return fail(c, WDC_ERR_INVALID_ARG, "layer/stream out of range");
+    const int li = layer * t->S + stream;
+    Lin* lin = nullptr;
+    bool bias = (id % 2) == 1;
+    switch (id) {
+        case WDC_T_PATCH_W: case WDC_T_PATCH_B: lin = &t->patch; break;
+        case WDC_T_COND_W: case WDC_T_COND_B: lin = &t->cond; break;
+        case WDC_T_T1_W: case WDC_T_T1_B: lin = &t->t1; break;
+        case WDC_T_T2_W: case WDC_T_T2_B: lin = &t->t2; break;
+        case WDC_T_FINAL_W: case WDC_T_FINAL_B: lin = &t->fin; break;
+        case WDC_T_QKV_W: case WDC_T_QKV_B: lin = &t->qkv[li]; break;
+        case WDC_T_O_W: case WDC_T_O_B: lin = &t->o[li]; break;
+        case WDC_T_FC1_W: case WDC_T_FC1_B: lin = &t->fc1[li]; break;
+        case WDC_T_FC2_W: case WDC_T_FC2_B: lin = &t->fc2[li]; break;
+        case WDC_T_MOD_W: case WDC_T_MOD_B: case WDC_T_FMOD_W: case WDC_T_FMOD_B: {
+            const size_t row0 = (id == WDC_T_MOD_W || id == WDC_T_MOD_B) ? (size_t)li * 6 * t->D
+                                                                         : (size_t)t->layers * t->S * 6 * t->D;
+            const size_t rows = (id == WDC_T_MOD_W || id == WDC_T_MOD_B) ? 6 * (size_t)t->D : 2 * (size_t)t->D;
+            if (bias) {
+                if (count != rows) return fail(c, WDC_ERR_INVALID_ARG, "modulation bias size mismatch");
+                return upload(c, t->modB + row0, host, count, false);
+            }
+            if (count != rows * t->E) return fail(c, WDC_ERR_INVALID_ARG, "modulation weight size mismatch");
+            return upload(c, (char*)t->modW + row0 * t->E * t->esz, host, count, true);
+        }
+        default: return fail(c, WDC_ERR_INVALID_ARG, "unknown tensor id");
+    }
+    if (bias) {
+        if (count != (size_t)lin->out) return fail(c, WDC_ERR_INVALID_ARG, "bias size mismatch");
+        return upload(c, lin->b, host, count, false);
+    }
+    if (count != (size_t)lin->out * lin->in) return fail(c, WDC_ERR_INVALID_ARG, "weight size mismatch");
+    return upload(c, lin->w, host, count, true);
+}
+
+static void init_normal(Ctx* c, void* dst, size_t n, unsigned long long seed, uint32_t sid, float std) {
+    const unsigned grid = blocks_for((long long)(n + 3) / 4, 256);
+    if (c->dit->dtype == WDC_BF16)
+        normal_init_kernel<__nv_bfloat16><<<grid, 256>>>((__nv_bfloat16*)dst, (long long)n, seed, sid, std);
+    else
+        normal_init_kernel<float><<<grid, 256>>>((float*)dst, (long long)n, seed, sid, std);
+    c->launches++;
+}
+
+wdc_status dit_init_weights(Ctx* c, unsigned long long seed, float std) {
+    DiT* t = c->dit;
+    if (!t) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
+    uint32_t sid = 1;
+    auto lin = [&](Lin& l) {
+        init_normal(c, l.w, (size_t)l.out * l.in, seed, sid++, std);
+        cudaMemset(l.b, 0, (size_t)l.out * sizeof(float));
+    };
+    lin(t->patch); lin(t->cond); lin(t->t1); lin(t->t2); lin(t->fin);
+    init_normal(c, t->modW, t->mod_rows * t->E, seed, sid++, std);
+    cudaMemset(t->modB, 0, t->mod_rows * sizeof(float));
+    for (size_t i = 0; i < t->qkv.size(); ++i) { lin(t->qkv[i]); lin(t->o[i]); lin(t->fc1[i]); lin(t->fc2[i]); }
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("init_weights: ") + cudaGetErrorString(e));
+    return WDC_OK;
+}
+
+// ---------------------------------------------------------------- forward
+wdc_status dit_modulation(Ctx* c, float t_model, float* mod_out, cudaStream_t s) {
+    DiT* t = c->dit;
+    if (!t) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
+    float* dst = mod_out ? mod_out : t->mods;
+    const int half = t->Fd / 2;
+    features_kernel<<<blocks_for(half, 128), 128, 0, s>>>(t_model, half, t->feat);
+    auto gv = [&](const void* W, const float* x, const float* b, float* y, int rows, int cols, int act) {
+        const unsigned grid = blocks_for((long long)rows * 32, 256);
+        if (t->dtype == WDC_BF16)
+            gemv_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)W, x, b, y, rows, cols, act);
+        else
+            gemv_kernel<float><<<grid, 256, 0, s>>>((const float*)W, x, b, y, rows, cols, act);
+    };
+    gv(t->t1.w, t->feat, t->t1.b, t->h1, t->E, t->Fd, 1);
+    gv(t->t2.w, t->h1, t->t2.b, t->temb, t->E, t->E, 1);   // SiLU(temb)
+    gv(t->modW, t->temb, t->modB, dst, (int)t->mod_rows, t->E, 0);
+    c->launches += 4;
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("modulation: ") + cudaGetErrorString(e));
+    return WDC_OK;
+}
+
+// One block on x (device, [L, D]) with mod (device fp32, [S][6][D]).
+static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, cudaStream_t s) {
+    DiT* t = c->dit;
+    const int D = t->D;
+    const size_t es = t->esz;
+    // stream s rows: s = 0 video [Lc, L), s = 1 cond [0, Lc); single stream: all rows
+    int r0[2], r1[2];
+    if (t->S == 2) { r0[0] = t->Lc; r1[0] = t->L; r0[1] = 0; r1[1] = t->Lc; }
+    else { r0[0] = 0; r1[0] = t->L; }
+    wdc_status st;
+    for (int sidx = 0; sidx < t->S; ++sidx) {
+        const float* m6 = mod + (size_t)sidx * 6 * D;
+        ln_mod(c, x, t->h, r0[sidx], r1[sidx], m6 + 0 * D, m6 + 1 * D, 0, s);
+        const Lin& w = t->qkv[layer * t->S + sidx];
+        Epi e{};
+        e.mode = kEpiQKV; e.bias = w.b; e.q = t->q; e.k = t->k; e.vt = t->vt;
+        e.L = t->L; e.H = t->H; e.d = t->d; e.D = D; e.row_off = r0[sidx];
+        if ((st = gemm(c, (char*)t->h + (size_t)r0[sidx] * D * es, w.w, r1[sidx] - r0[sidx], 3 * D, D, e, s))) return st;
+    }
+    if ((st = attention(c, t->q, t->k, t->vt, t->ao, t->H, t->L, t->d, s))) return st;
+    for (int sidx = 0; sidx < t->S; ++sidx) {
+        const float* m6 = mod + (size_t)sidx * 6 * D;
+        const int rows = r1[sidx] - r0[sidx];
+        char* xr = (char*)x + (size_t)r0[sidx] * D * es;
+        {
+            const Lin& w = t->o[layer * t->S + sidx];
+            Epi e{};
+            e.mode = kEpiResid; e.bias = w.b; e.out = xr; e.res = xr; e.ldo = D; e.gate = m6 + 2 * D;
+            if ((st = gemm(c, (char*)t->ao + (size_t)r0[sidx] * D * es, w.w, rows, D, D, e, s))) return st;
+        }
+        ln_mod(c, x, t->h, r0[sidx], r1[sidx], m6 + 3 * D, m6 + 4 * D, 0, s);
+        {
+            const Lin& w = t->fc1[layer * t->S + sidx];
+            Epi e{};
+            e.mode = kEpiStore; e.bias = w.b; e.gelu = 1; e.out = (char*)t->m + (size_t)r0[sidx] * t->M * es; e.ldo = t->M;
+            if ((st = gemm(c, (char*)t->h + (size_t)r0[sidx] * D * es, w.w, rows, t->M, D, e, s))) return st;
+        }
+        {
+            const Lin& w = t->fc2[layer * t->S + sidx];
+            Epi e{};
+            e.mode = kEpiResid; e.bias = w.b; e.out = xr; e.res = xr; e.ldo = D; e.gate = m6 + 5 * D;
+            if ((st = gemm(c, (char*)t->m + (size_t)r0[sidx] * t->M * es, w.w, rows, D, t->M, e, s))) return st;
+        }
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("block: ") + cudaGetErrorString(e));
+    return WDC_OK;
+}
+
+wdc_status dit_block(Ctx* c, int layer, void* x, const float* mod6, cudaStream_t s) {
+    if (!c->dit) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
+    if (layer < 0 || layer >= c->dit->layers) return fail(c, WDC_ERR_INVALID_ARG, "layer out of range");
+    if (!x || !mod6) return fail(c, WDC_ERR_INVALID_ARG, "null pointer");
+    return run_block(c, layer, x, mod6, s);
+}
+
+wdc_status dit_forward(Ctx* c, const float* z, float t_model, const float* cond, float* v, cudaStream_t s) {
+    DiT* t = c->dit;
+    if (!t) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
+    if (!z || !v || (t->Lc > 0 && !cond)) return fail(c, WDC_ERR_INVALID_ARG, "null pointer");
+    wdc_status st;
+    if ((st = dit_modulation(c, t_model, nullptr, s))) return st;
+    const int D = t->D;
+    const size_t es = t->esz;
+    const wdc_dit_config& g = c->cfg;
+    // embed: condition tokens, then patches + position
+    if (t->Lc > 0) {
+        const long long nc = (long long)t->Lc * t->Dc;
+        if (t->dtype == WDC_BF16)
+            convert_kernel<__nv_bfloat16><<<blocks_for(nc, 256), 256, 0, s>>>(cond, (__nv_bfloat16*)t->condx, nc);
+        else
+            convert_kernel<float><<<blocks_for(nc, 256), 256, 0, s>>>(cond, (float*)t->condx, nc);
+        c->launches++;
+        Epi e{};
+        e.mode = kEpiStore; e.bias = t->cond.b; e.out = t->x; e.ldo = D;
+        if ((st = gemm(c, t->condx, t->cond.w, t->Lc, D, t->Dc, e, s))) return st;
+    }
+    {
+        const long long nt = (long long)t->Lv * t->P;
+        if (t->dtype == WDC_BF16)
+            patchify_kernel<__nv_bfloat16><<<blocks_for(nt, 256), 256, 0, s>>>(z, (__nv_bfloat16*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
+        else
+            patchify_kernel<float><<<blocks_for(nt, 256), 256, 0, s>>>(z, (float*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
+        c->launches++;
+        Epi e{};
+        char* xv = (char*)t->x + (size_t)t->Lc * D * es;
+        e.mode = kEpiResid; e.bias = t->patch.b; e.out = xv; e.res = t->pe; e.ldo = D; e.gate = nullptr;
+        if ((st = gemm(c, t->tok, t->patch.w, t->Lv, D, t->P, e, s))) return st;
+    }
+    for (int l = 0; l < t->layers; ++l)
+        if ((st = run_block(c, l, t->x, t->mods + (size_t)l * t->S * 6 * D, s))) return st;
+    // final layer on the video tokens, unpatchified into v (fp32)
+    const float* fm = t->mods + (size_t)t->layers * t->S * 6 * D;
+    ln_mod(c, t->x, t->h, t->Lc, t->L, fm, fm + D, t->Lc, s);
+    Epi e{};
+    e.mode = kEpiUnpatch; e.bias = t->fin.b; e.v = v; e.C = g.in_ch; e.F = g.frames; e.Hh = g.height; e.Ww = g.width; e.p = g.patch;
+    if ((st = gemm(c, t->h, t->fin.w, t->Lv, t->P, D, e, s))) return st;
+    cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("forward: ") + cudaGetErrorString(ce));
+    return WDC_OK;
+}
+
+// ---------------------------------------------------------------- operators
+wdc_status op_gemm(Ctx* c, const void* A, const void* W, const float* bias, void* C, int M, int N, int K, int gelu,
+                   const void* res, const float* gate, cudaStream_t s) {
+    if (!A || !W || !C || M <= 0 || N <= 0 || K <= 0) return fail(c, WDC_ERR_INVALID_ARG, "bad gemm arguments");
+    Epi e{};
+    e.mode = res ? kEpiResid : kEpiStore; e.bias = bias; e.gelu = gelu; e.out = C; e.ldo = N; e.res = res; e.gate = gate;
+    wdc_status st = gemm(c, A, W, M, N, K, e, s);
+    if (st) return st;
+    cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("gemm: ") + cudaGetErrorString(ce));
+    return WDC_OK;
+}
+
+wdc_status op_attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
+                        cudaStream_t s) {
+    if (!q || !k || !vt || !o || H <= 0 || L <= 0 || (d != 64 && d != 128))
+        return fail(c, WDC_ERR_INVALID_ARG, "bad attention arguments");
+    wdc_status st = attention(c, q, k, vt, o, H, L, d, s);
+    if (st) return st;
+    cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("attention: ") + cudaGetErrorString(ce));
+    return WDC_OK;
+}
+
+}  // namespace wdc

@@ -1,0 +1,79 @@
+// Shared device pieces of the DiT denoiser: element access for fp32/bf16
+// activations and the fused GEMM epilogues used by both the SIMT and the
+// tcgen05 GEMM kernels.
+#pragma once
+
+#include "wdc_internal.h"
+
+namespace wdc {
+
+template <typename T> __device__ __forceinline__ float ld_act(const T* p);
+template <> __device__ __forceinline__ float ld_act<float>(const float* p) { return *p; }
+template <> __device__ __forceinline__ float ld_act<__nv_bfloat16>(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+
+template <typename T> __device__ __forceinline__ T to_act(float v);
+template <> __device__ __forceinline__ float to_act<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 to_act<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+__device__ __forceinline__ float gelu_tanh_f(float x) {
+    const float k0 = 0.7978845608028654f;   // sqrt(2/pi)
+    const float k1 = 0.044715f;
+    return 0.5f * x * (1.0f + tanhf(k0 * (x + k1 * x * x * x)));
+}
+
+enum EpiMode { kEpiStore = 0, kEpiResid = 1, kEpiQKV = 2, kEpiUnpatch = 3 };
+
+// Epilogue of C = A W^T on one output element (row m of this GEMM, column n).
+struct Epi {
+    int mode;
+    const float* bias;        // [N] or null
+    int gelu;
+    void* out;                // kEpiStore / kEpiResid: [M, ldo]
+    int ldo;
+    const void* res;          // kEpiResid: [M, ldo] (may equal out)
+    const float* gate;        // kEpiResid: [N] or null (= 1)
+    // kEpiQKV: q, k [H, L, d], vt [H, d, L]; token = row_off + m
+    void* q; void* k; void* vt;
+    int L, H, d, D, row_off;
+    // kEpiUnpatch: v fp32 [C, F, Hh, Ww]; token m = (f, h', w'), column = (c, ph, pw)
+    float* v;
+    int C, F, Hh, Ww, p;
+};
+
+template <typename T>
+__device__ __forceinline__ void epi_apply(const Epi& e, int m, int n, float acc) {
+    float x = acc + (e.bias ? e.bias[n] : 0.0f);
+    if (e.gelu) x = gelu_tanh_f(x);
+    switch (e.mode) {
+        case kEpiStore:
+            reinterpret_cast<T*>(e.out)[(size_t)m * e.ldo + n] = to_act<T>(x);
+            break;
+        case kEpiResid: {
+            const size_t idx = (size_t)m * e.ldo + n;
+            const float r = ld_act<T>(reinterpret_cast<const T*>(e.res) + idx);
+            const float g = e.gate ? e.gate[n] : 1.0f;
+            reinterpret_cast<T*>(e.out)[idx] = to_act<T>(fmaf(g, x, r));
+            break;
+        }
+        case kEpiQKV: {
+            const int which = n / e.D, c = n % e.D, h = c / e.d, dd = c % e.d;
+            const int tok = e.row_off + m;
+            if (which == 0)
+                reinterpret_cast<T*>(e.q)[((size_t)h * e.L + tok) * e.d + dd] = to_act<T>(x);
+            else if (which == 1)
+                reinterpret_cast<T*>(e.k)[((size_t)h * e.L + tok) * e.d + dd] = to_act<T>(x);
+            else
+                reinterpret_cast<T*>(e.vt)[((size_t)h * e.d + dd) * e.L + tok] = to_act<T>(x);
+            break;
+        }
+        case kEpiUnpatch: {
+            const int hp = e.Hh / e.p, wp = e.Ww / e.p;
+            const int f = m / (hp * wp), rem = m % (hp * wp), h2 = rem / wp, w2 = rem % wp;
+            const int c = n / (e.p * e.p), r2 = n % (e.p * e.p), ph = r2 / e.p, pw = r2 % e.p;
+            e.v[(((size_t)c * e.F + f) * e.Hh + h2 * e.p + ph) * e.Ww + w2 * e.p + pw] = x;
+            break;
+        }
+    }
+}
+
+}  // namespace wdc

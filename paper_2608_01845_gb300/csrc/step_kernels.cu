@@ -1,0 +1,654 @@
+// Fused, HBM-bound latent passes of the cached rollout.
+//
+//  * skip pass   (wdc_surrogate_step): per-CTA scalar head = lift summary
+//    (Eq. 2), transition retrieval (Eq. 3), scheduler scaling and lifted
+//    evolution in summary space (Eq. 4), observation weights (Eq. 5); then one
+//    streaming pass z_hat = sum_i kappa_i z_out_i (Eq. 5) that also reduces the
+//    statistics the next step's lift needs; the last CTA runs the controller
+//    tail: proxy (Eq. 6), risk (Eq. 9), Available and the decision (Eq. 10).
+//  * anchor pass (wdc_risk_update): z_exact = Psi(z_k, v) (Eq. 1) written into
+//    the bank slot, counterfactual-defect sums (Eq. 7) and the new record's
+//    statistics in the same pass; the last CTA calibrates eta_d (Eq. 8),
+//    decays R and inserts the record (section "Reliability Decision").
+//  * stats pass  (state reset/set): statistics of the current latent and the
+//    anchor.
+//
+// Summary statistics: because the summary's latent blocks are a linear sketch
+// S of RMS-normalised vectors, S(nu(z)) = S(z)/(rms(z)+eps_nu) and
+// S(nu(z - z_a)) = (S(z) - S(z_a))/(rms(z - z_a)+eps_nu); a pass therefore
+// reduces raw signed bucket sums and sums of squares, never a normalised copy.
+// The sketch assigns element i to bucket floor(i/128) mod 120 with sign bit 31
+// of lowbias32(i ^ seed) (C. Wellons' integer hash), so one warp handles one
+// 128-element run = one bucket with 128-bit loads.
+//
+// Reductions are deterministic: per-warp bucket rows in shared memory, fixed-
+// order block combination in fp64, per-block partials, and a last-block-done
+// final reduction in fixed order.  No kernel here waits on another CTA.
+#include "wdc_internal.h"
+
+#include <cmath>
+
+namespace wdc {
+
+namespace {
+
+constexpr int kThreads = 1024;
+constexpr int kWarps = kThreads / 32;
+
+__device__ __forceinline__ uint32_t lowbias32(uint32_t x) {
+    x ^= x >> 16;
+    x *= 0x7feb352du;
+    x ^= x >> 15;
+    x *= 0x846ca68bu;
+    x ^= x >> 16;
+    return x;
+}
+
+// sign(i) * x: flips the sign bit of x when bit 31 of the hash is set.
+__device__ __forceinline__ float signed_term(uint32_t idx, uint32_t seed, float x) {
+    uint32_t h = lowbias32(idx ^ seed) & 0x80000000u;
+    return __int_as_float(__float_as_int(x) ^ (int)h);
+}
+
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ double warp_sum_d(double v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Sum NV values over the first 256 threads (8 warps) in fixed order; result in
+// out[0..NV) (shared).  Every thread of the block must call it.
+template <int NV>
+__device__ __forceinline__ void reduce256(double (&v)[NV], double* scratch, double* out) {
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) v[j] = warp_sum_d(v[j]);
+    if (lane == 0 && w < 8) {
+#pragma unroll
+        for (int j = 0; j < NV; ++j) scratch[w * NV + j] = v[j];
+    }
+    __syncthreads();
+    if (t < NV) {
+        double s = 0.0;
+        for (int q = 0; q < 8; ++q) s += scratch[q * NV + t];
+        out[t] = s;
+    }
+    __syncthreads();
+}
+
+struct HeadShared {
+    double phi[kSummary];
+    double hat[kSummary];
+    double scratch[8 * (kMaxBank + 1)];
+    double red[kMaxBank + 1];
+    double sim_in[kMaxBank], sim_out[kMaxBank], pi[kMaxBank], kappa[kMaxBank];
+    double alpha;
+    int compat[kMaxBank];
+    int n_compat, supported;
+};
+
+// Skip-pass head (every CTA, redundantly): Eq. 2-5 scalar part.
+template <int K>
+__device__ void skip_head(const PassArgs& a, HeadShared& hs) {
+    const DevState* st = a.st;
+    const int t = threadIdx.x;
+    const double N = (double)a.n;
+    const double sc = sqrt((double)kSketch / N);
+    // s(phi_k): current-state summary (Eq. 2 through the linear sketch)
+    if (t < kSummary) {
+        double val;
+        if (t < kSketch) {
+            val = sc * st->cur_S[t] / (sqrt(st->cur_sumsq / N) + a.prm.eps_nu);
+        } else if (t < 2 * kSketch) {
+            const int b = t - kSketch;
+            val = sc * (st->cur_S[b] - st->anchor_S[b]) / (sqrt(st->cur_sumsq_anchor / N) + a.prm.eps_nu);
+        } else if (t < kOffDepth) {
+            val = a.cam[t - kOffCam];
+        } else if (t < kOffQ) {
+            val = a.depth[t - kOffDepth];
+        } else if (t == kOffQ) {
+            val = a.q_k;
+        } else {
+            // h(H): [r_1..3, T*(q_in - q_out)_1..3, n_bank/K], newest record first
+            const int j = t - kOffH;
+            val = 0.0;
+            if (j < 3) {
+                if (j < a.nsrc) val = st->rec[a.slot[a.nsrc - 1 - j]].r;
+            } else if (j < 6) {
+                if (j - 3 < a.nsrc) {
+                    const DevRecord& r = st->rec[a.slot[a.nsrc - 1 - (j - 3)]];
+                    val = (double)a.T * (r.q_in - r.q_out);
+                }
+            } else {
+                val = (double)a.nsrc / (double)a.prm.K;
+            }
+        }
+        hs.phi[t] = val;
+    }
+    __syncthreads();
+    if (K == 0) return;
+
+    // Eq. 3: similarities with the records' lifted inputs
+    {
+        double v[K + 1];
+        const double ph = (t < kSummary) ? hs.phi[t] : 0.0;
+#pragma unroll
+        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? ph * st->rec[a.slot[i]].s_in[t] : 0.0;
+        v[K] = ph * ph;
+        reduce256<K + 1>(v, hs.scratch, hs.red);
+    }
+    if (t == 0) {
+        const double nphi = sqrt(hs.red[K]);
+        int nc = 0;
+        double mx = -INFINITY;
+        double ell[K > 0 ? K : 1];
+#pragma unroll
+        for (int i = 0; i < K; ++i) {
+            const DevRecord& r = st->rec[a.slot[i]];
+            const double s = (nphi == 0.0 || r.n_in == 0.0) ? 0.0 : hs.red[i] / (nphi * r.n_in);
+            const double dq = a.q_k - r.q_in;
+            hs.sim_in[i] = s;
+            const int c = (s >= a.prm.sim_min) && (fabs(dq) <= a.prm.q_gap_max);
+            hs.compat[i] = c;
+            ell[i] = (s - a.prm.gamma_q * dq * dq) / a.prm.tau_in;
+            if (c) { ++nc; mx = fmax(mx, ell[i]); }
+        }
+        double tot = 0.0;
+#pragma unroll
+        for (int i = 0; i < K; ++i) {
+            hs.pi[i] = hs.compat[i] ? exp(ell[i] - mx) : 0.0;
+            tot += hs.pi[i];
+        }
+#pragma unroll
+        for (int i = 0; i < K; ++i) hs.pi[i] = (nc > 0) ? hs.pi[i] / tot : 0.0;
+        hs.n_compat = nc;
+        hs.supported = nc >= a.prm.min_support;
+        // Eq. 4: alpha = clip(|q_{t-1}-q_t| / (|q_{a-1}-q_a| + eps), alpha_min, alpha_max)
+        const double raw = fabs(a.q_next - a.q_k) / (fabs(st->q_a_out - st->q_a_in) + a.prm.eps);
+        hs.alpha = fmin(fmax(raw, a.prm.alpha_min), a.prm.alpha_max);
+    }
+    __syncthreads();
+    // Eq. 4 in summary space, then Eq. 5 similarities with the lifted outputs
+    {
+        double v[K + 1];
+        double hv = 0.0;
+        if (t < kSummary) {
+            double acc = 0.0;
+#pragma unroll
+            for (int i = 0; i < K; ++i)
+                if (hs.pi[i] != 0.0) acc += hs.pi[i] * st->rec[a.slot[i]].s_dphi[t];
+            hv = hs.phi[t] + hs.alpha * acc;
+            hs.hat[t] = hv;
+        }
+#pragma unroll
+        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? hv * st->rec[a.slot[i]].s_out[t] : 0.0;
+        v[K] = hv * hv;
+        reduce256<K + 1>(v, hs.scratch, hs.red);
+    }
+    if (t == 0) {
+        const double nh = sqrt(hs.red[K]);
+        double mx = -INFINITY;
+        double e[K > 0 ? K : 1];
+#pragma unroll
+        for (int i = 0; i < K; ++i) {
+            const DevRecord& r = st->rec[a.slot[i]];
+            const double s = (nh == 0.0 || r.n_out == 0.0) ? 0.0 : hs.red[i] / (nh * r.n_out);
+            hs.sim_out[i] = s;
+            e[i] = s / a.prm.tau_obs;
+            mx = fmax(mx, e[i]);
+        }
+        double tot = 0.0;
+#pragma unroll
+        for (int i = 0; i < K; ++i) { e[i] = exp(e[i] - mx); tot += e[i]; }
+#pragma unroll
+        for (int i = 0; i < K; ++i) hs.kappa[i] = e[i] / tot;
+    }
+    __syncthreads();
+}
+
+struct PassShared {
+    float wb[2][kWarps][kSketch];     // per-warp bucket rows (2 sketches for the stats pass)
+    double blk[kWarps][8];
+    double fin[kPartials];
+    int last;
+};
+
+template <int MODE, int K>
+__global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant__ PassArgs a) {
+    __shared__ HeadShared hs;
+    __shared__ PassShared ps;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const uint32_t seed = a.prm.seed;
+    const long long n = a.n;
+    const long long nruns = (n + kRun - 1) / kRun;
+    const long long full = n / kRun;
+
+    for (int i = t; i < 2 * kWarps * kSketch; i += kThreads) (&ps.wb[0][0][0])[i] = 0.f;
+
+    bool do_stream = true;
+    float kap[K > 0 ? K : 1];
+    if (MODE == kModeSkip) {
+        skip_head<K>(a, hs);
+        do_stream = (K > 0) && hs.supported;
+#pragma unroll
+        for (int i = 0; i < K; ++i) kap[i] = (float)hs.kappa[i];
+    } else {
+        __syncthreads();
+    }
+
+    // per-thread accumulators: fp32 over up to 16 runs, flushed to fp64
+    double acc[5] = {0, 0, 0, 0, 0};
+    float fac[5] = {0, 0, 0, 0, 0};
+    int nonfinite = 0;
+    int since = 0;
+    const float dsig = a.dsig;
+
+    if (do_stream) {
+        const long long gw = (long long)blockIdx.x * kWarps + warp;
+        const long long stride = (long long)gridDim.x * kWarps;
+        for (long long r = gw; r < nruns; r += stride) {
+            const long long base = r * kRun + lane * 4;
+            float o[4], sa[4], sb[4];   // o: primary value, sa/sb: stats-pass anchor
+            bool valid[4];
+            if (r < full) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) valid[e] = true;
+                if constexpr (MODE == kModeSkip && K > 0) {
+                    float4 x[K];
+#pragma unroll
+                    for (int i = 0; i < K; ++i) x[i] = __ldg(reinterpret_cast<const float4*>(a.src[i] + base));
+                    float4 zh;
+                    zh.x = kap[0] * x[0].x; zh.y = kap[0] * x[0].y; zh.z = kap[0] * x[0].z; zh.w = kap[0] * x[0].w;
+#pragma unroll
+                    for (int i = 1; i < K; ++i) {
+                        zh.x = fmaf(kap[i], x[i].x, zh.x); zh.y = fmaf(kap[i], x[i].y, zh.y);
+                        zh.z = fmaf(kap[i], x[i].z, zh.z); zh.w = fmaf(kap[i], x[i].w, zh.w);
+                    }
+                    *reinterpret_cast<float4*>(a.out + base) = zh;
+                    o[0] = zh.x; o[1] = zh.y; o[2] = zh.z; o[3] = zh.w;
+                    sa[0] = x[K - 1].x; sa[1] = x[K - 1].y; sa[2] = x[K - 1].z; sa[3] = x[K - 1].w;
+                } else if constexpr (MODE == kModeAnchor) {
+                    // plain loads: z_k / z_a may alias the slot written below (bank capacity 1)
+                    const float4 z = *reinterpret_cast<const float4*>(a.src[0] + base);
+                    const float4 v = *reinterpret_cast<const float4*>(a.v + base);
+                    const float4 za = *reinterpret_cast<const float4*>(a.anchor + base);
+                    float4 ze;
+                    ze.x = fmaf(dsig, v.x, z.x); ze.y = fmaf(dsig, v.y, z.y);
+                    ze.z = fmaf(dsig, v.z, z.z); ze.w = fmaf(dsig, v.w, z.w);
+                    *reinterpret_cast<float4*>(a.out + base) = ze;
+                    o[0] = ze.x; o[1] = ze.y; o[2] = ze.z; o[3] = ze.w;
+                    sa[0] = za.x; sa[1] = za.y; sa[2] = za.z; sa[3] = za.w;
+                    sb[0] = z.x; sb[1] = z.y; sb[2] = z.z; sb[3] = z.w;
+                    if (a.zcf) {
+                        const float4 c = *reinterpret_cast<const float4*>(a.zcf + base);
+                        fac[0] += fabsf(ze.x - c.x) + fabsf(ze.y - c.y) + fabsf(ze.z - c.z) + fabsf(ze.w - c.w);
+                    }
+                } else if constexpr (MODE == kModeStats) {
+                    const float4 z = __ldg(reinterpret_cast<const float4*>(a.src[0] + base));
+                    const float4 za = __ldg(reinterpret_cast<const float4*>(a.anchor + base));
+                    o[0] = z.x; o[1] = z.y; o[2] = z.z; o[3] = z.w;
+                    sa[0] = za.x; sa[1] = za.y; sa[2] = za.z; sa[3] = za.w;
+                }
+            } else {
+                // ragged last run: scalar, bounds-checked
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const long long idx = base + e;
+                    valid[e] = idx < n;
+                    o[e] = 0.f; sa[e] = 0.f; sb[e] = 0.f;
+                    if (!valid[e]) continue;
+                    if constexpr (MODE == kModeSkip && K > 0) {
+                        float zh = kap[0] * a.src[0][idx];
+#pragma unroll
+                        for (int i = 1; i < K; ++i) zh = fmaf(kap[i], a.src[i][idx], zh);
+                        a.out[idx] = zh;
+                        o[e] = zh;
+                        sa[e] = a.src[K - 1][idx];
+                    } else if constexpr (MODE == kModeAnchor) {
+                        const float z = a.src[0][idx];
+                        const float ze = fmaf(dsig, a.v[idx], z);
+                        a.out[idx] = ze;
+                        o[e] = ze;
+                        sa[e] = a.anchor[idx];
+                        sb[e] = z;
+                        if (a.zcf) fac[0] += fabsf(ze - a.zcf[idx]);
+                    } else if constexpr (MODE == kModeStats) {
+                        o[e] = a.src[0][idx];
+                        sa[e] = a.anchor[idx];
+                    }
+                }
+            }
+            // statistics of the primary value
+            float sg = 0.f, sg2 = 0.f;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                if (!valid[e]) continue;
+                const float x = o[e];
+                const float d = x - sa[e];
+                const uint32_t idx = (uint32_t)(base + e);
+                sg += signed_term(idx, seed, x);
+                if (MODE == kModeSkip) {
+                    fac[0] += x * x;
+                    fac[1] += d * d;
+                    nonfinite += isfinite(x) ? 0 : 1;
+                } else if (MODE == kModeAnchor) {
+                    fac[1] += fabsf(x);
+                    fac[2] += x * x;
+                    fac[3] += d * d;
+                    const float dz = x - sb[e];
+                    fac[4] += dz * dz;
+                } else {
+                    fac[0] += x * x;
+                    fac[1] += d * d;
+                    fac[2] += sa[e] * sa[e];
+                    sg2 += signed_term(idx, seed, sa[e]);
+                }
+            }
+            sg = warp_sum_f(sg);
+            const int bucket = (int)(r % kSketch);
+            if (lane == 0) ps.wb[0][warp][bucket] += sg;
+            if (MODE == kModeStats) {
+                sg2 = warp_sum_f(sg2);
+                if (lane == 0) ps.wb[1][warp][bucket] += sg2;
+            }
+            if (++since == 16) {
+#pragma unroll
+                for (int j = 0; j < 5; ++j) { acc[j] += (double)fac[j]; fac[j] = 0.f; }
+                since = 0;
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 5; ++j) acc[j] += (double)fac[j];
+    double cnt = (double)nonfinite;
+
+    // block combination (fixed order)
+#pragma unroll
+    for (int j = 0; j < 5; ++j) acc[j] = warp_sum_d(acc[j]);
+    cnt = warp_sum_d(cnt);
+    if (lane == 0) {
+#pragma unroll
+        for (int j = 0; j < 5; ++j) ps.blk[warp][j] = acc[j];
+        ps.blk[warp][5] = cnt;
+    }
+    __syncthreads();
+    double* part = a.partials + (size_t)blockIdx.x * kPartials;
+    if (t < 2 * kSketch) {
+        const int s = t / kSketch, b = t % kSketch;
+        double v = 0.0;
+        for (int w = 0; w < kWarps; ++w) v += (double)ps.wb[s][w][b];
+        part[t] = v;
+    } else if (t < 2 * kSketch + 6) {
+        const int j = t - 2 * kSketch;
+        double v = 0.0;
+        for (int w = 0; w < kWarps; ++w) v += ps.blk[w][j];
+        part[t] = v;
+    }
+    __threadfence();
+    __syncthreads();
+    if (t == 0) {
+        const unsigned prev = atomicAdd(a.counter, 1u);
+        ps.last = (prev == gridDim.x - 1);
+    }
+    __syncthreads();
+    if (!ps.last) return;
+    __threadfence();
+
+    // final reduction over blocks, fixed order: 4 threads per value
+    {
+        // the per-warp bucket rows are no longer needed: reuse them as scratch
+        double (*tmp)[kPartials] = reinterpret_cast<double (*)[kPartials]>(&ps.wb[0][0][0]);
+        const int v = t % 256, g = t / 256;
+        if (v < 2 * kSketch + 6) {
+            double s = 0.0;
+            for (int b = g; b < (int)gridDim.x; b += 4) s += __ldcg(a.partials + (size_t)b * kPartials + v);
+            tmp[g][v] = s;
+        }
+        __syncthreads();
+        if (t < 2 * kSketch + 6) ps.fin[t] = ((tmp[0][t] + tmp[1][t]) + tmp[2][t]) + tmp[3][t];
+        __syncthreads();
+    }
+    if (t == 0) *a.counter = 0u;
+
+    DevState* st = a.st;
+    const double N = (double)n;
+    const double* fin = ps.fin;
+    const int sc0 = 2 * kSketch;   // scalar sums start here
+
+    if (MODE == kModeStats) {
+        if (t < kSketch) {
+            st->cur_S[t] = fin[t];
+            st->anchor_S[t] = fin[kSketch + t];
+        }
+        if (t == 0) {
+            st->cur_sumsq = fin[sc0 + 0];
+            st->cur_sumsq_anchor = fin[sc0 + 1];
+            st->anchor_sumsq = fin[sc0 + 2];
+        }
+        return;
+    }
+
+    if (MODE == kModeSkip) {
+        if (t < kSummary) st->s_phi[t] = hs.phi[t];
+        const int supported = (K > 0) && hs.supported;
+        const int finite = supported && (fin[sc0 + 5] == 0.0);
+        __shared__ int s_dec;
+        if (t == 0) {
+            const ParamsDev& p = a.prm;
+            const double d_z = sqrt(st->cur_sumsq_anchor / N) / (sqrt(st->anchor_sumsq / N) + p.eps);
+            const double d_age = (double)a.age;
+            const double d_phase = fabs(a.q_next - st->q_a_out);
+            double dc = 0.0, dd = 0.0, uc = 0.0, ud = 0.0;
+            for (int j = 0; j < 4; ++j) {
+                dc += (a.cam[j] - st->cam_a[j]) * (a.cam[j] - st->cam_a[j]);
+                dd += (a.depth[j] - st->depth_a[j]) * (a.depth[j] - st->depth_a[j]);
+                uc += a.cam[j] * a.cam[j];
+                ud += a.depth[j] * a.depth[j];
+            }
+            const double pt = p.w_z * d_z + p.w_age * d_age + p.w_phase * d_phase + p.w_cam * sqrt(dc) +
+                              p.w_depth * sqrt(dd);
+            const double d_hat = st->eta * pt;
+            const double w = fmin(2.0, 1.0 + p.a_cam * sqrt(uc) + p.a_depth * sqrt(ud) + p.a_phase * a.q_k);
+            const double delta = w * d_hat;
+            const double R_cand = p.lam * st->R + delta;
+            const bool avail = (a.nsrc > 0) && (a.age <= p.max_age) &&
+                               (fabs(a.q_k - st->q_a_out) <= p.q_gap_max) && finite && supported &&
+                               (a.k >= p.n_init_exact) && (a.k < a.T - p.n_final_exact);
+            const int dec = (avail && R_cand <= p.tau_risk) ? 1 : 0;
+            StepOut& o = st->out;
+            o.decision = dec;
+            o.finite = finite;
+            o.supported = supported;
+            o.n_compat = (K > 0) ? hs.n_compat : 0;
+            o.q = a.q_k;
+            o.alpha = (K > 0) ? hs.alpha : 0.0;
+            o.p = pt;
+            o.d_hat = d_hat;
+            o.w = w;
+            o.delta = delta;
+            o.R_cand = R_cand;
+            o.d_cf = nan("");
+            o.d_z = d_z;
+            o.r = 0.0;
+            for (int i = 0; i < kMaxBank; ++i) {
+                o.kappa[i] = (i < K) ? hs.kappa[i] : 0.0;
+                o.pi[i] = (i < K) ? hs.pi[i] : 0.0;
+            }
+            if (dec) st->R = R_cand;
+            o.R = st->R;
+            o.eta = st->eta;
+            st->cand_k = a.k;
+            st->cand_supported = supported;
+            st->cand_finite = finite;
+            st->cand_p = pt;
+            st->cand_sumsq = fin[sc0 + 0];
+            st->cand_sumsq_anchor = fin[sc0 + 1];
+            s_dec = dec;
+        }
+        __syncthreads();
+        if (t < kSketch) {
+            st->cand_S[t] = fin[t];
+            if (s_dec) st->cur_S[t] = fin[t];
+        }
+        if (t == 0 && s_dec) {
+            st->cur_sumsq = fin[sc0 + 0];
+            st->cur_sumsq_anchor = fin[sc0 + 1];
+        }
+        return;
+    }
+
+    // ---- anchor pass tail (MODE == kModeAnchor)
+    __shared__ double s_rms[2];
+    if (t == 0) {
+        const ParamsDev& p = a.prm;
+        st->R = p.lam * st->R;
+        double d_cf = nan("");
+        if (a.zcf != nullptr && st->cand_k == a.k && st->cand_supported && st->cand_finite) {
+            d_cf = (fin[sc0 + 0] / N) / (fin[sc0 + 1] / N + p.eps);
+            const double v = p.beta_d * st->eta + (1.0 - p.beta_d) * d_cf / (st->cand_p + p.eps);
+            st->eta = fmin(fmax(v, p.eta_min), p.eta_max);
+        }
+        st->out.d_cf = d_cf;
+        st->out.R = st->R;
+        st->out.eta = st->eta;
+        const double r = sqrt(fin[sc0 + 4] / N) / (sqrt(st->cur_sumsq / N) + p.eps);
+        st->out.r = r;
+        st->rec[a.ins_slot].r = r;
+        s_rms[0] = sqrt(fin[sc0 + 2] / N);
+        s_rms[1] = sqrt(fin[sc0 + 3] / N);
+    }
+    __syncthreads();
+    DevRecord& rec = st->rec[a.ins_slot];
+    const double sc = sqrt((double)kSketch / N);
+    double so = 0.0, si = 0.0;
+    if (t < kSummary) {
+        if (t < kSketch) {
+            so = sc * fin[t] / (s_rms[0] + a.prm.eps_nu);
+        } else if (t < 2 * kSketch) {
+            const int b = t - kSketch;
+            so = sc * (fin[b] - st->anchor_S[b]) / (s_rms[1] + a.prm.eps_nu);
+        } else if (t < kOffDepth) {
+            so = a.cam[t - kOffCam];
+        } else if (t < kOffQ) {
+            so = a.depth[t - kOffDepth];
+        } else if (t == kOffQ) {
+            so = a.q_next;
+        } else {
+            so = st->s_phi[t];     // pre-insertion history h(H)
+        }
+        si = st->s_phi[t];
+    }
+    __syncthreads();               // everyone has read anchor_S and s_phi
+    if (t < kSummary) {
+        rec.s_in[t] = si;
+        rec.s_out[t] = so;
+        rec.s_dphi[t] = so - si;
+    }
+    {
+        double v[2] = {si * si, so * so};
+        reduce256<2>(v, hs.scratch, hs.red);
+    }
+    if (t < kSketch) {
+        st->anchor_S[t] = fin[t];
+        st->cur_S[t] = fin[t];
+    }
+    if (t == 0) {
+        rec.n_in = sqrt(hs.red[0]);
+        rec.n_out = sqrt(hs.red[1]);
+        rec.q_in = a.q_k;
+        rec.q_out = a.q_next;
+        for (int j = 0; j < 4; ++j) {
+            rec.cam[j] = a.cam[j];
+            rec.depth[j] = a.depth[j];
+            st->cam_a[j] = a.cam[j];
+            st->depth_a[j] = a.depth[j];
+        }
+        st->anchor_sumsq = fin[sc0 + 2];
+        st->cur_sumsq = fin[sc0 + 2];
+        st->cur_sumsq_anchor = 0.0;
+        st->q_a_in = a.q_k;
+        st->q_a_out = a.q_next;
+    }
+}
+
+template <int K>
+void launch_skip(const PassArgs& a, int grid, cudaStream_t s) {
+    pass_kernel<kModeSkip, K><<<grid, kThreads, 0, s>>>(a);
+}
+
+}  // namespace
+
+int pass_grid(const Ctx* c) {
+    const long long nruns = ((long long)c->n + kRun - 1) / kRun;
+    long long g = (nruns + kWarps - 1) / kWarps;
+    if (g > c->num_sms) g = c->num_sms;
+    if (g < 1) g = 1;
+    return (int)g;
+}
+
+wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s) {
+    const int grid = pass_grid(c);
+    switch (mode) {
+        case kModeStats: pass_kernel<kModeStats, 0><<<grid, kThreads, 0, s>>>(a); break;
+        case kModeAnchor: pass_kernel<kModeAnchor, 0><<<grid, kThreads, 0, s>>>(a); break;
+        case kModeSkip:
+            switch (a.nsrc) {
+                case 0: launch_skip<0>(a, grid, s); break;
+                case 1: launch_skip<1>(a, grid, s); break;
+                case 2: launch_skip<2>(a, grid, s); break;
+                case 3: launch_skip<3>(a, grid, s); break;
+                case 4: launch_skip<4>(a, grid, s); break;
+                case 5: launch_skip<5>(a, grid, s); break;
+                case 6: launch_skip<6>(a, grid, s); break;
+                case 7: launch_skip<7>(a, grid, s); break;
+                case 8: launch_skip<8>(a, grid, s); break;
+                default: return fail(c, WDC_ERR_INVALID_ARG, "bank size out of range");
+            }
+            break;
+        default: return fail(c, WDC_ERR_INVALID_ARG, "unknown pass mode");
+    }
+    c->launches += 1;
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("latent pass launch: ") + cudaGetErrorString(e));
+    return WDC_OK;
+}
+
+ParamsDev to_dev_params(const wdc_cache_params& p) {
+    ParamsDev d;
+    d.K = p.bank_capacity;
+    d.min_support = p.min_support;
+    d.max_age = p.max_age;
+    d.n_init_exact = p.n_init_exact;
+    d.n_final_exact = p.n_final_exact;
+    d.seed = p.sketch_seed;
+    d.sim_min = p.sim_min;
+    d.q_gap_max = p.q_gap_max;
+    d.gamma_q = p.gamma_q;
+    d.tau_in = p.tau_in;
+    d.tau_obs = p.tau_obs;
+    d.alpha_min = p.alpha_min;
+    d.alpha_max = p.alpha_max;
+    d.eps = p.eps;
+    d.eps_nu = p.eps_nu;
+    d.w_z = p.w_z;
+    d.w_age = p.w_age;
+    d.w_phase = p.w_phase;
+    d.w_cam = p.w_cam;
+    d.w_depth = p.w_depth;
+    d.eta_min = p.eta_min;
+    d.eta_max = p.eta_max;
+    d.beta_d = p.beta_d;
+    d.a_cam = p.a_cam;
+    d.a_depth = p.a_depth;
+    d.a_phase = p.a_phase;
+    d.lam = p.lambda_;
+    d.tau_risk = p.tau_risk;
+    return d;
+}
+
+}  // namespace wdc

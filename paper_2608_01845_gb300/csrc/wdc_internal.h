@@ -1,0 +1,155 @@
+// Internal declarations shared by the libwdc translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+#include <cstddef>
+#include <string>
+#include <vector>
+
+#include "../../include/wdc.h"
+
+namespace wdc {
+
+constexpr int kSketch = WDC_SKETCH;          // 120 buckets per latent block
+constexpr int kRun = 128;                    // elements per sketch run
+constexpr int kSummary = WDC_SUMMARY_DIM;    // 256
+constexpr int kMaxBank = WDC_MAX_BANK;
+constexpr int kOffDz = kSketch;              // offsets inside a summary vector
+constexpr int kOffCam = 2 * kSketch;
+constexpr int kOffDepth = kOffCam + 4;
+constexpr int kOffQ = kOffDepth + 4;
+constexpr int kOffH = kOffQ + 1;
+
+// Error bits written by kernels into the context's device error word.
+enum : unsigned { kErrTimeout = 1u, kErrBounds = 2u, kErrTmem = 4u };
+
+// ---------------------------------------------------------------- device state
+// One bank record; summaries in fp64 (section "Local Lifted Evolution").
+struct DevRecord {
+    double s_in[kSummary], s_out[kSummary], s_dphi[kSummary];
+    double n_in, n_out;           // Euclidean norms of s_in and s_out
+    double q_in, q_out, r;
+    double cam[4], depth[4];
+};
+
+// Per-step output mirrored to the host.
+struct StepOut {
+    int decision, finite, supported, n_compat;
+    double q, alpha, p, d_hat, w, delta, R_cand, R, eta, d_cf, d_z, r;
+    double kappa[kMaxBank], pi[kMaxBank];
+};
+
+// Continuous controller/memory state (discrete state -- bank ring, age -- is
+// owned by the host and passed per launch).
+struct DevState {
+    double R, eta;
+    double q_a_in, q_a_out;
+    double cam_a[4], depth_a[4];
+    DevRecord rec[kMaxBank];                       // indexed by ring slot
+    double cur_S[kSketch], cur_sumsq, cur_sumsq_anchor;   // raw sums over the current latent
+    double anchor_S[kSketch], anchor_sumsq;
+    double s_phi[kSummary];                        // summary of the current state (this step)
+    int cand_k, cand_supported, cand_finite;
+    double cand_p;
+    double cand_S[kSketch], cand_sumsq, cand_sumsq_anchor;
+    StepOut out;
+};
+
+struct ParamsDev {
+    int K, min_support, max_age, n_init_exact, n_final_exact;
+    unsigned seed;
+    double sim_min, q_gap_max, gamma_q, tau_in, tau_obs, alpha_min, alpha_max, eps, eps_nu;
+    double w_z, w_age, w_phase, w_cam, w_depth, eta_min, eta_max, beta_d;
+    double a_cam, a_depth, a_phase, lam, tau_risk;
+};
+
+enum StreamMode { kModeStats = 0, kModeSkip = 1, kModeAnchor = 2 };
+
+// Launch arguments of the fused latent-pass kernels (passed by value).
+struct PassArgs {
+    long long n;
+    int nsrc;                          // skip: records in age order (oldest first)
+    const float* src[kMaxBank];        // skip: bank latents by age; anchor/stats: src[0] = z_k
+    int slot[kMaxBank];                // ring slot of each record, by age
+    const float* anchor;               // z_a
+    const float* v;                    // anchor: velocity
+    const float* zcf;                  // anchor: counterfactual candidate or nullptr
+    float* out;                        // skip: z_hat; anchor: z_exact (bank slot)
+    float dsig;                        // anchor: sigma_{k+1} - sigma_k (fp32)
+    int k, T, age, ins_slot;
+    double q_k, q_next;
+    double cam[4], depth[4];
+    ParamsDev prm;
+    DevState* st;
+    double* partials;                  // [gridDim.x][kPartials]
+    unsigned* counter;
+    unsigned* err;
+};
+
+// ---------------------------------------------------------------- context
+struct Ctx {
+    wdc_dit_config cfg{};
+    wdc_schedule sched{};
+    wdc_cache_params prm{};
+    int device = 0;
+    int num_sms = 0;
+    size_t n = 0;                      // latent numel
+    std::vector<double> sigma;         // T+1 noise levels (host, fp64)
+    std::string last_error;
+    unsigned long long launches = 0;
+
+    // memory
+    DevState* st = nullptr;
+    double* partials = nullptr;
+    unsigned* counter = nullptr;
+    unsigned* err = nullptr;
+    StepOut* out_host = nullptr;       // pinned
+    float* bank[kMaxBank] = {};
+    float* z_init = nullptr;           // anchor before the first exact step
+    float* cand[2] = {};               // rollout candidate buffers
+    float* vbuf = nullptr;
+    float* zstage = nullptr;           // host-pointer staging for rollouts
+
+    // host mirror of the discrete state
+    int n_bank = 0, head = 0, age = 0;
+    int last_surrogate_k = -1;
+    int anchor_is_init = 1;
+
+    // denoiser
+    struct DiT* dit = nullptr;
+};
+
+// ---------------------------------------------------------------- helpers
+#define WDC_CUDA_TRY(ctx, call)                                                   \
+    do {                                                                          \
+        cudaError_t e__ = (call);                                                 \
+        if (e__ != cudaSuccess) {                                                 \
+            (ctx)->last_error = std::string(#call) + ": " + cudaGetErrorString(e__); \
+            return e__ == cudaErrorMemoryAllocation ? WDC_ERR_OOM : WDC_ERR_CUDA; \
+        }                                                                         \
+    } while (0)
+
+wdc_status fail(Ctx* c, wdc_status s, const std::string& msg);
+
+// step_kernels.cu
+constexpr int kPartials = 2 * kSketch + 8;     // per-block partial sums
+int pass_grid(const Ctx* c);
+wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s);
+ParamsDev to_dev_params(const wdc_cache_params& p);
+
+// dit.cu
+wdc_status dit_create(Ctx* c);
+void dit_destroy(Ctx* c);
+wdc_status dit_set_tensor(Ctx* c, int id, int layer, int stream, const float* host, size_t count);
+wdc_status dit_init_weights(Ctx* c, unsigned long long seed, float std);
+wdc_status dit_forward(Ctx* c, const float* z, float t, const float* cond, float* v, cudaStream_t s);
+wdc_status dit_block(Ctx* c, int layer, void* x, const float* mod6, cudaStream_t s);
+wdc_status dit_modulation(Ctx* c, float t, float* mod_out, cudaStream_t s);
+wdc_status op_gemm(Ctx* c, const void* A, const void* W, const float* bias, void* C, int M, int N, int K,
+                   int gelu, const void* res, const float* gate, cudaStream_t s);
+wdc_status op_attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int heads, int L,
+                        int d, cudaStream_t s);
+
+}  // namespace wdc

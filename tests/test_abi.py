@@ -1,0 +1,40 @@
+"""The C-ABI library loads and exports every entry point include/wdc.h declares
+(no compute call: this runs without a GPU)."""
+import ctypes
+import os
+import re
+
+from paper_2608_01845_gb300 import wdc
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "wdc.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(wdc_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for required in ["wdc_dit_forward", "wdc_scheduler_step", "wdc_surrogate_step", "wdc_risk_update", "wdc_rollout"]:
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol():
+    lib = ctypes.CDLL(wdc.LIB_PATH)
+    missing = [n for n in _declared() if not hasattr(lib, n)]
+    assert missing == []
+
+
+def test_default_params_and_status_strings():
+    p = wdc.default_params()
+    assert p.bank_capacity == 4 and p.max_age == 6 and p.flags == 0
+    assert wdc.LIB.wdc_status_string(0) == b"ok"
+    assert wdc.LIB.wdc_status_string(6) == b"call out of order"
+
+
+def test_struct_sizes_match_the_header_layout():
+    # wdc_step_info: 7 ints, pad to 8-byte alignment, 12 doubles, 2 x 8 doubles
+    assert ctypes.sizeof(wdc.StepInfo) == 8 * 4 + 12 * 8 + 16 * 8
+    assert ctypes.sizeof(wdc.Cond) == 8 + 8 * 8

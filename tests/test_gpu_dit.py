@@ -1,0 +1,146 @@
+"""Parity of the denoiser F_theta's CUDA kernels with the CPU checker.
+
+fp32 mode: full forward of the 2-layer D=256 model (and a dual-stream
+variant), rel L2 <= 1e-5 against fp64.  bf16 mode: the GEMM and attention
+operators on shapes spanning several tiles with ragged tails, and one block of
+the 5B-scale model (L = 17776, D = 3072, 48 x 64 heads) on 256 sampled query
+rows; rel L2 <= 2e-2 (bf16 operands, fp32 accumulation) against fp64."""
+import numpy as np
+import pytest
+import torch
+
+from helpers import rel_l2
+from oracle import dit
+from oracle.params import DiTConfig
+from paper_2608_01845_gb300 import synth, wdc
+
+pytestmark = pytest.mark.gpu
+BF16_TOL = 2e-2
+
+CFG0 = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
+            height=16, width=16, patch=2, cond_tokens=16, cond_dim=256, dual_stream=0)
+
+
+def _ctx(cfgd, dtype, T=10):
+    cfg = wdc.make_config(dtype=dtype, **cfgd)
+    return wdc.Context(cfg, T)
+
+
+def _to_dev(a, dtype=torch.float32):
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).cuda().to(dtype)
+
+
+@pytest.mark.parametrize("dual", [0, 1])
+def test_fp32_forward_matches_oracle(dual):
+    cfgd = dict(CFG0, dual_stream=dual, layers=2 if not dual else 1)
+    W = synth.dit_weights(cfgd, 7, std=0.02, bias_std=0.02)
+    ctx = _ctx(cfgd, wdc.F32)
+    ctx.set_weights(W)
+    z = synth.latent(3, (16, 4, 16, 16))
+    ct = synth.cond_tokens(4, 16, 256)
+    v = torch.empty(z.size, dtype=torch.float32, device="cuda")
+    ctx.dit_forward(_to_dev(z), 731.0, _to_dev(ct), v)
+    torch.cuda.synchronize()
+    want = dit.forward(W, DiTConfig(**cfgd), z, 731.0, ct)
+    assert rel_l2(v.cpu().numpy(), want) <= 1e-5
+
+
+def test_fp32_modulation_matches_oracle():
+    W = synth.dit_weights(CFG0, 8, std=0.05, bias_std=0.02)
+    ctx = _ctx(CFG0, wdc.F32)
+    ctx.set_weights(W)
+    D = 256
+    out = torch.empty(2 * 6 * D + 2 * D, dtype=torch.float32, device="cuda")
+    ctx.dit_modulation(250.0, out)
+    torch.cuda.synchronize()
+    _, mods, fm = dit.conditioning(W, DiTConfig(**CFG0), 250.0)
+    want = np.concatenate([mods[(0, 0)].ravel(), mods[(1, 0)].ravel(), fm.ravel()])
+    assert rel_l2(out.cpu().numpy(), want) <= 1e-5
+
+
+def _bf(a):
+    return synth.bf16_round(np.asarray(a, dtype=np.float32))
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 384, 320), (128, 256, 64), (1000, 768, 1024), (17, 64, 128)])
+@pytest.mark.parametrize("mode", ["store", "gelu", "resid"])
+def test_bf16_gemm_matches_oracle(M, N, K, mode):
+    ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
+    A = _bf(synth.normal(1, (M, K)))
+    W = _bf(synth.normal(2, (N, K), 0.05))
+    b = synth.normal(3, (N,), 0.1)
+    acc = A.astype(np.float64) @ W.astype(np.float64).T + b
+    C = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    kw = {}
+    if mode == "gelu":
+        kw["gelu"] = True
+        want = dit.gelu_tanh(acc)
+    elif mode == "resid":
+        R = _bf(synth.normal(4, (M, N)))
+        g = synth.normal(5, (N,), 1.0)
+        Rt = _to_dev(R, torch.bfloat16)
+        C = Rt                                      # in place, as in the block
+        kw.update(res=Rt, gate=_to_dev(g))
+        want = R.astype(np.float64) + g * acc
+    else:
+        want = acc
+    ctx.op_gemm(_to_dev(A, torch.bfloat16), _to_dev(W, torch.bfloat16), C, bias=_to_dev(b), **kw)
+    torch.cuda.synchronize()
+    assert rel_l2(C.float().cpu().numpy(), want) <= 1e-2
+
+
+@pytest.mark.parametrize("H,L,d", [(2, 300, 64), (1, 1000, 128), (3, 129, 64), (1, 64, 128)])
+def test_bf16_attention_matches_oracle(H, L, d):
+    ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
+    q = _bf(synth.normal(11, (H, L, d)))
+    k = _bf(synth.normal(12, (H, L, d)))
+    v = _bf(synth.normal(13, (H, L, d)))
+    o = torch.empty(L, H * d, dtype=torch.bfloat16, device="cuda")
+    ctx.op_attention(_to_dev(q, torch.bfloat16), _to_dev(k, torch.bfloat16),
+                     _to_dev(np.ascontiguousarray(v.transpose(0, 2, 1)), torch.bfloat16), o)
+    torch.cuda.synchronize()
+    qf = q.transpose(1, 0, 2).reshape(L, H * d).astype(np.float64)
+    kf = k.transpose(1, 0, 2).reshape(L, H * d).astype(np.float64)
+    vf = v.transpose(1, 0, 2).reshape(L, H * d).astype(np.float64)
+    want = dit.attention(qf, kf, vf, H)
+    assert rel_l2(o.float().cpu().numpy(), want) <= 1e-2
+
+
+@pytest.mark.parametrize("H,L,d", [(2, 300, 64), (2, 257, 128)])
+def test_fp32_attention_matches_oracle(H, L, d):
+    ctx = _ctx(dict(CFG0, layers=1), wdc.F32)
+    q, k, v = (synth.normal(s, (H, L, d)) for s in (21, 22, 23))
+    o = torch.empty(L, H * d, dtype=torch.float32, device="cuda")
+    ctx.op_attention(_to_dev(q), _to_dev(k), _to_dev(np.ascontiguousarray(v.transpose(0, 2, 1))), o)
+    torch.cuda.synchronize()
+    f = lambda a: a.transpose(1, 0, 2).reshape(L, H * d).astype(np.float64)
+    assert rel_l2(o.cpu().numpy(), dit.attention(f(q), f(k), f(v), H)) <= 1e-5
+
+
+BLOCK5B = dict(layers=1, hidden=3072, heads=48, head_dim=64, mlp=12288, temb_dim=512, freq_dim=256, in_ch=16,
+               frames=13, height=60, width=90, patch=2, cond_tokens=226, cond_dim=3072, dual_stream=0)
+
+
+def test_bf16_block_5b_scale_sampled_rows():
+    """One block at the Aether-5B-like shape (L = 226 + 17550 = 17776 tokens),
+    compared on 256 seeded rows (keys/values for all rows on the CPU)."""
+    cfgd = BLOCK5B
+    ctx = _ctx(cfgd, wdc.BF16)
+    names = [f"L0.s0.{n}" for n in ["qkv.w", "qkv.b", "o.w", "o.b", "fc1.w", "fc1.b", "fc2.w", "fc2.b"]]
+    W = synth.dit_weights(cfgd, 5, std=0.02, bias_std=0.02, bf16=True, names=names)
+    ctx.set_weights(W)
+    L, D = 17776, 3072
+    x = _bf(synth.normal(31, (L, D)))
+    mod = synth.normal(32, (6, D), 0.3)
+    mod[2] = 1.0 + mod[2]                         # gates of order one: the block's delta dominates
+    mod[5] = 1.0 + mod[5]
+    xt = _to_dev(x, torch.bfloat16)
+    ctx.dit_block_forward(0, xt, _to_dev(mod))
+    torch.cuda.synchronize()
+    rows = np.sort(np.random.default_rng(33).choice(L, 256, replace=False))
+    got = xt.float().cpu().numpy()[rows]
+    want = dit.block_rows(x.astype(np.float64), W, DiTConfig(**cfgd), 0, [mod.astype(np.float64)], rows)
+    delta_got = got - x[rows]
+    delta_want = want - x[rows]
+    assert rel_l2(delta_got, delta_want) <= BF16_TOL
+    assert rel_l2(got, want) <= BF16_TOL
