@@ -1,8 +1,348 @@
-// tcgen05 flash attention (placeholder until the TMEM kernel lands).
+// Non-causal softmax attention on the tcgen05 tensor cores (sm_103a):
+// O = softmax(Q K^T / sqrt(d)) V per head, joint over all L tokens (the DiT's
+// full spatio-temporal attention).  Q, K [H, L, d], V^T [H, d, L], O [L, H*d],
+// bf16 with fp32 softmax and accumulation; d = 64 or 128.
+//
+// One CTA per (head, 256 query rows), 10 warps:
+//   warp 0      TMA producer: the two 128-row Q tiles once, then K / V^T tiles
+//               of 128 keys into a shared-memory ring (128-byte swizzle);
+//   warp 1      MMA issuer (one thread), ping-pong over the two query tiles:
+//                 PV0(j-1), S0(j), PV1(j-1), S1(j)
+//               S = Q K^T lands in TMEM (128 fp32 columns per tile); the
+//               softmax overwrites its first 64 columns with P (bf16 pairs),
+//               which the PV MMA reads as its A operand from TMEM;
+//   warps 2-5   softmax of query tile 0, warps 6-9 of tile 1 (one thread per
+//               query row = TMEM lane): online max / exp2 / row sum, O
+//               rescaling in TMEM when the running max moves, final 1/l
+//               normalisation and the bf16 store.
+// A commit after S(j) also covers PV(j-1) of the same tile (tcgen05 ops of
+// one thread complete in order), so the softmax may rescale O as soon as S(j)
+// is ready.  Keys past L are masked (TMA zero-fills out-of-range K / V^T).
+// Every mbarrier wait is bounded.
 #include "dit_kernels.cuh"
+#include "ptx.cuh"
+
 namespace wdc {
-bool tc_attention_supported(int, int) { return false; }
-wdc_status tc_attention(Ctx* c, const void*, const void*, const void*, void*, int, int, int, cudaStream_t) {
-    return fail(c, WDC_ERR_UNSUPPORTED, "tcgen05 attention not built");
+
+namespace {
+
+constexpr int kAttnThreads = 320;
+constexpr int BQ = 128;        // query rows per tile (two tiles per CTA)
+constexpr int BKV = 128;       // keys per tile
+
+template <int D>
+struct AttnCfg {
+    static constexpr int ATOMS = D / 64;                    // 128-byte atoms along d
+    static constexpr uint32_t Q_TILE = BQ * D * 2;          // one query tile
+    static constexpr uint32_t K_TILE = BKV * D * 2;
+    static constexpr uint32_t V_TILE = D * BKV * 2;
+    static constexpr uint32_t STAGE = K_TILE + V_TILE;
+    static constexpr int STAGES = D == 64 ? 3 : 2;
+    static constexpr uint32_t SMEM = 2 * Q_TILE + STAGES * STAGE + 1024 + 256;
+    static constexpr uint32_t TMEM_O = 256;                 // O tiles after the two S tiles
+    static constexpr uint32_t TMEM_COLS = 512;
+};
+
+struct AttnArgs {
+    int H, L, n_kv, q_blocks;
+    float scale_log2;
+    __nv_bfloat16* o;
+    unsigned* err;
+};
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
 }
+
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kAttnThreads, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
+                   const __grid_constant__ CUtensorMap tv, const __grid_constant__ AttnArgs g) {
+    using C = AttnCfg<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sq = smem;                                       // [2 tiles][ATOMS][128 x 128 B]
+    uint8_t* skv = smem + 2 * C::Q_TILE;                      // [STAGES][K | V^T]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(skv + C::STAGES * C::STAGE);
+    uint64_t* q_full = bars;
+    uint64_t* kv_full = q_full + 1;
+    uint64_t* kv_empty = kv_full + C::STAGES;
+    uint64_t* s_full = kv_empty + C::STAGES;                  // [2]
+    uint64_t* p_full = s_full + 2;                            // [2]
+    uint64_t* o_final = p_full + 2;                           // [2]
+    uint64_t* mma_done = o_final + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int h = blockIdx.x / g.q_blocks;
+    const int q0 = (blockIdx.x % g.q_blocks) * (2 * BQ);
+    const int n_kv = g.n_kv;
+
+    if (threadIdx.x == 0) {
+        mbar_init(q_full, 1);
+        for (int s = 0; s < C::STAGES; ++s) {
+            mbar_init(&kv_full[s], 1);
+            mbar_init(&kv_empty[s], 1);
+        }
+        for (int w = 0; w < 2; ++w) {
+            mbar_init(&s_full[w], 1);
+            mbar_init(&p_full[w], 4);
+            mbar_init(&o_final[w], 1);
+        }
+        mbar_init(mma_done, 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 0 && lane == 0) {
+        prefetch_tmap(&tq);
+        prefetch_tmap(&tk);
+        prefetch_tmap(&tv);
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, C::TMEM_COLS);
+        tmem_relinquish();
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // Q: two tiles x ATOMS boxes of [128 rows x 64 d]
+            mbar_arrive_expect_tx(q_full, 2 * C::Q_TILE);
+            for (int t = 0; t < 2; ++t)
+                for (int a = 0; a < C::ATOMS; ++a)
+                    tma_load_3d(sq + t * C::Q_TILE + a * (BQ * 128), &tq, q_full, 64 * a, q0 + t * BQ, h);
+            int stage = 0;
+            uint32_t phase = 0;
+            bool armed[C::STAGES];
+            uint32_t armed_phase[C::STAGES];
+            for (int s = 0; s < C::STAGES; ++s) armed[s] = false;
+            for (int j = 0; j < n_kv; ++j) {
+                if (!mbar_wait(&kv_empty[stage], phase ^ 1u, abort_flag, g.err)) break;
+                mbar_arrive_expect_tx(&kv_full[stage], C::STAGE);
+                uint8_t* sk = skv + stage * C::STAGE;
+                uint8_t* sv = sk + C::K_TILE;
+                for (int a = 0; a < C::ATOMS; ++a) tma_load_3d(sk + a * (BKV * 128), &tk, &kv_full[stage], 64 * a, j * BKV, h);
+                for (int a = 0; a < BKV / 64; ++a) tma_load_3d(sv + a * (D * 128), &tv, &kv_full[stage], j * BKV + 64 * a, 0, h);
+                armed[stage] = true;
+                armed_phase[stage] = phase;
+                if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
+            }
+            {
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(q_full, 0) && globaltimer() - t0 < kWaitLimitNs) {
+                }
+            }
+            for (int s = 0; s < C::STAGES; ++s) {
+                if (!armed[s]) continue;
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(&kv_full[s], armed_phase[s]) && globaltimer() - t0 < kWaitLimitNs) {
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc_s = idesc_bf16(BQ, BKV);
+            constexpr uint32_t idesc_o = idesc_bf16(BQ, D);
+            const uint32_t sq0 = smem_u32(sq);
+            bool ok = mbar_wait(q_full, 0, abort_flag, g.err);
+            int stage = 0, prev = 0;
+            uint32_t phase = 0;
+            // S(t) = Q(t) K^T into TMEM columns [128 t, 128 t + 128)
+            auto issue_s = [&](int t, int st) {
+                const uint32_t kb = smem_u32(skv + st * C::STAGE);
+                const uint32_t qb = sq0 + t * C::Q_TILE;
+#pragma unroll
+                for (int ks = 0; ks < D / 16; ++ks) {
+                    const uint32_t off = (ks >> 2) * (BQ * 128) + (ks & 3) * 32;
+                    const uint32_t koff = (ks >> 2) * (BKV * 128) + (ks & 3) * 32;
+                    tc_mma(tmem + t * 128, sdesc_sw128(qb + off), sdesc_sw128(kb + koff), idesc_s, ks != 0);
+                }
+            };
+            // O(t) (+)= P(t) V: A = P in TMEM (bf16 pairs over S(t)'s first 64 columns)
+            auto issue_pv = [&](int t, int st, bool acc) {
+                const uint32_t vb = smem_u32(skv + st * C::STAGE + C::K_TILE);
+#pragma unroll
+                for (int ks = 0; ks < BKV / 16; ++ks) {
+                    const uint32_t voff = (ks >> 2) * (D * 128) + (ks & 3) * 32;
+                    tc_mma_ts(tmem + C::TMEM_O + t * D, tmem + t * 128 + ks * 8, sdesc_sw128(vb + voff), idesc_o,
+                              (acc || ks != 0) ? 1u : 0u);
+                }
+            };
+            for (int j = 0; j < n_kv && ok; ++j) {
+                if (!mbar_wait(&kv_full[stage], phase, abort_flag, g.err)) { ok = false; break; }
+                tc_fence_after();
+                for (int t = 0; t < 2; ++t) {
+                    if (j > 0) {
+                        if (!mbar_wait(&p_full[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
+                        tc_fence_after();
+                        issue_pv(t, prev, j > 1);
+                        if (t == 1) tc_commit(&kv_empty[prev]);
+                    }
+                    issue_s(t, stage);
+                    tc_commit(&s_full[t]);
+                }
+                prev = stage;
+                if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
+            }
+            if (ok) {
+                for (int t = 0; t < 2; ++t) {
+                    if (!mbar_wait(&p_full[t], (n_kv - 1) & 1, abort_flag, g.err)) break;
+                    tc_fence_after();
+                    issue_pv(t, prev, n_kv > 1);
+                    if (t == 1) tc_commit(&kv_empty[prev]);
+                    tc_commit(&o_final[t]);
+                }
+            }
+            tc_commit(mma_done);
+            const unsigned long long t0 = globaltimer();
+            while (!mbar_try_wait(mma_done, 0) && globaltimer() - t0 < kWaitLimitNs) {
+            }
+        }
+    } else {
+        // softmax warpgroups: t = query tile, quarter = TMEM lane quarter
+        const int t = (warp - 2) >> 2;
+        const int quarter = warp & 3;
+        const int row = quarter * 32 + lane;                 // row within the tile = TMEM lane
+        const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+        const uint32_t s_addr = tmem + lane_base + (uint32_t)(t * 128);
+        const uint32_t o_addr = tmem + lane_base + C::TMEM_O + (uint32_t)(t * D);
+        const int last_valid = g.L - (n_kv - 1) * BKV;       // keys in the last tile
+        float m_run = -INFINITY, l_run = 0.f;
+        bool ok = true;
+        for (int j = 0; j < n_kv; ++j) {
+            if (!mbar_wait(&s_full[t], j & 1, abort_flag, g.err)) { ok = false; break; }
+            tc_fence_after();
+            float s[BKV];
+#pragma unroll
+            for (int c = 0; c < BKV / 32; ++c) tmem_ld32(s_addr + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&s[c * 32]));
+            tmem_ld_wait();
+            if (j == n_kv - 1 && last_valid < BKV) {
+#pragma unroll
+                for (int c = 0; c < BKV; ++c)
+                    if (c >= last_valid) s[c] = -INFINITY;
+            }
+            float mx = s[0];
+#pragma unroll
+            for (int c = 1; c < BKV; ++c) mx = fmaxf(mx, s[c]);
+            const float m_new = fmaxf(m_run, mx * g.scale_log2);
+            const float corr = ex2(m_run - m_new);
+            float sum = 0.f;
+            uint32_t p[BKV / 2];
+#pragma unroll
+            for (int c = 0; c < BKV; c += 2) {
+                const float a = ex2(fmaf(s[c], g.scale_log2, -m_new));
+                const float b = ex2(fmaf(s[c + 1], g.scale_log2, -m_new));
+                sum += a + b;
+                p[c / 2] = pack2(a, b);
+            }
+            l_run = l_run * corr + sum;
+            m_run = m_new;
+            if (j > 0 && __any_sync(0xffffffffu, corr < 1.0f)) {
+                // PV(j-1) of this tile completed before S(j) was committed: rescale O in place
+#pragma unroll
+                for (int c = 0; c < D; c += 32) {
+                    uint32_t o[32];
+                    tmem_ld32(o_addr + c, o);
+                    tmem_ld_wait();
+                    uint32_t lo[16], hi[16];
+#pragma unroll
+                    for (int q = 0; q < 16; ++q) {
+                        lo[q] = __float_as_uint(__uint_as_float(o[q]) * corr);
+                        hi[q] = __float_as_uint(__uint_as_float(o[16 + q]) * corr);
+                    }
+                    tmem_st16(o_addr + c, lo);
+                    tmem_st16(o_addr + c + 16, hi);
+                }
+            }
+            // P over the first 64 columns of S(t)
+#pragma unroll
+            for (int c = 0; c < BKV / 2; c += 16) tmem_st16(s_addr + c, *reinterpret_cast<uint32_t(*)[16]>(&p[c]));
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&p_full[t]);
+        }
+        if (ok && mbar_wait(&o_final[t], 0, abort_flag, g.err)) {
+            tc_fence_after();
+            const int tok = q0 + t * BQ + row;
+            const float inv = 1.0f / l_run;
+#pragma unroll
+            for (int c = 0; c < D; c += 32) {
+                uint32_t o[32];
+                tmem_ld32(o_addr + c, o);
+                tmem_ld_wait();
+                if (tok < g.L) {
+                    uint4* dst = reinterpret_cast<uint4*>(g.o + (size_t)tok * g.H * D + (size_t)h * D + c);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint4 w;
+                        w.x = pack2(__uint_as_float(o[8 * q + 0]) * inv, __uint_as_float(o[8 * q + 1]) * inv);
+                        w.y = pack2(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv);
+                        w.z = pack2(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv);
+                        w.w = pack2(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv);
+                        dst[q] = w;
+                    }
+                }
+            }
+        }
+        tc_fence_before();
+    }
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::TMEM_COLS);
+    }
+}
+
+template <int D>
+wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, cudaStream_t s) {
+    using Cf = AttnCfg<D>;
+    static bool attr = false;
+    if (!attr) {
+        cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cf::SMEM);
+        attr = true;
+    }
+    CUtensorMap tq, tk, tv;
+    std::string why;
+    const uint64_t row = (uint64_t)D * 2, head = (uint64_t)L * D * 2;
+    if (!encode_tmap_3d(&tq, q, D, L, H, row, head, 64, BQ, 1, &why) ||
+        !encode_tmap_3d(&tk, k, D, L, H, row, head, 64, BKV, 1, &why) ||
+        !encode_tmap_3d(&tv, vt, L, D, H, (uint64_t)L * 2, (uint64_t)L * D * 2, 64, D, 1, &why))
+        return fail(c, WDC_ERR_CUDA, why);
+    AttnArgs g;
+    g.H = H;
+    g.L = L;
+    g.n_kv = (L + BKV - 1) / BKV;
+    g.q_blocks = (L + 2 * BQ - 1) / (2 * BQ);
+    g.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
+    g.o = reinterpret_cast<__nv_bfloat16*>(o);
+    g.err = c->err;
+    attn_tc_kernel<D><<<H * g.q_blocks, kAttnThreads, Cf::SMEM, s>>>(tq, tk, tv, g);
+    c->launches++;
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 attention launch: ") + cudaGetErrorString(e));
+    return WDC_OK;
+}
+
+}  // namespace
+
+bool tc_attention_supported(int L, int d) { return L > 0 && L % 8 == 0 && (d == 64 || d == 128); }
+
+wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
+                        cudaStream_t s) {
+    if (((uintptr_t)q | (uintptr_t)k | (uintptr_t)vt | (uintptr_t)o) & 15)
+        return fail(c, WDC_ERR_INVALID_ARG, "attention operands must be 16-byte aligned");
+    return d == 64 ? launch<64>(c, q, k, vt, o, H, L, s) : launch<128>(c, q, k, vt, o, H, L, s);
+}
+
 }  // namespace wdc

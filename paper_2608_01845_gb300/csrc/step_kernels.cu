@@ -310,11 +310,13 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                         o[e] = zh;
                         sa[e] = a.src[K - 1][idx];
                     } else if constexpr (MODE == kModeAnchor) {
+                        // read z_k and z_a before the store: they may alias the slot
                         const float z = a.src[0][idx];
+                        const float za = a.anchor[idx];
                         const float ze = fmaf(dsig, a.v[idx], z);
                         a.out[idx] = ze;
                         o[e] = ze;
-                        sa[e] = a.anchor[idx];
+                        sa[e] = za;
                         sb[e] = z;
                         if (a.zcf) fac[0] += fabsf(ze - a.zcf[idx]);
                     } else if constexpr (MODE == kModeStats) {

@@ -167,9 +167,11 @@ def _stream(s):
 
 
 def make_cond(tokens=None, cam=None, depth=None):
+    """wdc_cond for one step.  The returned object keeps ``tokens`` alive."""
     c = Cond()
     c.tokens = None if tokens is None else (tokens.data_ptr() if hasattr(tokens, "data_ptr") else
                                             tokens.ctypes.data)
+    c._keep = tokens
     for j in range(4):
         c.cam[j] = 0.0 if cam is None else float(cam[j])
         c.depth[j] = 0.0 if depth is None else float(depth[j])
