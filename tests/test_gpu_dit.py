@@ -89,8 +89,11 @@ def test_bf16_gemm_matches_oracle(M, N, K, mode):
     assert rel_l2(C.float().cpu().numpy(), want) <= 1e-2
 
 
-@pytest.mark.parametrize("H,L,d", [(2, 300, 64), (1, 1000, 128), (3, 129, 64), (1, 64, 128)])
+@pytest.mark.parametrize("H,L,d", [(2, 1000, 64), (1, 1000, 128), (3, 264, 64), (1, 64, 128), (2, 4104, 64),
+                                   (1, 2056, 128), (2, 300, 64), (1, 129, 128)])
 def test_bf16_attention_matches_oracle(H, L, d):
+    """L % 8 == 0 runs the tcgen05 kernel (ragged against its 128-key and
+    256-query tiles); other L the SIMT kernel."""
     ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
     q = _bf(synth.normal(11, (H, L, d)))
     k = _bf(synth.normal(12, (H, L, d)))
@@ -144,3 +147,25 @@ def test_bf16_block_5b_scale_sampled_rows():
     delta_want = want - x[rows]
     assert rel_l2(delta_got, delta_want) <= BF16_TOL
     assert rel_l2(got, want) <= BF16_TOL
+
+
+@pytest.mark.parametrize("H,L,d", [(48, 17776, 64), (24, 13568, 128)])
+def test_bf16_attention_full_size_sampled_rows(H, L, d):
+    """The attention shapes of the 5B-scale (48 x 64 heads, L = 17776) and
+    13B-scale (24 x 128 heads, L = 13568) models; 96 sampled query rows per
+    head compared with fp64."""
+    ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
+    g = np.random.default_rng(44)
+    q = _bf(g.standard_normal((H, L, d), dtype=np.float32))
+    k = _bf(g.standard_normal((H, L, d), dtype=np.float32))
+    v = _bf(g.standard_normal((H, L, d), dtype=np.float32))
+    o = torch.empty(L, H * d, dtype=torch.bfloat16, device="cuda")
+    ctx.op_attention(_to_dev(q, torch.bfloat16), _to_dev(k, torch.bfloat16),
+                     _to_dev(np.ascontiguousarray(v.transpose(0, 2, 1)), torch.bfloat16), o)
+    torch.cuda.synchronize()
+    got = o.float().cpu().numpy()
+    rows = np.sort(g.choice(L, 96, replace=False))
+    rows[-1] = L - 1
+    for h in range(0, H, 7):
+        want = dit.attention(q[h, rows].astype(np.float64), k[h].astype(np.float64), v[h].astype(np.float64), 1)
+        assert rel_l2(got[rows, h * d:(h + 1) * d], want) <= 1e-2, h
