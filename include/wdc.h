@@ -172,6 +172,10 @@ wdc_status wdc_default_cache_params(wdc_cache_params* out);
 wdc_status wdc_create(const wdc_dit_config* cfg, const wdc_schedule* sched,
                       const wdc_cache_params* params, int device, wdc_ctx** out);
 void wdc_destroy(wdc_ctx* ctx);
+/* Replaces the constants of Eq. 3-10 (validated as in wdc_create).  The bank
+ * capacity must stay the same (WDC_ERR_INVALID_ARG otherwise); the state is
+ * kept, so call it between rollouts. */
+wdc_status wdc_set_cache_params(wdc_ctx* ctx, const wdc_cache_params* params);
 const char* wdc_last_error(const wdc_ctx* ctx);
 size_t wdc_latent_numel(const wdc_ctx* ctx);
 /* Number of kernels this context has launched so far (all streams). */
@@ -259,6 +263,25 @@ wdc_status wdc_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* conds, in
 /* The uncached rollout: wdc_dit_forward + wdc_scheduler_step at every step. */
 wdc_status wdc_native_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* conds, int n_cond,
                               float* z_out, wdc_stream stream);
+
+/* ------------------------------------------------------------------ profiling
+ * Per-kernel-class timing for roofline reporting: when enabled, every launch
+ * of the library is bracketed by two CUDA events recorded on its launch
+ * stream.  wdc_profile_read synchronises the device and returns, per class,
+ * the summed event time (ms) and the launch count since the last enable or
+ * read (which clears them).  Disabled by default; costs two cudaEventRecord
+ * calls per launch when on.  Not a method step (no counterpart in the paper). */
+enum wdc_kernel_class {
+    WDC_K_GEMM = 0,    /* tcgen05 / SIMT GEMMs of the denoiser            */
+    WDC_K_ATTN = 1,    /* attention                                      */
+    WDC_K_NORM = 2,    /* LayerNorm + modulation                         */
+    WDC_K_SKIP = 3,    /* fused skip pass (wdc_surrogate_step)           */
+    WDC_K_ANCHOR = 4,  /* fused anchor pass (wdc_risk_update)            */
+    WDC_K_OTHER = 5,   /* timestep MLP, patchify, Psi, statistics, init  */
+    WDC_K_COUNT = 6
+};
+wdc_status wdc_profile_enable(wdc_ctx* ctx, int on);
+wdc_status wdc_profile_read(wdc_ctx* ctx, double* ms, unsigned long long* launches);
 
 /* ------------------------------------------------------------------ operators
  * The denoiser's hot kernels, exposed for parity tests and roofline timing.   */

@@ -20,6 +20,35 @@ wdc_status fail(Ctx* c, wdc_status s, const std::string& msg) {
     if (c) c->last_error = msg;
     return s;
 }
+
+static cudaEvent_t next_event(Ctx* c, int cls) {
+    auto& v = c->ev[cls];
+    if (c->ev_used[cls] == v.size()) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) { cudaGetLastError(); return nullptr; }
+        v.push_back(e);
+    }
+    return v[c->ev_used[cls]++];
+}
+
+LaunchScope::LaunchScope(Ctx* c_, int cls_, cudaStream_t s_) : c(c_), cls(cls_), s(s_) {
+    c->launches++;
+    c->cls_launches[cls]++;
+    if (c->prof) {
+        // reserve both events of the pair up front so begin/end never misalign
+        cudaEvent_t b = next_event(c, cls);
+        cudaEvent_t e = b ? next_event(c, cls) : nullptr;
+        if (b && e) {
+            cudaEventRecord(b, s);
+            end = e;
+        } else if (b) {
+            c->ev_used[cls]--;
+        }
+    }
+}
+LaunchScope::~LaunchScope() {
+    if (end) cudaEventRecord(end, s);
+}
 }  // namespace wdc
 
 namespace {
@@ -278,7 +307,20 @@ void wdc_destroy(wdc_ctx* h) {
     cudaFree(c->vbuf);
     cudaFree(c->zstage);
     if (c->out_host) cudaFreeHost(c->out_host);
+    for (int k = 0; k < WDC_K_COUNT; ++k)
+        for (cudaEvent_t e : c->ev[k]) cudaEventDestroy(e);
     delete c;
+}
+
+wdc_status wdc_set_cache_params(wdc_ctx* h, const wdc_cache_params* params) {
+    Ctx* c = reinterpret_cast<Ctx*>(h);
+    if (!c || !params) return WDC_ERR_INVALID_ARG;
+    wdc_status st = check_params(c, *params);
+    if (st) return st;
+    if (params->bank_capacity != c->prm.bank_capacity)
+        return fail(c, WDC_ERR_INVALID_ARG, "bank_capacity cannot change after wdc_create");
+    c->prm = *params;
+    return WDC_OK;
 }
 
 const char* wdc_last_error(const wdc_ctx* h) {
@@ -289,6 +331,36 @@ const char* wdc_last_error(const wdc_ctx* h) {
 size_t wdc_latent_numel(const wdc_ctx* h) {
     const Ctx* c = reinterpret_cast<const Ctx*>(h);
     return c ? c->n : 0;
+}
+
+wdc_status wdc_profile_enable(wdc_ctx* h, int on) {
+    Ctx* c = reinterpret_cast<Ctx*>(h);
+    if (!c) return WDC_ERR_INVALID_ARG;
+    cudaSetDevice(c->device);
+    WDC_CUDA_TRY(c, cudaDeviceSynchronize());
+    c->prof = on != 0;
+    for (int k = 0; k < WDC_K_COUNT; ++k) { c->ev_used[k] = 0; c->cls_launches[k] = 0; }
+    return WDC_OK;
+}
+
+wdc_status wdc_profile_read(wdc_ctx* h, double* ms, unsigned long long* launches) {
+    Ctx* c = reinterpret_cast<Ctx*>(h);
+    if (!c || !ms || !launches) return WDC_ERR_INVALID_ARG;
+    cudaSetDevice(c->device);
+    WDC_CUDA_TRY(c, cudaDeviceSynchronize());
+    for (int k = 0; k < WDC_K_COUNT; ++k) {
+        double tot = 0.0;
+        for (size_t i = 0; i + 1 < c->ev_used[k]; i += 2) {
+            float t = 0.f;
+            if (cudaEventElapsedTime(&t, c->ev[k][i], c->ev[k][i + 1]) == cudaSuccess) tot += t;
+            else cudaGetLastError();
+        }
+        ms[k] = tot;
+        launches[k] = c->cls_launches[k];
+        c->ev_used[k] = 0;
+        c->cls_launches[k] = 0;
+    }
+    return WDC_OK;
 }
 
 unsigned long long wdc_launch_count(const wdc_ctx* h) {
@@ -342,8 +414,10 @@ wdc_status wdc_scheduler_step(wdc_ctx* h, int k, const float* z_t, const float* 
     cudaSetDevice(c->device);
     const long long n = (long long)c->n;
     const unsigned grid = (unsigned)(((n + 3) / 4 + 255) / 256);
-    psi_kernel<<<grid, 256, 0, (cudaStream_t)stream>>>(z_t, v, z_next, n, (float)(c->sigma[k + 1] - c->sigma[k]));
-    c->launches++;
+    {
+        LaunchScope ls(c, WDC_K_OTHER, (cudaStream_t)stream);
+        psi_kernel<<<grid, 256, 0, (cudaStream_t)stream>>>(z_t, v, z_next, n, (float)(c->sigma[k + 1] - c->sigma[k]));
+    }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("scheduler_step: ") + cudaGetErrorString(e));
     return WDC_OK;

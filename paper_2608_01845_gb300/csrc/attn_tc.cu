@@ -328,7 +328,6 @@ wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o,
     g.o = reinterpret_cast<__nv_bfloat16*>(o);
     g.err = c->err;
     attn_tc_kernel<D><<<H * g.q_blocks, kAttnThreads, Cf::SMEM, s>>>(tq, tk, tv, g);
-    c->launches++;
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 attention launch: ") + cudaGetErrorString(e));
     return WDC_OK;

@@ -300,6 +300,7 @@ void launch_ln_mod(const void* x, void* h, int r0, int r1, int D, const float* s
 // ---------------------------------------------------------------- dispatch
 static wdc_status gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, const Epi& e, cudaStream_t s) {
     if (M <= 0 || N <= 0) return WDC_OK;
+    LaunchScope ls(c, WDC_K_GEMM, s);
     if (c->cfg.dtype == WDC_BF16 && tc_gemm_supported(M, N, K)) return tc_gemm(c, A, W, M, N, K, e, s);
     dim3 grid(blocks_for(N, 64), blocks_for(M, 64));
     if (c->cfg.dtype == WDC_BF16)
@@ -308,12 +309,12 @@ static wdc_status gemm(Ctx* c, const void* A, const void* W, int M, int N, int K
     else
         gemm_simt_kernel<float><<<grid, 256, 0, s>>>(reinterpret_cast<const float*>(A),
                                                      reinterpret_cast<const float*>(W), M, N, K, e);
-    c->launches++;
     return WDC_OK;
 }
 
 static wdc_status attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
                             cudaStream_t s) {
+    LaunchScope ls(c, WDC_K_ATTN, s);
     if (c->cfg.dtype == WDC_BF16 && tc_attention_supported(L, d)) return tc_attention(c, q, k, vt, o, H, L, d, s);
     dim3 grid(blocks_for(L, 128), H);
     const float scale = 1.0f / sqrtf((float)d);
@@ -330,18 +331,17 @@ static wdc_status attention(Ctx* c, const void* q, const void* k, const void* vt
         else
             attn_simt_kernel<T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
     }
-    c->launches++;
     return WDC_OK;
 }
 
 static void ln_mod(Ctx* c, const void* x, void* h, int r0, int r1, const float* shift, const float* scale,
                    int h_row_off, cudaStream_t s) {
     if (r1 <= r0) return;
+    LaunchScope ls(c, WDC_K_NORM, s);
     if (c->cfg.dtype == WDC_BF16)
         launch_ln_mod<__nv_bfloat16>(x, h, r0, r1, c->cfg.hidden, shift, scale, h_row_off, s);
     else
         launch_ln_mod<float>(x, h, r0, r1, c->cfg.hidden, shift, scale, h_row_off, s);
-    c->launches++;
 }
 
 // ---------------------------------------------------------------- lifetime
@@ -417,11 +417,11 @@ wdc_status dit_create(Ctx* c) {
     if ((s = dalloc(c, (void**)&t->temb, (size_t)t->E * sizeof(float)))) return s;
     if ((s = dalloc(c, (void**)&t->mods, t->mod_rows * sizeof(float)))) return s;
     const long long npe = (long long)t->Lv * t->D;
+    LaunchScope ls(c, WDC_K_OTHER, 0);
     if (t->dtype == WDC_BF16)
         posemb_kernel<__nv_bfloat16><<<blocks_for(npe, 256), 256>>>((__nv_bfloat16*)t->pe, t->Lv, t->D);
     else
         posemb_kernel<float><<<blocks_for(npe, 256), 256>>>((float*)t->pe, t->Lv, t->D);
-    c->launches++;
     cudaError_t e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("DiT init: ") + cudaGetErrorString(e));
     return WDC_OK;
@@ -496,11 +496,11 @@ wdc_status dit_set_tensor(Ctx* c, int id, int layer, int stream, const float* ho
 
 static void init_normal(Ctx* c, void* dst, size_t n, unsigned long long seed, uint32_t sid, float std) {
     const unsigned grid = blocks_for((long long)(n + 3) / 4, 256);
+    LaunchScope ls(c, WDC_K_OTHER, 0);
     if (c->dit->dtype == WDC_BF16)
         normal_init_kernel<__nv_bfloat16><<<grid, 256>>>((__nv_bfloat16*)dst, (long long)n, seed, sid, std);
     else
         normal_init_kernel<float><<<grid, 256>>>((float*)dst, (long long)n, seed, sid, std);
-    c->launches++;
 }
 
 wdc_status dit_init_weights(Ctx* c, unsigned long long seed, float std) {
@@ -526,9 +526,13 @@ wdc_status dit_modulation(Ctx* c, float t_model, float* mod_out, cudaStream_t s)
     if (!t) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
     float* dst = mod_out ? mod_out : t->mods;
     const int half = t->Fd / 2;
-    features_kernel<<<blocks_for(half, 128), 128, 0, s>>>(t_model, half, t->feat);
+    {
+        LaunchScope ls(c, WDC_K_OTHER, s);
+        features_kernel<<<blocks_for(half, 128), 128, 0, s>>>(t_model, half, t->feat);
+    }
     auto gv = [&](const void* W, const float* x, const float* b, float* y, int rows, int cols, int act) {
         const unsigned grid = blocks_for((long long)rows * 32, 256);
+        LaunchScope ls(c, WDC_K_OTHER, s);
         if (t->dtype == WDC_BF16)
             gemv_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)W, x, b, y, rows, cols, act);
         else
@@ -537,7 +541,6 @@ wdc_status dit_modulation(Ctx* c, float t_model, float* mod_out, cudaStream_t s)
     gv(t->t1.w, t->feat, t->t1.b, t->h1, t->E, t->Fd, 1);
     gv(t->t2.w, t->h1, t->t2.b, t->temb, t->E, t->E, 1);   // SiLU(temb)
     gv(t->modW, t->temb, t->modB, dst, (int)t->mod_rows, t->E, 0);
-    c->launches += 4;
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("modulation: ") + cudaGetErrorString(e));
     return WDC_OK;
@@ -611,22 +614,26 @@ wdc_status dit_forward(Ctx* c, const float* z, float t_model, const float* cond,
     // embed: condition tokens, then patches + position
     if (t->Lc > 0) {
         const long long nc = (long long)t->Lc * t->Dc;
-        if (t->dtype == WDC_BF16)
-            convert_kernel<__nv_bfloat16><<<blocks_for(nc, 256), 256, 0, s>>>(cond, (__nv_bfloat16*)t->condx, nc);
-        else
-            convert_kernel<float><<<blocks_for(nc, 256), 256, 0, s>>>(cond, (float*)t->condx, nc);
-        c->launches++;
+        {
+            LaunchScope ls(c, WDC_K_OTHER, s);
+            if (t->dtype == WDC_BF16)
+                convert_kernel<__nv_bfloat16><<<blocks_for(nc, 256), 256, 0, s>>>(cond, (__nv_bfloat16*)t->condx, nc);
+            else
+                convert_kernel<float><<<blocks_for(nc, 256), 256, 0, s>>>(cond, (float*)t->condx, nc);
+        }
         Epi e{};
         e.mode = kEpiStore; e.bias = t->cond.b; e.out = t->x; e.ldo = D;
         if ((st = gemm(c, t->condx, t->cond.w, t->Lc, D, t->Dc, e, s))) return st;
     }
     {
         const long long nt = (long long)t->Lv * t->P;
-        if (t->dtype == WDC_BF16)
-            patchify_kernel<__nv_bfloat16><<<blocks_for(nt, 256), 256, 0, s>>>(z, (__nv_bfloat16*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
-        else
-            patchify_kernel<float><<<blocks_for(nt, 256), 256, 0, s>>>(z, (float*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
-        c->launches++;
+        {
+            LaunchScope ls(c, WDC_K_OTHER, s);
+            if (t->dtype == WDC_BF16)
+                patchify_kernel<__nv_bfloat16><<<blocks_for(nt, 256), 256, 0, s>>>(z, (__nv_bfloat16*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
+            else
+                patchify_kernel<float><<<blocks_for(nt, 256), 256, 0, s>>>(z, (float*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
+        }
         Epi e{};
         char* xv = (char*)t->x + (size_t)t->Lc * D * es;
         e.mode = kEpiResid; e.bias = t->patch.b; e.out = xv; e.res = t->pe; e.ldo = D; e.gate = nullptr;

@@ -359,7 +359,6 @@ wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, co
     const int tiles = g.m_tiles * g.n_tiles;
     const int grid = tiles < c->num_sms ? tiles : c->num_sms;
     gemm_tc_kernel<<<grid, kGemmThreads, SMEM_BYTES, s>>>(ta, tb, g);
-    c->launches++;
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(err));
     return WDC_OK;

@@ -595,6 +595,7 @@ int pass_grid(const Ctx* c) {
 
 wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s) {
     const int grid = pass_grid(c);
+    LaunchScope ls(c, mode == kModeSkip ? WDC_K_SKIP : (mode == kModeAnchor ? WDC_K_ANCHOR : WDC_K_OTHER), s);
     switch (mode) {
         case kModeStats: pass_kernel<kModeStats, 0><<<grid, kThreads, 0, s>>>(a); break;
         case kModeAnchor: pass_kernel<kModeAnchor, 0><<<grid, kThreads, 0, s>>>(a); break;
@@ -614,7 +615,6 @@ wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s) {
             break;
         default: return fail(c, WDC_ERR_INVALID_ARG, "unknown pass mode");
     }
-    c->launches += 1;
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("latent pass launch: ") + cudaGetErrorString(e));
     return WDC_OK;
@@ -654,3 +654,4 @@ ParamsDev to_dev_params(const wdc_cache_params& p) {
 }
 
 }  // namespace wdc
+

@@ -119,6 +119,22 @@ struct Ctx {
 
     // denoiser
     struct DiT* dit = nullptr;
+
+    // optional per-class event timing (wdc_profile_enable)
+    bool prof = false;
+    std::vector<cudaEvent_t> ev[WDC_K_COUNT];      // begin/end pairs
+    size_t ev_used[WDC_K_COUNT] = {};
+    unsigned long long cls_launches[WDC_K_COUNT] = {};
+};
+
+// Brackets one launch for the optional profiler and counts it.
+struct LaunchScope {
+    Ctx* c;
+    int cls;
+    cudaStream_t s;
+    cudaEvent_t end = nullptr;
+    LaunchScope(Ctx* c_, int cls_, cudaStream_t s_);
+    ~LaunchScope();
 };
 
 // ---------------------------------------------------------------- helpers

@@ -103,6 +103,9 @@ def _load():
         "wdc_create": (I, [ctypes.POINTER(DitConfig), ctypes.POINTER(Schedule), ctypes.POINTER(CacheParams), I,
                            ctypes.POINTER(P)]),
         "wdc_destroy": (None, [P]),
+        "wdc_set_cache_params": (I, [P, ctypes.POINTER(CacheParams)]),
+        "wdc_profile_enable": (I, [P, I]),
+        "wdc_profile_read": (I, [P, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_ulonglong)]),
         "wdc_last_error": (ctypes.c_char_p, [P]),
         "wdc_latent_numel": (S, [P]),
         "wdc_launch_count": (ctypes.c_ulonglong, [P]),
@@ -214,6 +217,21 @@ class Context:
     def launches(self):
         return LIB.wdc_launch_count(self._h)
 
+    def set_cache_params(self, params):
+        self._check(LIB.wdc_set_cache_params(self._h, ctypes.byref(params)), "set_cache_params")
+        self.params = params
+
+    def profile_enable(self, on=True):
+        self._check(LIB.wdc_profile_enable(self._h, int(on)), "profile_enable")
+
+    def profile_read(self):
+        """{class name: (ms, launches)} since the last enable/read."""
+        ms = (ctypes.c_double * 6)()
+        n = (ctypes.c_ulonglong * 6)()
+        self._check(LIB.wdc_profile_read(self._h, ms, n), "profile_read")
+        names = ["gemm", "attention", "norm", "skip", "anchor", "other"]
+        return {names[i]: (ms[i], n[i]) for i in range(6)}
+
     def set_tensor(self, tensor_id, array, layer=0, stream=0):
         import numpy as np
         a = np.ascontiguousarray(array, dtype=np.float32)
@@ -299,3 +317,4 @@ class Context:
         H, L, d = q.shape
         self._check(LIB.wdc_op_attention(self._h, _ptr(q), _ptr(k), _ptr(vt), _ptr(o), H, L, d, _stream(stream)),
                     "op_attention")
+
