@@ -297,6 +297,40 @@ wdc_status wdc_op_gemm(wdc_ctx* ctx, const void* A, const void* W, const float* 
 wdc_status wdc_op_attention(wdc_ctx* ctx, const void* q, const void* k, const void* vt, void* o,
                             int heads, int L, int d, wdc_stream stream);
 
+/* ------------------------------------------------------------------ allocation-free variant
+ * wdc_observe_noalloc: the streaming half of the skip pass -- the kernelised
+ * observation z_hat = sum_i kappa_i z_out_i over K latents together with the
+ * statistics the next lift needs -- for callers that cannot call cudaMalloc
+ * (code running under another framework's memory manager or inside a
+ * pre-sized arena, processes that must not allocate device memory after set-up).
+ * The paper has no counterpart: it is a deployment variant of the same kernel.
+ *
+ * It allocates nothing and needs no wdc_ctx.  Its scratch (per-CTA partial sums
+ * and a completion counter, 256 CTAs x 248 doubles + 256 bytes = 508 KB) is a
+ * file-scope __device__ array that every GPU loading libwdc.so holds until the
+ * process exits.  The first call on a device, with that device current, looks
+ * up the array's device address (cudaGetSymbolAddress) and caches it; make that
+ * first call before any stream capture.  Each call clears the counter on
+ * `stream` before its kernel.  All calls on a device share the scratch, so
+ * calls that overlap on the GPU (different streams, no ordering) race; order
+ * them on one stream.
+ *
+ *   z_out      host array of K device pointers (fp32 latents, n elements,
+ *              16-byte aligned), 1 <= K <= WDC_MAX_BANK
+ *   kappa      host array of K weights (used in fp32, as the skip pass does)
+ *   z_a        device fp32 latent (the anchor) for sum (z_hat - z_a)^2
+ *   z_hat      device fp32 output, n elements (must not alias the inputs)
+ *   stats      device output, 123 doubles: [0..119] raw signed bucket sums
+ *              sum_{bucket(i)=b} sign(i) z_hat_i (the summary sketch before its
+ *              sqrt(120/n) scale), [120] sum z_hat^2, [121] sum (z_hat - z_a)^2,
+ *              [122] count of non-finite z_hat elements
+ *   n          elements, 1 <= n < 2^31 (the sign hash indexes 32 bits)
+ *   sketch_seed  seed of the sign hash (wdc_cache_params.sketch_seed)
+ * Returns WDC_ERR_INVALID_ARG for sizes or pointers outside these limits,
+ * WDC_ERR_CUDA if the symbol lookup or the launch fails.  Asynchronous. */
+wdc_status wdc_observe_noalloc(const float* const* z_out, int K, const double* kappa, const float* z_a,
+                               float* z_hat, double* stats, size_t n, uint32_t sketch_seed, wdc_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -27,6 +27,8 @@
 #include "wdc_internal.h"
 
 #include <cmath>
+#include <cstring>
+#include <mutex>
 
 namespace wdc {
 
@@ -237,6 +239,10 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
         do_stream = (K > 0) && hs.supported;
 #pragma unroll
         for (int i = 0; i < K; ++i) kap[i] = (float)hs.kappa[i];
+    } else if (MODE == kModeObserve) {
+#pragma unroll
+        for (int i = 0; i < K; ++i) kap[i] = a.kappa[i];
+        __syncthreads();
     } else {
         __syncthreads();
     }
@@ -272,6 +278,21 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                     *reinterpret_cast<float4*>(a.out + base) = zh;
                     o[0] = zh.x; o[1] = zh.y; o[2] = zh.z; o[3] = zh.w;
                     sa[0] = x[K - 1].x; sa[1] = x[K - 1].y; sa[2] = x[K - 1].z; sa[3] = x[K - 1].w;
+                } else if constexpr (MODE == kModeObserve && K > 0) {
+                    float4 x[K];
+#pragma unroll
+                    for (int i = 0; i < K; ++i) x[i] = __ldg(reinterpret_cast<const float4*>(a.src[i] + base));
+                    const float4 za = __ldg(reinterpret_cast<const float4*>(a.anchor + base));
+                    float4 zh;
+                    zh.x = kap[0] * x[0].x; zh.y = kap[0] * x[0].y; zh.z = kap[0] * x[0].z; zh.w = kap[0] * x[0].w;
+#pragma unroll
+                    for (int i = 1; i < K; ++i) {
+                        zh.x = fmaf(kap[i], x[i].x, zh.x); zh.y = fmaf(kap[i], x[i].y, zh.y);
+                        zh.z = fmaf(kap[i], x[i].z, zh.z); zh.w = fmaf(kap[i], x[i].w, zh.w);
+                    }
+                    *reinterpret_cast<float4*>(a.out + base) = zh;
+                    o[0] = zh.x; o[1] = zh.y; o[2] = zh.z; o[3] = zh.w;
+                    sa[0] = za.x; sa[1] = za.y; sa[2] = za.z; sa[3] = za.w;
                 } else if constexpr (MODE == kModeAnchor) {
                     // plain loads: z_k / z_a may alias the slot written below (bank capacity 1)
                     const float4 z = *reinterpret_cast<const float4*>(a.src[0] + base);
@@ -309,6 +330,13 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                         a.out[idx] = zh;
                         o[e] = zh;
                         sa[e] = a.src[K - 1][idx];
+                    } else if constexpr (MODE == kModeObserve && K > 0) {
+                        float zh = kap[0] * a.src[0][idx];
+#pragma unroll
+                        for (int i = 1; i < K; ++i) zh = fmaf(kap[i], a.src[i][idx], zh);
+                        a.out[idx] = zh;
+                        o[e] = zh;
+                        sa[e] = a.anchor[idx];
                     } else if constexpr (MODE == kModeAnchor) {
                         // read z_k and z_a before the store: they may alias the slot
                         const float z = a.src[0][idx];
@@ -334,7 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                 const float d = x - sa[e];
                 const uint32_t idx = (uint32_t)(base + e);
                 sg += signed_term(idx, seed, x);
-                if (MODE == kModeSkip) {
+                if (MODE == kModeSkip || MODE == kModeObserve) {
                     fac[0] += x * x;
                     fac[1] += d * d;
                     nonfinite += isfinite(x) ? 0 : 1;
@@ -416,6 +444,17 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
         __syncthreads();
     }
     if (t == 0) *a.counter = 0u;
+
+    if (MODE == kModeObserve) {
+        // raw signed bucket sums of z_hat, sum z_hat^2, sum (z_hat - z_a)^2, non-finite count
+        if (t < kSketch) a.stats_out[t] = ps.fin[t];
+        if (t == 0) {
+            a.stats_out[kSketch + 0] = ps.fin[2 * kSketch + 0];
+            a.stats_out[kSketch + 1] = ps.fin[2 * kSketch + 1];
+            a.stats_out[kSketch + 2] = ps.fin[2 * kSketch + 5];
+        }
+        return;
+    }
 
     DevState* st = a.st;
     const double N = (double)n;
@@ -655,3 +694,107 @@ ParamsDev to_dev_params(const wdc_cache_params& p) {
 
 }  // namespace wdc
 
+// ---------------------------------------------------------------------------
+// Allocation-free variant of the observation pass (wdc_observe_noalloc).
+//
+// Some callers cannot call cudaMalloc: code that runs inside another
+// framework's memory manager or a pre-sized arena, and processes that must not
+// allocate device memory once they are set up.  For them this entry point
+// keeps its scratch -- the per-CTA partial sums and the last-CTA counter of
+// the fused pass -- in the file-scope array below, which every GPU that loads
+// this library holds until the process exits.
+namespace wdc {
+namespace {
+
+constexpr int kNoAllocMaxBlocks = 256;                       // CTAs the scratch can serve
+constexpr size_t kNoAllocPartialBytes = (size_t)kNoAllocMaxBlocks * kPartials * sizeof(double);
+constexpr size_t kNoAllocBytes = kNoAllocPartialBytes + 256;  // + the done counter
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+
+constexpr int kMaxDevices = 64;
+struct NoAllocDevice {
+    bool ready = false;
+    unsigned char* scratch = nullptr;   // device address of g_noalloc_scratch on this device
+    int num_sms = 0;
+};
+NoAllocDevice g_noalloc_dev[kMaxDevices];
+std::mutex g_noalloc_mu;
+
+template <int K>
+void launch_observe(const PassArgs& a, int grid, cudaStream_t s) {
+    pass_kernel<kModeObserve, K><<<grid, kThreads, 0, s>>>(a);
+}
+
+}  // namespace
+}  // namespace wdc
+
+extern "C" wdc_status wdc_observe_noalloc(const float* const* z_out, int K, const double* kappa, const float* z_a,
+                                          float* z_hat, double* stats, size_t n, uint32_t sketch_seed,
+                                          wdc_stream stream) {
+    using namespace wdc;
+    if (!z_out || !kappa || !z_a || !z_hat || !stats) return WDC_ERR_INVALID_ARG;
+    if (K < 1 || K > kMaxBank) return WDC_ERR_INVALID_ARG;
+    if (n == 0 || n >= (1ull << 31)) return WDC_ERR_INVALID_ARG;
+    for (int i = 0; i < K; ++i)
+        if (!z_out[i] || ((uintptr_t)z_out[i] & 15)) return WDC_ERR_INVALID_ARG;
+    if (((uintptr_t)z_a & 15) || ((uintptr_t)z_hat & 15) || ((uintptr_t)stats & 7)) return WDC_ERR_INVALID_ARG;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return WDC_ERR_CUDA; }
+    if (dev < 0 || dev >= kMaxDevices) return WDC_ERR_UNSUPPORTED;
+    NoAllocDevice d;
+    {
+        // once per device, with that device current: the host-side name of the
+        // array is not a device address, so look the address up
+        std::lock_guard<std::mutex> lock(g_noalloc_mu);
+        if (!g_noalloc_dev[dev].ready) {
+            void* p = nullptr;
+            if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) {
+                cudaGetLastError();
+                return WDC_ERR_CUDA;
+            }
+            int sms = 0;
+            if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+                cudaGetLastError();
+                return WDC_ERR_CUDA;
+            }
+            g_noalloc_dev[dev].scratch = static_cast<unsigned char*>(p);
+            g_noalloc_dev[dev].num_sms = sms;
+            g_noalloc_dev[dev].ready = true;
+        }
+        d = g_noalloc_dev[dev];
+    }
+    PassArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.n = (long long)n;
+    a.nsrc = K;
+    for (int i = 0; i < K; ++i) {
+        a.src[i] = z_out[i];
+        a.kappa[i] = (float)kappa[i];
+    }
+    a.anchor = z_a;
+    a.out = z_hat;
+    a.prm.seed = sketch_seed;
+    a.partials = reinterpret_cast<double*>(d.scratch);
+    a.counter = reinterpret_cast<unsigned*>(d.scratch + kNoAllocPartialBytes);
+    a.stats_out = stats;
+    const long long nruns = ((long long)n + kRun - 1) / kRun;
+    long long grid = (nruns + kWarps - 1) / kWarps;
+    if (grid > d.num_sms) grid = d.num_sms;
+    if (grid > kNoAllocMaxBlocks) grid = kNoAllocMaxBlocks;
+    if (grid < 1) grid = 1;
+    cudaStream_t s = (cudaStream_t)stream;
+    // the last-CTA counter must start at zero (a failed earlier call may have left it set)
+    if (cudaMemsetAsync(a.counter, 0, sizeof(unsigned), s) != cudaSuccess) { cudaGetLastError(); return WDC_ERR_CUDA; }
+    switch (K) {
+        case 1: launch_observe<1>(a, (int)grid, s); break;
+        case 2: launch_observe<2>(a, (int)grid, s); break;
+        case 3: launch_observe<3>(a, (int)grid, s); break;
+        case 4: launch_observe<4>(a, (int)grid, s); break;
+        case 5: launch_observe<5>(a, (int)grid, s); break;
+        case 6: launch_observe<6>(a, (int)grid, s); break;
+        case 7: launch_observe<7>(a, (int)grid, s); break;
+        default: launch_observe<8>(a, (int)grid, s); break;
+    }
+    if (cudaGetLastError() != cudaSuccess) return WDC_ERR_CUDA;
+    return WDC_OK;
+}

@@ -65,7 +65,7 @@ struct ParamsDev {
     double a_cam, a_depth, a_phase, lam, tau_risk;
 };
 
-enum StreamMode { kModeStats = 0, kModeSkip = 1, kModeAnchor = 2 };
+enum StreamMode { kModeStats = 0, kModeSkip = 1, kModeAnchor = 2, kModeObserve = 3 };
 
 // Launch arguments of the fused latent-pass kernels (passed by value).
 struct PassArgs {
@@ -86,6 +86,8 @@ struct PassArgs {
     double* partials;                  // [gridDim.x][kPartials]
     unsigned* counter;
     unsigned* err;
+    float kappa[kMaxBank];             // observe: caller-given weights
+    double* stats_out;                 // observe: caller-given statistics output
 };
 
 // ---------------------------------------------------------------- context

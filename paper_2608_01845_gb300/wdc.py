@@ -124,6 +124,7 @@ def _load():
         "wdc_native_rollout": (I, [P, P, ctypes.POINTER(Cond), I, P, P]),
         "wdc_op_gemm": (I, [P, P, P, P, P, I, I, I, I, P, P, P]),
         "wdc_op_attention": (I, [P, P, P, P, P, I, I, I, P]),
+        "wdc_observe_noalloc": (I, [ctypes.POINTER(P), I, ctypes.POINTER(D), P, P, P, S, ctypes.c_uint32, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -318,3 +319,15 @@ class Context:
         self._check(LIB.wdc_op_attention(self._h, _ptr(q), _ptr(k), _ptr(vt), _ptr(o), H, L, d, _stream(stream)),
                     "op_attention")
 
+
+def observe_noalloc(z_out, kappa, z_a, z_hat, stats, sketch_seed=0x2545F491, stream=None):
+    """wdc_observe_noalloc: z_hat = sum_i kappa_i z_out_i plus the next lift's
+    statistics (stats: device float64 tensor of 123 values), with no device
+    allocation inside the call (see include/wdc.h)."""
+    K = len(z_out)
+    ptrs = (ctypes.c_void_p * K)(*[t.data_ptr() for t in z_out])
+    kap = (ctypes.c_double * K)(*[float(x) for x in kappa])
+    st = LIB.wdc_observe_noalloc(ptrs, K, kap, _ptr(z_a), _ptr(z_hat), _ptr(stats), z_hat.numel(), sketch_seed,
+                                 _stream(stream))
+    if st != 0:
+        raise WdcError(st, "wdc_observe_noalloc failed")
