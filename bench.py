@@ -43,6 +43,17 @@ WORKLOAD_5B = dict(
     in_ch=16, frames=13, height=60, width=90, patch=2, cond_tokens=226, cond_dim=3072, dual_stream=0,
     T=50, tau_risk=0.1, target_exact=23, weight_seed=1234, input_seed=77,
 )
+# The HunyuanVoyager-13B-like cached rollout: 60 dual-stream layers (separate
+# condition-token weights, joint attention), 24 heads x 128, latent 16x13x64x64
+# (13312 video tokens) + 256 condition tokens.  Paper target exact-call ratio
+# 20% (section "Experimental Settings").
+WORKLOAD_13B = dict(
+    name="cached rollout, 60-layer dual-stream bf16 DiT 3072/24x128/12288 (~14.7B), latent 16x13x64x64 + 256 cond tokens, T=50",
+    layers=60, hidden=3072, heads=24, head_dim=128, mlp=12288, temb_dim=512, freq_dim=256,
+    in_ch=16, frames=13, height=64, width=64, patch=2, cond_tokens=256, cond_dim=3072, dual_stream=1,
+    T=50, tau_risk=0.1, target_exact=10, weight_seed=4321, input_seed=91,
+)
+WORKLOADS = {"5b": WORKLOAD_5B, "13b": WORKLOAD_13B}
 SKIP_SWEEP_N = 1 << 28          # fused skip pass measured at 2^28 fp32 elements, bank of 4
 
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
@@ -418,7 +429,7 @@ def run_op(args):
     launches, CUDA-event timing printed as JSON."""
     import torch
     from paper_2608_01845_gb300 import wdc
-    w = WORKLOAD_5B
+    w = WORKLOADS[args.workload]
     peaks, _ = load_peaks()
     L, D, H, d = tokens(w), w["hidden"], w["heads"], w["head_dim"]
     dev = torch.device("cuda")
@@ -439,7 +450,7 @@ def run_op(args):
     elif args.op == "block":
         ctx.init_weights(1, 0.02)
         x = torch.randn(L, D, device=dev).bfloat16()
-        mod = 0.1 * torch.randn(6, D, device=dev)
+        mod = 0.1 * torch.randn((2 if w["dual_stream"] else 1) * 6, D, device=dev)
         fn, work, unit = (lambda: ctx.dit_block_forward(0, x, mod)), sum(block_flops(w)), "TFLOP/s"
     else:
         r = skip_pass_gbps(torch, wdc, peaks)
@@ -457,7 +468,7 @@ def run_op(args):
         torch.cuda.synchronize()
         ts.append(a.elapsed_time(b))
     ms = statistics.median(ts)
-    print(json.dumps({"op": args.op, "ms": ms, unit: work / (ms * 1e-3) / 1e12}))
+    print(json.dumps({"op": args.op, "workload": args.workload, "ms": ms, unit: work / (ms * 1e-3) / 1e12}))
 
 
 def main():
@@ -470,6 +481,8 @@ def main():
     ap.add_argument("--op", choices=["attention", "gemm", "block", "skip"],
                     help="time one operator at its 5B-scale shape (profiler captures)")
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="5b",
+                    help="shape of --op (5b: 48x64 heads, L=17776; 13b: 24x128 heads, L=13568, dual stream)")
     args = ap.parse_args()
     if args.op:
         return run_op(args)

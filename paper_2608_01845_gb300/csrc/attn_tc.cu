@@ -3,22 +3,31 @@
 // full spatio-temporal attention).  Q, K [H, L, d], V^T [H, d, L], O [L, H*d],
 // bf16 with fp32 softmax and accumulation; d = 64 or 128.
 //
-// One CTA per (head, 256 query rows), 10 warps:
+// One CTA per (head, 256 query rows), 11 (d = 64) or 10 (d = 128) warps:
 //   warp 0      TMA producer: the two 128-row Q tiles once, then K / V^T tiles
 //               of 128 keys into a shared-memory ring (128-byte swizzle);
-//   warp 1      MMA issuer (one thread), ping-pong over the two query tiles:
-//                 PV0(j-1), S0(j), PV1(j-1), S1(j)
-//               S = Q K^T lands in TMEM (128 fp32 columns per tile); the
-//               softmax overwrites its first 64 columns with P (bf16 pairs),
-//               which the PV MMA reads as its A operand from TMEM;
+//   warp 1(,10) MMA issuer(s): one thread per query tile (d = 64) or one
+//               thread for both (d = 128):
+//               S(t) = Q(t) K^T into TMEM (128 fp32 columns per tile) and
+//               O(t) += P(t) V into TMEM;
 //   warps 2-5   softmax of query tile 0, warps 6-9 of tile 1 (one thread per
-//               query row = TMEM lane): online max / exp2 / row sum, O
-//               rescaling in TMEM when the running max moves, final 1/l
-//               normalisation and the bf16 store.
-// A commit after S(j) also covers PV(j-1) of the same tile (tcgen05 ops of
-// one thread complete in order), so the softmax may rescale O as soon as S(j)
-// is ready.  Keys past L are masked (TMA zero-fills out-of-range K / V^T).
-// Every mbarrier wait is bounded.
+//               query row = TMEM lane): online max, exp2, row sums, O
+//               rescaling in TMEM when the running max grows by more than 2^8,
+//               final 1/l normalisation and the bf16 store.
+// P (bf16 pairs) is written to tensor memory and read as the TMEM A operand
+// of the PV MMA (shared memory is left to Q, K and V).  Two TMEM layouts:
+//   d = 64   per tile t: S (128 columns), P (64), O (64) = 256 columns, so P
+//            has its own columns: S(t) may be overwritten as soon as the
+//            softmax has loaded it, and the MMA of S(t, j+1) overlaps the
+//            softmax of tile j:
+//               S(t, j), PV(t, j-1)   (per issuer)
+//   d = 128  S (2 x 128) + O (2 x 128) fill TMEM, so P is written back over
+//            the first 64 columns of S(t); S(t, j+1) then follows PV(t, j):
+//               PV0(j-1), S0(j), PV1(j-1), S1(j)
+//            and the commit after S(t, j) also covers PV(t, j-1) (tcgen05 ops
+//            of one thread complete in order).
+// Keys past L are masked (TMA zero-fills out-of-range K / V^T).  Every
+// mbarrier wait is bounded.
 #include "dit_kernels.cuh"
 #include "ptx.cuh"
 
@@ -26,12 +35,14 @@ namespace wdc {
 
 namespace {
 
-constexpr int kAttnThreads = 320;
 constexpr int BQ = 128;        // query rows per tile (two tiles per CTA)
 constexpr int BKV = 128;       // keys per tile
 
 template <int D>
 struct AttnCfg {
+    static constexpr bool P_SEP = D == 64;                  // P in its own TMEM columns, one issuer per tile
+    static constexpr int THREADS = P_SEP ? 352 : 320;       // 11 or 10 warps
+    static constexpr int ISSUERS = P_SEP ? 2 : 1;
     static constexpr int ATOMS = D / 64;                    // 128-byte atoms along d
     static constexpr uint32_t Q_TILE = BQ * D * 2;          // one query tile
     static constexpr uint32_t K_TILE = BKV * D * 2;
@@ -39,8 +50,11 @@ struct AttnCfg {
     static constexpr uint32_t STAGE = K_TILE + V_TILE;
     static constexpr int STAGES = D == 64 ? 3 : 2;
     static constexpr uint32_t SMEM = 2 * Q_TILE + STAGES * STAGE + 1024 + 256;
-    static constexpr uint32_t TMEM_O = 256;                 // O tiles after the two S tiles
     static constexpr uint32_t TMEM_COLS = 512;
+    // TMEM column of S, P and O of query tile t
+    __device__ static constexpr uint32_t s_col(int t) { return P_SEP ? 256u * t : 128u * t; }
+    __device__ static constexpr uint32_t p_col(int t) { return P_SEP ? 256u * t + 128u : 128u * t; }
+    __device__ static constexpr uint32_t o_col(int t) { return P_SEP ? 256u * t + 192u : 256u + (uint32_t)D * t; }
 };
 
 struct AttnArgs {
@@ -56,13 +70,20 @@ __device__ __forceinline__ float ex2(float x) {
     return y;
 }
 
+// Three-input maximum (one instruction for two comparisons).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
     __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
     return *reinterpret_cast<uint32_t*>(&h);
 }
 
 template <int D>
-__global__ void __launch_bounds__(kAttnThreads, 1)
+__global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
                    const __grid_constant__ CUtensorMap tv, const __grid_constant__ AttnArgs g) {
     using C = AttnCfg<D>;
@@ -75,8 +96,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint64_t* kv_full = q_full + 1;
     uint64_t* kv_empty = kv_full + C::STAGES;
     uint64_t* s_full = kv_empty + C::STAGES;                  // [2]
-    uint64_t* p_full = s_full + 2;                            // [2]
-    uint64_t* o_final = p_full + 2;                           // [2]
+    uint64_t* s_free = s_full + 2;                            // [2] (separate P)
+    uint64_t* p_full = s_free + 2;                            // [2]
+    uint64_t* p_free = p_full + 2;                            // [2] (separate P)
+    uint64_t* o_final = p_free + 2;                           // [2]
     uint64_t* mma_done = o_final + 2;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -90,14 +113,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         mbar_init(q_full, 1);
         for (int s = 0; s < C::STAGES; ++s) {
             mbar_init(&kv_full[s], 1);
-            mbar_init(&kv_empty[s], 1);
+            mbar_init(&kv_empty[s], C::ISSUERS);   // one commit per MMA issuer
         }
         for (int w = 0; w < 2; ++w) {
             mbar_init(&s_full[w], 1);
+            mbar_init(&s_free[w], 4);
             mbar_init(&p_full[w], 4);
+            mbar_init(&p_free[w], 1);
             mbar_init(&o_final[w], 1);
         }
-        mbar_init(mma_done, 1);
+        mbar_init(mma_done, C::ISSUERS);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -149,7 +174,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 }
             }
         }
-    } else if (warp == 1) {
+    } else if (warp == 1 || (C::P_SEP && warp == 10)) {
         if (lane == 0) {
             constexpr uint32_t idesc_s = idesc_bf16(BQ, BKV);
             constexpr uint32_t idesc_o = idesc_bf16(BQ, D);
@@ -157,7 +182,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             bool ok = mbar_wait(q_full, 0, abort_flag, g.err);
             int stage = 0, prev = 0;
             uint32_t phase = 0;
-            // S(t) = Q(t) K^T into TMEM columns [128 t, 128 t + 128)
+            // S(t) = Q(t) K^T into TMEM (128 fp32 columns)
             auto issue_s = [&](int t, int st) {
                 const uint32_t kb = smem_u32(skv + st * C::STAGE);
                 const uint32_t qb = sq0 + t * C::Q_TILE;
@@ -165,42 +190,75 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 for (int ks = 0; ks < D / 16; ++ks) {
                     const uint32_t off = (ks >> 2) * (BQ * 128) + (ks & 3) * 32;
                     const uint32_t koff = (ks >> 2) * (BKV * 128) + (ks & 3) * 32;
-                    tc_mma(tmem + t * 128, sdesc_sw128(qb + off), sdesc_sw128(kb + koff), idesc_s, ks != 0);
+                    tc_mma(tmem + C::s_col(t), sdesc_sw128(qb + off), sdesc_sw128(kb + koff), idesc_s, ks != 0);
                 }
             };
-            // O(t) (+)= P(t) V: A = P in TMEM (bf16 pairs over S(t)'s first 64 columns)
+            // O(t) (+)= P(t) V, A = P in TMEM (16 bf16 = 8 columns per K step)
             auto issue_pv = [&](int t, int st, bool acc) {
                 const uint32_t vb = smem_u32(skv + st * C::STAGE + C::K_TILE);
 #pragma unroll
                 for (int ks = 0; ks < BKV / 16; ++ks) {
                     const uint32_t voff = (ks >> 2) * (D * 128) + (ks & 3) * 32;
-                    tc_mma_ts(tmem + C::TMEM_O + t * D, tmem + t * 128 + ks * 8, sdesc_sw128(vb + voff), idesc_o,
+                    tc_mma_ts(tmem + C::o_col(t), tmem + C::p_col(t) + ks * 8, sdesc_sw128(vb + voff), idesc_o,
                               (acc || ks != 0) ? 1u : 0u);
                 }
             };
-            for (int j = 0; j < n_kv && ok; ++j) {
-                if (!mbar_wait(&kv_full[stage], phase, abort_flag, g.err)) { ok = false; break; }
-                tc_fence_after();
-                for (int t = 0; t < 2; ++t) {
+            if constexpr (C::P_SEP) {
+                // this thread issues the MMAs of query tile t only; the other
+                // tile has its own issuer, so neither waits behind the other's
+                // softmax
+                const int t = (warp == 1) ? 0 : 1;
+                for (int j = 0; j < n_kv && ok; ++j) {
+                    if (!mbar_wait(&kv_full[stage], phase, abort_flag, g.err)) { ok = false; break; }
+                    tc_fence_after();
+                    if (j > 0) {
+                        if (!mbar_wait(&s_free[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
+                        tc_fence_after();
+                    }
+                    issue_s(t, stage);
+                    tc_commit(&s_full[t]);
                     if (j > 0) {
                         if (!mbar_wait(&p_full[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
                         tc_fence_after();
                         issue_pv(t, prev, j > 1);
-                        if (t == 1) tc_commit(&kv_empty[prev]);
+                        tc_commit(&p_free[t]);
+                        tc_commit(&kv_empty[prev]);
                     }
-                    issue_s(t, stage);
-                    tc_commit(&s_full[t]);
+                    prev = stage;
+                    if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
                 }
-                prev = stage;
-                if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
-            }
-            if (ok) {
-                for (int t = 0; t < 2; ++t) {
-                    if (!mbar_wait(&p_full[t], (n_kv - 1) & 1, abort_flag, g.err)) break;
+                if (ok && mbar_wait(&p_full[t], (n_kv - 1) & 1, abort_flag, g.err)) {
                     tc_fence_after();
                     issue_pv(t, prev, n_kv > 1);
-                    if (t == 1) tc_commit(&kv_empty[prev]);
+                    tc_commit(&kv_empty[prev]);
                     tc_commit(&o_final[t]);
+                }
+            } else {
+                // one issuer interleaving both tiles: PV0(j-1), S0(j), PV1(j-1), S1(j)
+                for (int j = 0; j < n_kv && ok; ++j) {
+                    if (!mbar_wait(&kv_full[stage], phase, abort_flag, g.err)) { ok = false; break; }
+                    tc_fence_after();
+                    for (int t = 0; t < 2; ++t) {
+                        if (j > 0) {
+                            if (!mbar_wait(&p_full[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
+                            tc_fence_after();
+                            issue_pv(t, prev, j > 1);
+                            if (t == 1) tc_commit(&kv_empty[prev]);
+                        }
+                        issue_s(t, stage);
+                        tc_commit(&s_full[t]);
+                    }
+                    prev = stage;
+                    if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
+                }
+                if (ok) {
+                    for (int t = 0; t < 2; ++t) {
+                        if (!mbar_wait(&p_full[t], (n_kv - 1) & 1, abort_flag, g.err)) break;
+                        tc_fence_after();
+                        issue_pv(t, prev, n_kv > 1);
+                        if (t == 1) tc_commit(&kv_empty[prev]);
+                        tc_commit(&o_final[t]);
+                    }
                 }
             }
             tc_commit(mma_done);
@@ -214,8 +272,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const int quarter = warp & 3;
         const int row = quarter * 32 + lane;                 // row within the tile = TMEM lane
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-        const uint32_t s_addr = tmem + lane_base + (uint32_t)(t * 128);
-        const uint32_t o_addr = tmem + lane_base + C::TMEM_O + (uint32_t)(t * D);
+        const uint32_t s_addr = tmem + lane_base + C::s_col(t);
+        const uint32_t p_addr = tmem + lane_base + C::p_col(t);
+        const uint32_t o_addr = tmem + lane_base + C::o_col(t);
         const int last_valid = g.L - (n_kv - 1) * BKV;       // keys in the last tile
         float m_run = -INFINITY, l_run = 0.f;
         bool ok = true;
@@ -226,29 +285,58 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 #pragma unroll
             for (int c = 0; c < BKV / 32; ++c) tmem_ld32(s_addr + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&s[c * 32]));
             tmem_ld_wait();
+            if constexpr (C::P_SEP) {
+                // S(t) is in registers: the MMA may compute S(t, j+1) now
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&s_free[t]);
+            }
             if (j == n_kv - 1 && last_valid < BKV) {
 #pragma unroll
                 for (int c = 0; c < BKV; ++c)
                     if (c >= last_valid) s[c] = -INFINITY;
             }
-            float mx = s[0];
+            // row max with 8 independent partial maxima (short dependency chains)
+            float m8[8];
 #pragma unroll
-            for (int c = 1; c < BKV; ++c) mx = fmaxf(mx, s[c]);
-            const float m_new = fmaxf(m_run, mx * g.scale_log2);
-            const float corr = ex2(m_run - m_new);
-            float sum = 0.f;
+            for (int i = 0; i < 8; ++i) m8[i] = fmaxf(s[i], s[8 + i]);
+#pragma unroll
+            for (int c = 16; c < BKV; c += 16)
+#pragma unroll
+                for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], s[c + i], s[c + 8 + i]);
+            const float mx = fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
+            // The exponent base only moves when the running max grows by more
+            // than 8 (a factor 256): O and l share the same base, so the result
+            // is unchanged, and most tiles skip the O rescale in TMEM.
+            const float m_cand = fmaxf(m_run, mx * g.scale_log2);
+            const bool grow = m_cand - m_run > 8.0f;
+            const float m_use = grow ? m_cand : m_run;
+            const float corr = grow ? ex2(m_run - m_cand) : 1.0f;
+            float sum8[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) sum8[i] = 0.f;
             uint32_t p[BKV / 2];
+            const float nm = -m_use;
 #pragma unroll
             for (int c = 0; c < BKV; c += 2) {
-                const float a = ex2(fmaf(s[c], g.scale_log2, -m_new));
-                const float b = ex2(fmaf(s[c + 1], g.scale_log2, -m_new));
-                sum += a + b;
+                const float a = ex2(fmaf(s[c], g.scale_log2, nm));
+                const float b = ex2(fmaf(s[c + 1], g.scale_log2, nm));
+                sum8[c & 7] += a;
+                sum8[(c + 1) & 7] += b;
                 p[c / 2] = pack2(a, b);
             }
+            const float sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
             l_run = l_run * corr + sum;
-            m_run = m_new;
-            if (j > 0 && __any_sync(0xffffffffu, corr < 1.0f)) {
-                // PV(j-1) of this tile completed before S(j) was committed: rescale O in place
+            m_run = m_use;
+            if constexpr (C::P_SEP) {
+                // PV(t, j-1) must be done before P(t) is overwritten and O(t) rescaled
+                if (j > 0) {
+                    if (!mbar_wait(&p_free[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
+                    tc_fence_after();
+                }
+            }
+            if (j > 0 && __any_sync(0xffffffffu, grow)) {
+                // PV(t, j-1) is complete (p_free, or the commit after S(t, j)): rescale O in place
 #pragma unroll
                 for (int c = 0; c < D; c += 32) {
                     uint32_t o[32];
@@ -264,9 +352,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     tmem_st16(o_addr + c + 16, hi);
                 }
             }
-            // P over the first 64 columns of S(t)
+            // P (64 columns of bf16 pairs)
 #pragma unroll
-            for (int c = 0; c < BKV / 2; c += 16) tmem_st16(s_addr + c, *reinterpret_cast<uint32_t(*)[16]>(&p[c]));
+            for (int c = 0; c < BKV / 2; c += 16) tmem_st16(p_addr + c, *reinterpret_cast<uint32_t(*)[16]>(&p[c]));
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
@@ -327,7 +415,7 @@ wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o,
     g.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
     g.o = reinterpret_cast<__nv_bfloat16*>(o);
     g.err = c->err;
-    attn_tc_kernel<D><<<H * g.q_blocks, kAttnThreads, Cf::SMEM, s>>>(tq, tk, tv, g);
+    attn_tc_kernel<D><<<H * g.q_blocks, Cf::THREADS, Cf::SMEM, s>>>(tq, tk, tv, g);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 attention launch: ") + cudaGetErrorString(e));
     return WDC_OK;

@@ -16,6 +16,7 @@
 
 #include <cmath>
 #include <cstring>
+#include <type_traits>
 #include <vector>
 
 namespace wdc {
@@ -114,6 +115,65 @@ __global__ void ln_mod_kernel(const T* __restrict__ x, T* __restrict__ h, int r0
     for (int i = 0; i < VPT; ++i) {
         const int c = lane + 32 * i;
         if (c < D) hr[c] = to_act<T>(fmaf((v[i] - mean) * rstd, 1.0f + scale[c], shift[c]));
+    }
+}
+
+// bf16 variant with 16-byte accesses: lane l owns the 8-element vectors
+// l, l+32, ..., so a warp moves 512 contiguous bytes per access (D % 256 == 0).
+template <int NV>
+__global__ void ln_mod_vec_kernel(const __nv_bfloat16* __restrict__ x, __nv_bfloat16* __restrict__ h, int r0, int r1,
+                                  int D, const float* __restrict__ shift, const float* __restrict__ scale,
+                                  int h_row_off) {
+    const int row = r0 + ((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    if (row >= r1) return;
+    const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)row * D);
+    float v[NV][8];
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const uint4 u = __ldg(xr + i * 32 + lane);
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[q]));
+            v[i][2 * q] = f.x;
+            v[i][2 * q + 1] = f.y;
+            s += f.x + f.y;
+        }
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const float mean = s / (float)D;
+    float q2 = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV; ++i)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const float dlt = v[i][e] - mean;
+            q2 += dlt * dlt;
+        }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) q2 += __shfl_xor_sync(0xffffffffu, q2, o);
+    const float rstd = 1.0f / sqrtf(q2 / (float)D + 1e-6f);
+    uint4* hr = reinterpret_cast<uint4*>(h + (size_t)(row - h_row_off) * D);
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const int c0 = (i * 32 + lane) * 8;
+        const float4 sc0 = __ldg(reinterpret_cast<const float4*>(scale + c0));
+        const float4 sc1 = __ldg(reinterpret_cast<const float4*>(scale + c0 + 4));
+        const float4 sh0 = __ldg(reinterpret_cast<const float4*>(shift + c0));
+        const float4 sh1 = __ldg(reinterpret_cast<const float4*>(shift + c0 + 4));
+        const float sc[8] = {sc0.x, sc0.y, sc0.z, sc0.w, sc1.x, sc1.y, sc1.z, sc1.w};
+        const float sh[8] = {sh0.x, sh0.y, sh0.z, sh0.w, sh1.x, sh1.y, sh1.z, sh1.w};
+        uint32_t w[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float a = fmaf((v[i][2 * q] - mean) * rstd, 1.0f + sc[2 * q], sh[2 * q]);
+            const float b = fmaf((v[i][2 * q + 1] - mean) * rstd, 1.0f + sc[2 * q + 1], sh[2 * q + 1]);
+            __nv_bfloat162 hb = __floats2bfloat162_rn(a, b);
+            w[q] = *reinterpret_cast<uint32_t*>(&hb);
+        }
+        hr[i * 32 + lane] = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
@@ -290,6 +350,14 @@ void launch_ln_mod(const void* x, void* h, int r0, int r1, int D, const float* s
     const unsigned grid = blocks_for((long long)rows * 32, 256);
     const T* xp = reinterpret_cast<const T*>(x);
     T* hp = reinterpret_cast<T*>(h);
+    if constexpr (std::is_same<T, __nv_bfloat16>::value) {
+        const bool vec_ok = D % 256 == 0 && ((uintptr_t)x & 15) == 0 && ((uintptr_t)h & 15) == 0 &&
+                            ((uintptr_t)shift & 15) == 0 && ((uintptr_t)scale & 15) == 0;
+        if (vec_ok && D == 3072) {
+            ln_mod_vec_kernel<12><<<grid, 256, 0, s>>>(xp, hp, r0, r1, D, shift, scale, h_row_off);
+            return;
+        }
+    }
     if (D <= 256) ln_mod_kernel<T, 8><<<grid, 256, 0, s>>>(xp, hp, r0, r1, D, shift, scale, h_row_off);
     else if (D <= 1024) ln_mod_kernel<T, 32><<<grid, 256, 0, s>>>(xp, hp, r0, r1, D, shift, scale, h_row_off);
     else ln_mod_kernel<T, 128><<<grid, 256, 0, s>>>(xp, hp, r0, r1, D, shift, scale, h_row_off);
