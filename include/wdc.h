@@ -180,6 +180,10 @@ const char* wdc_last_error(const wdc_ctx* ctx);
 size_t wdc_latent_numel(const wdc_ctx* ctx);
 /* Number of kernels this context has launched so far (all streams). */
 unsigned long long wdc_launch_count(const wdc_ctx* ctx);
+/* Synchronises the device and returns (then clears) the bits the kernels have
+ * set in the context's error word: 1 = a bounded device-side wait timed out,
+ * 4 = the two CTAs of a tensor-core pair saw different tensor-memory bases. */
+wdc_status wdc_device_errors(wdc_ctx* ctx, unsigned* bits);
 
 /* ------------------------------------------------------------------ weights */
 /* Copies one parameter tensor (host fp32, `count` elements, shape as listed in

@@ -333,6 +333,16 @@ size_t wdc_latent_numel(const wdc_ctx* h) {
     return c ? c->n : 0;
 }
 
+wdc_status wdc_device_errors(wdc_ctx* h, unsigned* bits) {
+    Ctx* c = reinterpret_cast<Ctx*>(h);
+    if (!c || !bits) return WDC_ERR_INVALID_ARG;
+    cudaSetDevice(c->device);
+    WDC_CUDA_TRY(c, cudaDeviceSynchronize());
+    WDC_CUDA_TRY(c, cudaMemcpy(bits, c->err, sizeof(unsigned), cudaMemcpyDeviceToHost));
+    WDC_CUDA_TRY(c, cudaMemset(c->err, 0, sizeof(unsigned)));
+    return WDC_OK;
+}
+
 wdc_status wdc_profile_enable(wdc_ctx* h, int on) {
     Ctx* c = reinterpret_cast<Ctx*>(h);
     if (!c) return WDC_ERR_INVALID_ARG;

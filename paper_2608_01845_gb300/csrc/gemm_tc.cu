@@ -279,6 +279,179 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
 }
 
+// ---------------------------------------------------------------------------
+// CTA-pair variant (clusters of 2, tcgen05 .cta_group::2): each pair computes a
+// 256 x 256 tile with 256 x 256 x 16 MMAs issued by the even CTA; each CTA
+// holds its 128 rows of A and its 128-row half of the W tile (32 KB per stage,
+// 6 stages), so twice the MMA work is buffered per shared-memory byte.  Both
+// CTAs' tile copies complete on the even CTA's mbarrier (the pair form of the
+// tensor copy), which the even CTA arms with both CTAs' bytes; the even CTA's
+// commits release both CTAs' stages and accumulators.  The
+// pair allocation is collective (both CTAs receive the same TMEM base; the
+// leader's base is used for every access and a mismatch is reported), and two
+// 256-column accumulators let a tile's epilogue overlap the next tile's MMAs.
+constexpr int STAGES2 = 6;
+constexpr uint32_t A2_BYTES = 128 * BK * 2;
+constexpr uint32_t B2_BYTES = 128 * BK * 2;                  // half of the 256-row W tile
+constexpr uint32_t STAGE2_BYTES = A2_BYTES + B2_BYTES;
+constexpr uint32_t TMEM2_COLS = 512;
+constexpr uint32_t IDESC2 = idesc_bf16(256, 256);
+constexpr size_t SMEM2_BYTES = STAGES2 * STAGE2_BYTES + 1024 + 512;
+
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const __grid_constant__ GemmArgs g) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES2 * STAGE2_BYTES);   // even CTA: both halves landed
+    uint64_t* empty = full + STAGES2;
+    uint64_t* tfull = empty + STAGES2;         // [2]
+    uint64_t* tempty = tfull + 2;              // [2] even CTA: both CTAs' epilogues are done
+    uint64_t* mma_done = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const int cluster_id = blockIdx.x >> 1, n_clusters = gridDim.x >> 1;
+    const int m_pairs = (g.m_tiles + 1) >> 1;  // 256-row tiles (m_tiles counts 128-row tiles)
+    const int num_tiles = m_pairs * g.n_tiles;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES2; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], 8);          // 4 epilogue warps in each CTA
+        }
+        mbar_init(mma_done, 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 0 && lane == 0) {
+        prefetch_tmap(&tmA);
+        prefetch_tmap(&tmB);
+    }
+    if (warp == 1) {
+        tmem_alloc2(tmem_slot, TMEM2_COLS);
+        tmem_relinquish2();
+    }
+    __syncthreads();
+    cluster_sync_all();
+    tc_fence_after();
+    const uint32_t own_base = *tmem_slot;
+    const uint32_t tmem = rank == 0 ? own_base : ld_shared_cluster_u32(mapa_shared(smem_u32(tmem_slot), 0));
+    if (threadIdx.x == 0 && tmem != own_base) atomicOr(g.err, kErrTmem);
+    const uint32_t leader_tempty0 = mapa_shared(smem_u32(&tempty[0]), 0);
+    const uint32_t leader_tempty1 = mapa_shared(smem_u32(&tempty[1]), 0);
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t armed_phase[STAGES2];
+            bool armed[STAGES2];
+            for (int s = 0; s < STAGES2; ++s) armed[s] = false;
+            bool ok = true;
+            for (int tile = cluster_id; tile < num_tiles && ok; tile += n_clusters) {
+                const int m0 = (tile % m_pairs) * 256 + (int)rank * 128;
+                const int n0 = (tile / m_pairs) * BN + (int)rank * 128;
+                for (int kb = 0; kb < g.k_blocks; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
+                    if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * STAGE2_BYTES);
+                    const uint32_t fb = mapa_shared(smem_u32(&full[stage]), 0);
+                    uint8_t* sa = smem + stage * STAGE2_BYTES;
+                    tma_load_2d_pair(sa, &tmA, fb, kb * BK, m0);
+                    tma_load_2d_pair(sa + A2_BYTES, &tmB, fb, kb * BK, n0);
+                    armed[stage] = true;
+                    armed_phase[stage] = phase;
+                    if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
+                }
+            }
+            // drain: every copy of the pair has landed (even CTA's full) and the
+            // MMAs have released every stage (both CTAs' empty)
+            for (int s = 0; s < STAGES2; ++s) {
+                if (!armed[s]) continue;
+                if (rank == 0) {
+                    const unsigned long long t0 = globaltimer();
+                    while (!mbar_try_wait(&full[s], armed_phase[s]) && globaltimer() - t0 < kWaitLimitNs) {
+                    }
+                }
+                const unsigned long long t1 = globaltimer();
+                while (!mbar_try_wait(&empty[s], armed_phase[s]) && globaltimer() - t1 < kWaitLimitNs) {
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && rank == 0) {
+            // MMA issuer for the pair
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            for (int tile = cluster_id; tile < num_tiles && ok; tile += n_clusters) {
+                if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, g.err)) break;
+                tc_fence_after();
+                const uint32_t d = tmem + (uint32_t)(acc * BN);
+                for (int kb = 0; kb < g.k_blocks; ++kb) {
+                    if (!mbar_wait(&full[stage], phase, abort_flag, g.err)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t a0 = smem_u32(smem + stage * STAGE2_BYTES);
+                    const uint32_t b0 = a0 + A2_BYTES;
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k)
+                        tc_mma2(d, sdesc_sw128(a0 + k * 32), sdesc_sw128(b0 + k * 32), IDESC2, (kb | k) != 0);
+                    tc_commit2_mc(&empty[stage], (uint16_t)0x3);
+                    if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
+                }
+                tc_commit2_mc(&tfull[acc], (uint16_t)0x3);
+                acc ^= 1;
+                if (acc == 0) acc_phase ^= 1u;
+            }
+            tc_commit2_mc(mma_done, (uint16_t)0x1);
+            const unsigned long long t0 = globaltimer();
+            while (!mbar_try_wait(mma_done, 0) && globaltimer() - t0 < kWaitLimitNs) {
+            }
+        }
+    } else {
+        const int lg = warp & 3;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = cluster_id; tile < num_tiles; tile += n_clusters) {
+            const int mrow = (tile % m_pairs) * 256 + (int)rank * 128;
+            const int n_blk = tile / m_pairs;
+            if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, g.err)) break;
+            tc_fence_after();
+            const int m = mrow + lg * 32 + lane;
+            const uint32_t taddr = tmem + ((uint32_t)(lg * 32) << 16) + (uint32_t)(acc * BN);
+            for (int c0 = 0; c0 < BN; c0 += 32) {
+                const int col0 = n_blk * BN + c0;
+                if (col0 >= g.N) break;
+                uint32_t r[32];
+                tmem_ld32(taddr + c0, r);
+                tmem_ld_wait();
+                if (m < g.M) epilogue_chunk(g.e, m, col0, r);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                if (rank == 0) mbar_arrive(&tempty[acc]);
+                else mbar_arrive_remote(acc == 0 ? leader_tempty0 : leader_tempty1);
+            }
+            acc ^= 1;
+            if (acc == 0) acc_phase ^= 1u;
+        }
+    }
+    __syncthreads();
+    cluster_sync_all();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc2(own_base, TMEM2_COLS);
+    }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     static std::once_flag once;
@@ -340,12 +513,14 @@ wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, co
     static bool attr_set = false;
     if (!attr_set) {
         cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+        cudaFuncSetAttribute(gemm_tc2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM2_BYTES);
         attr_set = true;
     }
+    const bool pair = M >= 256 && c->num_sms >= 2;
     CUtensorMap ta, tb;
     std::string why;
     if (!encode_tmap_2d(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, BK, BM, &why) ||
-        !encode_tmap_2d(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, BK, BN, &why))
+        !encode_tmap_2d(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, BK, pair ? BN / 2 : BN, &why))
         return fail(c, WDC_ERR_CUDA, why);
     GemmArgs g;
     g.M = M;
@@ -356,9 +531,37 @@ wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, co
     g.k_blocks = (K + BK - 1) / BK;
     g.e = e;
     g.err = c->err;
-    const int tiles = g.m_tiles * g.n_tiles;
-    const int grid = tiles < c->num_sms ? tiles : c->num_sms;
-    gemm_tc_kernel<<<grid, kGemmThreads, SMEM_BYTES, s>>>(ta, tb, g);
+    if (pair) {
+        const int tiles = ((g.m_tiles + 1) / 2) * g.n_tiles;
+        cudaLaunchConfig_t cfg = {};
+        cfg.blockDim = dim3(kGemmThreads, 1, 1);
+        cfg.dynamicSmemBytes = SMEM2_BYTES;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        // persistent grid: only as many pairs as can be resident at once
+        static int max_clusters = 0;
+        if (max_clusters == 0) {
+            cfg.gridDim = dim3(c->num_sms, 1, 1);
+            if (cudaOccupancyMaxActiveClusters(&max_clusters, gemm_tc2_kernel, &cfg) != cudaSuccess || max_clusters < 1) {
+                cudaGetLastError();
+                max_clusters = c->num_sms / 2;
+            }
+        }
+        int clusters = max_clusters < c->num_sms / 2 ? max_clusters : c->num_sms / 2;
+        if (tiles < clusters) clusters = tiles;
+        cfg.gridDim = dim3(2 * clusters, 1, 1);
+        cudaLaunchKernelEx(&cfg, gemm_tc2_kernel, ta, tb, g);
+    } else {
+        const int tiles = g.m_tiles * g.n_tiles;
+        const int grid = tiles < c->num_sms ? tiles : c->num_sms;
+        gemm_tc_kernel<<<grid, kGemmThreads, SMEM_BYTES, s>>>(ta, tb, g);
+    }
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(err));
     return WDC_OK;

@@ -105,6 +105,7 @@ def _load():
         "wdc_destroy": (None, [P]),
         "wdc_set_cache_params": (I, [P, ctypes.POINTER(CacheParams)]),
         "wdc_profile_enable": (I, [P, I]),
+        "wdc_device_errors": (I, [P, ctypes.POINTER(ctypes.c_uint)]),
         "wdc_profile_read": (I, [P, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_ulonglong)]),
         "wdc_last_error": (ctypes.c_char_p, [P]),
         "wdc_latent_numel": (S, [P]),
@@ -221,6 +222,12 @@ class Context:
     def set_cache_params(self, params):
         self._check(LIB.wdc_set_cache_params(self._h, ctypes.byref(params)), "set_cache_params")
         self.params = params
+
+    def device_errors(self):
+        """Error bits set by kernels since the last call (1 timeout, 4 TMEM pair mismatch)."""
+        b = ctypes.c_uint()
+        self._check(LIB.wdc_device_errors(self._h, ctypes.byref(b)), "device_errors")
+        return b.value
 
     def profile_enable(self, on=True):
         self._check(LIB.wdc_profile_enable(self._h, int(on)), "profile_enable")

@@ -169,3 +169,21 @@ def test_bf16_attention_full_size_sampled_rows(H, L, d):
     for h in range(0, H, 7):
         want = dit.attention(q[h, rows].astype(np.float64), k[h].astype(np.float64), v[h].astype(np.float64), 1)
         assert rel_l2(got[rows, h * d:(h + 1) * d], want) <= 1e-2, h
+
+
+@pytest.mark.parametrize("M,N,K", [(17776, 9216, 3072), (1000, 768, 1024)])
+def test_bf16_gemm_sampled_full_size_and_no_device_errors(M, N, K):
+    """Full 5B-scale QKV shape (the CTA-pair kernel) checked on 64 sampled rows;
+    no kernel reported a timeout or a tensor-memory pair mismatch."""
+    ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
+    g = np.random.default_rng(55)
+    A = _bf(g.standard_normal((M, K), dtype=np.float32))
+    W = _bf(0.05 * g.standard_normal((N, K), dtype=np.float32))
+    C = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    ctx.op_gemm(_to_dev(A, torch.bfloat16), _to_dev(W, torch.bfloat16), C)
+    torch.cuda.synchronize()
+    rows = np.sort(g.choice(M, 64, replace=False))
+    rows[-1] = M - 1
+    want = A[rows].astype(np.float64) @ W.astype(np.float64).T
+    assert rel_l2(C.float().cpu().numpy()[rows], want) <= 1e-2
+    assert ctx.device_errors() == 0
