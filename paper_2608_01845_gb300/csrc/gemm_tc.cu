@@ -14,6 +14,8 @@
 //               32-lane TMEM quarter = 32 rows), bias / GELU / gated residual /
 //               QKV scatter / unpatchify, 16-byte global stores; then release
 //               the accumulator so the next tile's MMAs overlap this epilogue.
+// Tiles are visited with N fastest: the W matrix (at most 75 MB here) stays
+// in L2 while A and the output stream through once.
 // Tails: TMA zero-fills rows past M / N and columns past K; the epilogue
 // masks rows >= M.  Every mbarrier wait is bounded.
 #include "dit_kernels.cuh"
@@ -195,7 +197,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             for (int s = 0; s < STAGES; ++s) armed[s] = false;
             bool ok = true;
             for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-                const int m_blk = tile % g.m_tiles, n_blk = tile / g.m_tiles;
+                const int m_blk = tile / g.n_tiles, n_blk = tile % g.n_tiles;
                 for (int kb = 0; kb < g.k_blocks; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
                     mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
@@ -252,7 +254,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
-            const int m_blk = tile % g.m_tiles, n_blk = tile / g.m_tiles;
+            const int m_blk = tile / g.n_tiles, n_blk = tile % g.n_tiles;
             if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, g.err)) break;
             tc_fence_after();
             const int m = m_blk * BM + lg * 32 + lane;
@@ -290,7 +292,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 // pair allocation is collective (both CTAs receive the same TMEM base; the
 // leader's base is used for every access and a mismatch is reported), and two
 // 256-column accumulators let a tile's epilogue overlap the next tile's MMAs.
-constexpr int STAGES2 = 6;
+constexpr int STAGES2 = 7;
 constexpr uint32_t A2_BYTES = 128 * BK * 2;
 constexpr uint32_t B2_BYTES = 128 * BK * 2;                  // half of the 256-row W tile
 constexpr uint32_t STAGE2_BYTES = A2_BYTES + B2_BYTES;
@@ -355,8 +357,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             for (int s = 0; s < STAGES2; ++s) armed[s] = false;
             bool ok = true;
             for (int tile = cluster_id; tile < num_tiles && ok; tile += n_clusters) {
-                const int m0 = (tile % m_pairs) * 256 + (int)rank * 128;
-                const int n0 = (tile / m_pairs) * BN + (int)rank * 128;
+                const int m0 = (tile / g.n_tiles) * 256 + (int)rank * 128;
+                const int n0 = (tile % g.n_tiles) * BN + (int)rank * 128;
                 for (int kb = 0; kb < g.k_blocks; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
                     if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * STAGE2_BYTES);
@@ -420,8 +422,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int tile = cluster_id; tile < num_tiles; tile += n_clusters) {
-            const int mrow = (tile % m_pairs) * 256 + (int)rank * 128;
-            const int n_blk = tile / m_pairs;
+            const int mrow = (tile / g.n_tiles) * 256 + (int)rank * 128;
+            const int n_blk = tile % g.n_tiles;
             if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, g.err)) break;
             tc_fence_after();
             const int m = mrow + lg * 32 + lane;
