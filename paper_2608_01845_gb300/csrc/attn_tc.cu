@@ -82,11 +82,46 @@ __device__ __forceinline__ uint32_t pack2(float a, float b) {
     return *reinterpret_cast<uint32_t*>(&h);
 }
 
+// Two f32 values as one paired-fp32 operand (lo = a, hi = b).
+__device__ __forceinline__ uint64_t pair(float a, float b) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+// Two softmax numerators in paired-fp32 form: x = s * scale + nm for both
+// (one fma.f32x2), 2^x, their running row sums acc += (a, b) (one
+// add.f32x2) and the packed bf16 pair of P (lo = first key).
+__device__ __forceinline__ uint32_t exp2_pair(float s0, float s1, uint64_t scale2, uint64_t nm2, uint64_t& acc) {
+    uint32_t p;
+    asm("{\n .reg .b64 x, e;\n .reg .f32 a, b;\n"
+        " mov.b64 x, {%2, %3};\n"
+        " fma.rn.f32x2 x, x, %4, %5;\n"
+        " mov.b64 {a, b}, x;\n"
+        " ex2.approx.ftz.f32 a, a;\n"
+        " ex2.approx.ftz.f32 b, b;\n"
+        " mov.b64 e, {a, b};\n"
+        " add.rn.f32x2 %1, %1, e;\n"
+        " cvt.rn.bf16x2.f32 %0, b, a;\n}"
+        : "=r"(p), "+l"(acc)
+        : "f"(s0), "f"(s1), "l"(scale2), "l"(nm2));
+    return p;
+}
+
+__device__ __forceinline__ float pair_sum(uint64_t v) {
+    float a, b;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+    return a + b;
+}
+
 template <int D>
 __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
                    const __grid_constant__ CUtensorMap tv, const __grid_constant__ AttnArgs g) {
     using C = AttnCfg<D>;
+    // paired-fp32 numerators (fma.f32x2 / add.f32x2) measured faster at
+    // d = 128 and slower at d = 64
+    constexpr bool kPairedExp = D == 128;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sq = smem;                                       // [2 tiles][ATOMS][128 x 128 B]
@@ -277,6 +312,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
         const uint32_t o_addr = tmem + lane_base + C::o_col(t);
         const int last_valid = g.L - (n_kv - 1) * BKV;       // keys in the last tile
         float m_run = -INFINITY, l_run = 0.f;
+        const uint64_t scale2 = pair(g.scale_log2, g.scale_log2);
         bool ok = true;
         for (int j = 0; j < n_kv; ++j) {
             if (!mbar_wait(&s_full[t], j & 1, abort_flag, g.err)) { ok = false; break; }
@@ -312,20 +348,32 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
             const bool grow = m_cand - m_run > 8.0f;
             const float m_use = grow ? m_cand : m_run;
             const float corr = grow ? ex2(m_run - m_cand) : 1.0f;
-            float sum8[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) sum8[i] = 0.f;
             uint32_t p[BKV / 2];
-            const float nm = -m_use;
+            float sum;
+            if constexpr (kPairedExp) {
+                // 2^(s * scale - m) in paired-fp32 form; 8 partial sums (4 pairs)
+                uint64_t sum4[4];
 #pragma unroll
-            for (int c = 0; c < BKV; c += 2) {
-                const float a = ex2(fmaf(s[c], g.scale_log2, nm));
-                const float b = ex2(fmaf(s[c + 1], g.scale_log2, nm));
-                sum8[c & 7] += a;
-                sum8[(c + 1) & 7] += b;
-                p[c / 2] = pack2(a, b);
+                for (int i = 0; i < 4; ++i) sum4[i] = 0ull;
+                const uint64_t nm2 = pair(-m_use, -m_use);
+#pragma unroll
+                for (int c = 0; c < BKV; c += 2) p[c / 2] = exp2_pair(s[c], s[c + 1], scale2, nm2, sum4[(c / 2) & 3]);
+                sum = (pair_sum(sum4[0]) + pair_sum(sum4[1])) + (pair_sum(sum4[2]) + pair_sum(sum4[3]));
+            } else {
+                float sum8[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) sum8[i] = 0.f;
+                const float nm = -m_use;
+#pragma unroll
+                for (int c = 0; c < BKV; c += 2) {
+                    const float a = ex2(fmaf(s[c], g.scale_log2, nm));
+                    const float b = ex2(fmaf(s[c + 1], g.scale_log2, nm));
+                    sum8[c & 7] += a;
+                    sum8[(c + 1) & 7] += b;
+                    p[c / 2] = pack2(a, b);
+                }
+                sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
             }
-            const float sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
             l_run = l_run * corr + sum;
             m_run = m_use;
             if constexpr (C::P_SEP) {
