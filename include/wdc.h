@@ -96,8 +96,46 @@ typedef struct wdc_cache_params {
     double lambda_, tau_risk;                     /* decay and threshold (Eq. 9-10) */
     int max_age;                /* pre-decision anchor age limit (Eq. 10 text)   */
     int n_init_exact, n_final_exact;              /* mandatory-exact phases      */
-    int flags;                  /* reserved, must be 0                           */
+    int flags;                  /* WDC_ABL_* ablation bits; 0 = the full method  */
+    int period;                 /* WDC_ABL_PERIODIC: exact step every `period`   */
+    double ridge;               /* WDC_ABL_LINEAR_OBS: relative ridge            */
 } wdc_cache_params;
+
+/* Ablation variants (section "Ablation Study", Tables 3 and 4), bits of
+ * wdc_cache_params.flags.  The paper names them and defers their definitions
+ * to supplementary material; these are this library's readings.  Any
+ * combination is accepted (WDC_ABL_SECANT makes WDC_ABL_LINEAR_OBS and
+ * WDC_ABL_NO_SUPPORT moot: the secant uses no retrieval or observation).
+ *   PERIODIC      Eq. 10's risk test replaced by a fixed period: Surrogate iff
+ *                 Available_t and age_t + 1 < period (Available_t kept).
+ *   SECANT        native latent secant candidate z_hat = z_t + alpha_t
+ *                 (z_a - z_a,in): the latest exact displacement scaled by
+ *                 Eq. 4's alpha; its support term holds whenever the bank is
+ *                 non-empty.  The context keeps that displacement (one more
+ *                 latent-sized buffer, written by the exact-step pass).
+ *   INSTANT_RISK  instantaneous risk: lambda = 0 in Eq. 9 (R_cand = Delta_t).
+ *   NO_IMPACT     w/o impact weighting: w_t = 1 in Eq. 9.
+ *   NO_CALIB      w/o counterfactual calibration: eta_d stays eta_init (d_cf
+ *                 is still measured and reported).
+ *   NO_SUPPORT    w/o support constraint: retrieval over the whole bank (no
+ *                 compatibility filter); the support term always holds.
+ *   LINEAR_OBS    linear observation: Eq. 5's softmax weights replaced by the
+ *                 ridge least-squares coefficients beta of s(phi_hat) on the
+ *                 records' output summaries, (G + rho I) beta = S_out s_hat,
+ *                 G_ij = s_out_i . s_out_j, rho = ridge * trace(G) / n_bank;
+ *                 z_hat = sum_i beta_i z_out_i.
+ *   NO_COND       condition descriptors left out of the lift (Eq. 2): the
+ *                 camera / depth entries of every summary are zero; the
+ *                 controller (Eq. 6, 9) still uses them. */
+#define WDC_ABL_PERIODIC     0x01
+#define WDC_ABL_SECANT       0x02
+#define WDC_ABL_INSTANT_RISK 0x04
+#define WDC_ABL_NO_IMPACT    0x08
+#define WDC_ABL_NO_CALIB     0x10
+#define WDC_ABL_NO_SUPPORT   0x20
+#define WDC_ABL_LINEAR_OBS   0x40
+#define WDC_ABL_NO_COND      0x80
+#define WDC_ABL_ALL          0xFF
 
 /* Model condition c of one step.  tokens: [cond_tokens, cond_dim] fp32, device
  * or host memory (NULL only when layers == 0).  cam/depth: the camera/motion
@@ -226,7 +264,9 @@ wdc_status wdc_state_get(wdc_ctx* ctx, wdc_state_host* out, wdc_stream stream);
 /* Installs a state: the small fields from `in`, bank latents copied from
  * z_out[0..in->n_bank-1] (device), the anchor = the newest record's latent
  * (or a copy of z_cur when the bank is empty), and recomputes the derived
- * statistics from z_cur (device) and the anchor.  For tests and resume. */
+ * statistics from z_cur (device) and the anchor.  For tests and resume.  The
+ * secant displacement of WDC_ABL_SECANT is not part of this state: it is
+ * cleared to zero (the secant candidate is z_t until the next exact step). */
 wdc_status wdc_state_set(wdc_ctx* ctx, const wdc_state_host* in, const float* const* z_out,
                          const float* z_cur, wdc_stream stream);
 

@@ -8,6 +8,18 @@ code with the product.
 """
 from dataclasses import dataclass, asdict
 
+# Ablation variants of the method (Tables 3 and 4, section "Ablation Study"):
+# bit flags of CacheParams.flags.  Their definitions are in oracle/ablation.py.
+ABL_PERIODIC = 0x01       # controller: periodic placement at a fixed period
+ABL_SECANT = 0x02         # surrogate: native latent secant
+ABL_INSTANT_RISK = 0x04   # instantaneous risk (no accumulation, lambda = 0)
+ABL_NO_IMPACT = 0x08      # w/o impact weighting (w = 1)
+ABL_NO_CALIB = 0x10       # w/o counterfactual calibration (eta_d fixed)
+ABL_NO_SUPPORT = 0x20     # w/o support constraint
+ABL_LINEAR_OBS = 0x40     # linear observation instead of Eq. 5's kernel
+ABL_NO_COND = 0x80        # lifted surrogate without condition descriptors
+ABL_ALL = 0xFF
+
 
 @dataclass
 class CacheParams:
@@ -43,6 +55,13 @@ class CacheParams:
     max_age: int = 6              # "pre-decision age at most six" (Eq. 10 text)
     n_init_exact: int = 1         # mandatory-exact initialisation steps
     n_final_exact: int = 0        # mandatory-exact refinement steps at the end
+    # Ablation variants (Tables 3 and 4).
+    flags: int = 0                # ABL_* bits; 0 = the full method
+    period: int = 8               # ABL_PERIODIC: one exact step every `period` steps
+    ridge: float = 1e-6           # ABL_LINEAR_OBS: ridge, relative to mean diag of the Gram matrix
+
+    def has(self, flag):
+        return bool(self.flags & flag)
 
     def as_dict(self):
         return asdict(self)

@@ -27,6 +27,7 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
+from . import ablation as ab
 from . import controller as ctl
 from . import schedule as sch
 from . import summary as sm
@@ -44,6 +45,7 @@ class CacheState:
     z_a: np.ndarray = None                     # latest exact anchor (float32)
     q_a_in: float = 1.0                        # latest exact interval q_{a} -> q_{a-1}
     q_a_out: float = 1.0
+    z_a_in: np.ndarray = None                  # input latent of the latest exact step (secant ablation)
     cam_a: np.ndarray = field(default_factory=lambda: np.zeros(4))
     depth_a: np.ndarray = field(default_factory=lambda: np.zeros(4))
     R: float = 0.0
@@ -78,15 +80,23 @@ def surrogate_step(state, z_k, k, cond, sigmas, p):
     q_k = float(sch.phase(sigmas[k]))
     q_next = float(sch.phase(sigmas[k + 1]))
     cam, depth = _cond_desc(cond)
+    lcam, ldepth = ab.lift_descriptors(cam, depth, p)
     z_k = np.asarray(z_k).reshape(-1)
     h = state.history(T, p)
-    s_phi = sm.summary_of_state(z_k, state.z_a, cam, depth, q_k, h, p.eps_nu, p.sketch_seed)
+    s_phi = sm.summary_of_state(z_k, state.z_a, lcam, ldepth, q_k, h, p.eps_nu, p.sketch_seed)
 
     info = {"k": k, "q": q_k, "s_phi": s_phi, "h": h, "n_bank": len(state.bank),
             "supported": False, "finite": False, "alpha": 0.0, "n_compat": 0,
             "kappa": np.zeros(0), "pi": np.zeros(0), "margins": []}
     z_hat = None
-    if state.bank:
+    if state.bank and p.has(ab.ABL_SECANT):
+        # native latent secant (ablation): no retrieval, extrapolate z_a - z_a,in
+        alpha = sg.scheduler_scaling(q_k, q_next, state.q_a_in, state.q_a_out, p)
+        z_hat = _f32(ab.secant_candidate(z_k, state.z_a, state.z_a_in, alpha))
+        info.update({"alpha": alpha, "supported": True, "n_compat": len(state.bank),
+                     "finite": bool(np.all(np.isfinite(z_hat)))})
+        info["margins"].append(abs(p.q_gap_max - abs(q_k - state.q_a_out)))
+    elif state.bank:
         head = sg.surrogate_head(s_phi, q_k, q_next, state.bank, state.q_a_in, state.q_a_out, p)
         info.update({"alpha": head["alpha"], "kappa": head["kappa"], "pi": head["pi"],
                      "sim_in": head["sim"], "sim_out": head["sim_out"], "s_hat": head["s_hat"],
@@ -105,14 +115,17 @@ def surrogate_step(state, z_k, k, cond, sigmas, p):
                             cam, state.cam_a, depth, state.depth_a, p)
     p_t = ctl.defect_proxy(sig, p)
     d_hat = state.eta * p_t
-    w = ctl.impact_weight(cam, depth, q_k, p)
-    delta, R_cand = ctl.candidate_risk(state.R, w, d_hat, p)
+    w = ab.impact_weight(ctl.impact_weight(cam, depth, q_k, p), p)
+    delta = w * d_hat
+    R_cand = ab.risk_decay(p) * state.R + delta                      # Eq. 9
     avail, terms = ctl.available(k, T, len(state.bank), state.age, q_k, state.q_a_out,
                                  info["finite"], info["supported"], p)
-    surrogate = ctl.decide(avail, R_cand, p)
-    others = all(v for key, v in terms.items())
-    if others:
-        info["margins"].append(abs(R_cand - p.tau_risk))
+    if p.has(ab.ABL_PERIODIC):
+        surrogate = ab.periodic_decision(avail, state.age, p)
+    else:
+        surrogate = ctl.decide(avail, R_cand, p)
+        if all(v for key, v in terms.items()):
+            info["margins"].append(abs(R_cand - p.tau_risk))
     info.update({"p": p_t, "d_hat": d_hat, "w": w, "delta": delta, "R_cand": R_cand,
                  "available": avail, "terms": terms, "decision": 1 if surrogate else 0,
                  "d_cf": float("nan"), "age": state.age, **sig})
@@ -137,15 +150,17 @@ def exact_step(state, z_k, v, z_hat, k, cond, sigmas, p, info):
     z_k = np.asarray(z_k).reshape(-1)
     z_ex = _f32(sch.psi(z_k, np.asarray(v).reshape(-1), sigmas[k], sigmas[k + 1]))
 
-    state.R = p.lam * state.R
+    state.R = ab.risk_decay(p) * state.R
     if z_hat is not None and info["supported"] and info["finite"]:
         d_cf = ctl.counterfactual_defect(z_ex, z_hat, p)
-        state.eta = ctl.calibrate(state.eta, d_cf, info["p"], p)
+        if ab.calibrates(p):
+            state.eta = ctl.calibrate(state.eta, d_cf, info["p"], p)
         info["d_cf"] = d_cf
 
     h = state.history(T, p)            # pre-insertion history
     s_in = info["s_phi"]
-    s_out = sm.summary_of_state(z_ex, state.z_a, cam, depth, q_next, h, p.eps_nu, p.sketch_seed)
+    lcam, ldepth = ab.lift_descriptors(cam, depth, p)
+    s_out = sm.summary_of_state(z_ex, state.z_a, lcam, ldepth, q_next, h, p.eps_nu, p.sketch_seed)
     r = sm.rms(z_ex.astype(np.float64) - z_k.astype(np.float64)) / (sm.rms(z_k) + p.eps)
     rec = sg.Record(s_in=np.array(s_in), s_out=s_out, s_dphi=s_out - s_in, z_out=z_ex,
                     q_in=q_k, q_out=q_next, r=r, cam=cam.copy(), depth=depth.copy())
@@ -153,6 +168,7 @@ def exact_step(state, z_k, v, z_hat, k, cond, sigmas, p, info):
     if len(state.bank) > p.bank_capacity:
         state.bank.pop(0)
     state.z_a = z_ex
+    state.z_a_in = _f32(z_k)
     state.q_a_in, state.q_a_out = q_k, q_next
     state.cam_a, state.depth_a = cam.copy(), depth.copy()
     state.age = 0

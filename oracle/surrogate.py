@@ -23,6 +23,7 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
+from . import ablation as ab
 from .summary import cosine
 
 
@@ -59,7 +60,10 @@ def retrieve(s_phi, q_t, bank, p):
     K = len(bank)
     sims = np.array([cosine(s_phi, rec.s_in) for rec in bank], dtype=np.float64)
     dq = np.array([q_t - rec.q_in for rec in bank], dtype=np.float64)
-    compat = np.array([(sims[i] >= p.sim_min) and (abs(dq[i]) <= p.q_gap_max) for i in range(K)], dtype=bool)
+    if ab.compat_filter(p):
+        compat = np.array([(sims[i] >= p.sim_min) and (abs(dq[i]) <= p.q_gap_max) for i in range(K)], dtype=bool)
+    else:
+        compat = np.ones(K, dtype=bool)          # w/o support constraint: N_t = the whole bank
     ell = sims - p.gamma_q * dq * dq
     pi = np.zeros(K, dtype=np.float64)
     if compat.any():
@@ -114,5 +118,7 @@ def surrogate_head(s_phi, q_t, q_next, bank, q_a_in, q_a_out, p):
     alpha = scheduler_scaling(q_t, q_next, q_a_in, q_a_out, p)
     s_hat = evolve_summary(s_phi, alpha, ret["pi"], bank)
     kappa, sims_out = observation_weights(s_hat, bank, p)
+    if p.has(ab.ABL_LINEAR_OBS):
+        kappa = ab.linear_readout(s_hat, bank, p)   # linear observation (ablation)
     ret.update({"alpha": alpha, "s_hat": s_hat, "kappa": kappa, "sim_out": sims_out})
     return ret

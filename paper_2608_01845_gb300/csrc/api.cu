@@ -106,7 +106,10 @@ wdc_status check_params(Ctx* c, const wdc_cache_params& p) {
     if (!(p.lambda_ >= 0)) return fail(c, WDC_ERR_INVALID_ARG, "lambda must be >= 0");
     if (p.min_support < 0 || p.max_age < 0 || p.n_init_exact < 0 || p.n_final_exact < 0)
         return fail(c, WDC_ERR_INVALID_ARG, "negative integer parameter");
-    if (p.flags != 0) return fail(c, WDC_ERR_UNSUPPORTED, "flags must be 0");
+    if (p.flags & ~WDC_ABL_ALL) return fail(c, WDC_ERR_INVALID_ARG, "unknown ablation flag");
+    if ((p.flags & WDC_ABL_PERIODIC) && p.period < 1) return fail(c, WDC_ERR_INVALID_ARG, "period must be >= 1");
+    if ((p.flags & WDC_ABL_LINEAR_OBS) && !(p.ridge >= 0 && p.ridge < 1e300))
+        return fail(c, WDC_ERR_INVALID_ARG, "ridge must be finite and >= 0");
     return WDC_OK;
 }
 
@@ -155,17 +158,24 @@ void set_cond(PassArgs& a, const wdc_cond* cd) {
 }
 
 // Skip pass + async copy of the step record into `dst` (pinned); no sync.
-wdc_status enqueue_skip(Ctx* c, int k, const wdc_cond* cd, float* z_hat, StepOut* dst, cudaStream_t s) {
+// z_cur (the current latent) is read only by the secant ablation.
+wdc_status enqueue_skip(Ctx* c, int k, const wdc_cond* cd, const float* z_cur, float* z_hat, StepOut* dst,
+                        cudaStream_t s) {
     PassArgs a = base_args(c, k);
     set_cond(a, cd);
     a.nsrc = c->n_bank;
-    for (int i = 0; i < c->n_bank; ++i) {
-        a.slot[i] = slot_of(c, i);
-        a.src[i] = c->bank[a.slot[i]];
+    for (int i = 0; i < c->n_bank; ++i) a.slot[i] = slot_of(c, i);
+    const bool secant = c->prm.flags & WDC_ABL_SECANT;
+    if (secant) {
+        if (!z_cur || !c->secant) return fail(c, WDC_ERR_STATE, "secant candidate needs the current latent");
+        a.src[0] = z_cur;
+        a.src[1] = c->secant;
+    } else {
+        for (int i = 0; i < c->n_bank; ++i) a.src[i] = c->bank[a.slot[i]];
     }
     a.anchor = anchor_ptr(c);
     a.out = z_hat;
-    wdc_status st = launch_pass(c, kModeSkip, a, s);
+    wdc_status st = launch_pass(c, secant ? kModeSecant : kModeSkip, a, s);
     if (st) return st;
     WDC_CUDA_TRY(c, cudaMemcpyAsync(dst, &c->st->out, sizeof(StepOut), cudaMemcpyDeviceToHost, s));
     return WDC_OK;
@@ -182,6 +192,7 @@ wdc_status enqueue_anchor(Ctx* c, int k, const wdc_cond* cd, const float* z_t, c
     a.zcf = z_cf;
     a.anchor = anchor_ptr(c);
     a.out = c->bank[ins];
+    a.out2 = (c->prm.flags & WDC_ABL_SECANT) ? c->secant : nullptr;
     a.ins_slot = ins;
     a.dsig = (float)(c->sigma[k + 1] - c->sigma[k]);
     wdc_status st = launch_pass(c, kModeAnchor, a, s);
@@ -193,6 +204,20 @@ wdc_status enqueue_anchor(Ctx* c, int k, const wdc_cond* cd, const float* z_t, c
     c->anchor_is_init = 0;
     c->last_surrogate_k = -1;
     if (z_next) *z_next = c->bank[ins];
+    c->cur_latent = c->bank[ins];
+    return WDC_OK;
+}
+
+// The secant ablation's displacement buffer (allocated on first use, zeroed).
+wdc_status ensure_secant(Ctx* c) {
+    if (!(c->prm.flags & WDC_ABL_SECANT) || c->secant) return WDC_OK;
+    WDC_CUDA_TRY(c, cudaMalloc((void**)&c->secant, c->n * sizeof(float)));
+    WDC_CUDA_TRY(c, cudaMemset(c->secant, 0, c->n * sizeof(float)));
+    return WDC_OK;
+}
+
+wdc_status clear_secant(Ctx* c, cudaStream_t s) {
+    if (c->secant) WDC_CUDA_TRY(c, cudaMemsetAsync(c->secant, 0, c->n * sizeof(float), s));
     return WDC_OK;
 }
 
@@ -236,6 +261,7 @@ wdc_status wdc_default_cache_params(wdc_cache_params* p) {
     p->eta_init = 1.0; p->eta_min = 0.1; p->eta_max = 10.0; p->beta_d = 0.8;
     p->a_cam = 0.5; p->a_depth = 0.5; p->a_phase = 1.0; p->lambda_ = 0.9; p->tau_risk = 0.5;
     p->max_age = 6; p->n_init_exact = 1; p->n_final_exact = 0; p->flags = 0;
+    p->period = 8; p->ridge = 1e-6;
     return WDC_OK;
 }
 
@@ -284,6 +310,7 @@ wdc_status wdc_create(const wdc_dit_config* cfg, const wdc_schedule* sched, cons
     if (!dm((void**)&c->cand[0], lat) || !dm((void**)&c->cand[1], lat)) return bail(WDC_ERR_OOM);
     if (!dm((void**)&c->vbuf, lat)) return bail(WDC_ERR_OOM);
     if (cudaMallocHost((void**)&c->out_host, sizeof(StepOut) * (sched->T + 2)) != cudaSuccess) return bail(WDC_ERR_OOM);
+    if ((st = ensure_secant(c))) return bail(st);
     if (cfg->layers > 0) {
         if ((st = dit_create(c))) return bail(st);
     }
@@ -306,6 +333,7 @@ void wdc_destroy(wdc_ctx* h) {
     cudaFree(c->cand[1]);
     cudaFree(c->vbuf);
     cudaFree(c->zstage);
+    cudaFree(c->secant);
     if (c->out_host) cudaFreeHost(c->out_host);
     for (int k = 0; k < WDC_K_COUNT; ++k)
         for (cudaEvent_t e : c->ev[k]) cudaEventDestroy(e);
@@ -320,7 +348,8 @@ wdc_status wdc_set_cache_params(wdc_ctx* h, const wdc_cache_params* params) {
     if (params->bank_capacity != c->prm.bank_capacity)
         return fail(c, WDC_ERR_INVALID_ARG, "bank_capacity cannot change after wdc_create");
     c->prm = *params;
-    return WDC_OK;
+    cudaSetDevice(c->device);
+    return ensure_secant(c);
 }
 
 const char* wdc_last_error(const wdc_ctx* h) {
@@ -445,6 +474,9 @@ wdc_status wdc_state_reset(wdc_ctx* h, const float* z_T, wdc_stream stream) {
     c->age = 0;
     c->anchor_is_init = 1;
     c->last_surrogate_k = -1;
+    c->cur_latent = c->z_init;
+    wdc_status cs = clear_secant(c, s);
+    if (cs) return cs;
     DevState* hs = nullptr;
     WDC_CUDA_TRY(c, cudaMallocHost((void**)&hs, sizeof(DevState)));
     std::memset(hs, 0, sizeof(DevState));
@@ -543,6 +575,8 @@ wdc_status wdc_state_set(wdc_ctx* h, const wdc_state_host* in, const float* cons
     c->n_bank = in->n_bank;
     c->age = in->age;
     c->last_surrogate_k = -1;
+    c->cur_latent = z_cur;
+    if (wdc_status cs = clear_secant(c, s)) return cs;
     for (int i = 0; i < in->n_bank; ++i)
         WDC_CUDA_TRY(c, cudaMemcpyAsync(c->bank[i], z_out[i], c->n * sizeof(float), cudaMemcpyDeviceToDevice, s));
     if (in->n_bank == 0) {
@@ -565,11 +599,14 @@ wdc_status wdc_surrogate_step(wdc_ctx* h, int k, const wdc_cond* cd, float* z_ha
     cudaSetDevice(c->device);
     cudaStream_t s = (cudaStream_t)stream;
     const int age_before = c->age, nb = c->n_bank;
-    wdc_status st = enqueue_skip(c, k, cd, z_hat, &c->out_host[0], s);
+    wdc_status st = enqueue_skip(c, k, cd, c->cur_latent, z_hat, &c->out_host[0], s);
     if (st) return st;
     if ((st = sync(c, s))) return st;
     const StepOut& o = c->out_host[0];
-    if (o.decision) c->age++;
+    if (o.decision) {
+        c->age++;
+        c->cur_latent = z_hat;
+    }
     c->last_surrogate_k = k;
     fill_info(o, k, nb, age_before, info);
     return WDC_OK;
@@ -647,7 +684,7 @@ static wdc_status rollout_impl(Ctx* c, const float* z_T, const wdc_cond* conds, 
             const wdc_cond* cd = &conds[ci];
             float* zh = c->cand[cur_cand == 0 ? 1 : 0];
             const int nb = c->n_bank, age_before = c->age;
-            if ((st = enqueue_skip(c, k, cd, zh, &c->out_host[k], s))) return st;
+            if ((st = enqueue_skip(c, k, cd, cur, zh, &c->out_host[k], s))) return st;
             if ((st = sync(c, s))) return st;
             const int dec = c->out_host[k].decision;
             c->last_surrogate_k = k;

@@ -88,11 +88,78 @@ struct HeadShared {
     double hat[kSummary];
     double scratch[8 * (kMaxBank + 1)];
     double red[kMaxBank + 1];
+    double gram[kMaxBank][kMaxBank];       // linear observation: the records' Gram matrix
     double sim_in[kMaxBank], sim_out[kMaxBank], pi[kMaxBank], kappa[kMaxBank];
     double alpha;
     int compat[kMaxBank];
     int n_compat, supported;
 };
+
+// Linear observation (ablation): kappa <- beta, the ridge least-squares
+// coefficients of s(phi_hat) on the records' output summaries,
+// (G + rho I) beta = S_out s_hat with G_ij = s_out_i . s_out_j and
+// rho = ridge * trace(G) / K, solved by Cholesky in fp64 (G + rho I is
+// positive definite for rho > 0).  hs.red[0..K) still holds S_out s_hat.
+template <int K>
+__device__ __noinline__ void linear_readout(const PassArgs& a, HeadShared& hs) {
+    if constexpr (K > 0) {
+        const int t = threadIdx.x;
+        const DevState* st = a.st;
+        double b[K];
+        if (t == 0) {
+#pragma unroll
+            for (int i = 0; i < K; ++i) b[i] = hs.red[i];
+        }
+        // one row of G per reduction (keeps K values per thread)
+        for (int i = 0; i < K; ++i) {
+            double v[K];
+            const double si = (t < kSummary) ? st->rec[a.slot[i]].s_out[t] : 0.0;
+#pragma unroll
+            for (int j = 0; j < K; ++j) v[j] = (t < kSummary) ? si * st->rec[a.slot[j]].s_out[t] : 0.0;
+            reduce256<K>(v, hs.scratch, hs.gram[i]);
+        }
+        if (t == 0) {
+            double A[K][K];
+            double tr = 0.0;
+            for (int i = 0; i < K; ++i) {
+                for (int j = 0; j < K; ++j) A[i][j] = 0.5 * (hs.gram[i][j] + hs.gram[j][i]);
+                tr += A[i][i];
+            }
+            if (tr == 0.0) {
+#pragma unroll
+                for (int i = 0; i < K; ++i) hs.kappa[i] = 0.0;
+            } else {
+                const double rho = a.prm.ridge * tr / K;
+#pragma unroll
+                for (int i = 0; i < K; ++i) A[i][i] += rho;
+                // Cholesky A = L L^T (L in the lower triangle of A)
+                for (int j = 0; j < K; ++j) {
+                    double d = A[j][j];
+                    for (int m = 0; m < j; ++m) d -= A[j][m] * A[j][m];
+                    d = sqrt(d);
+                    A[j][j] = d;
+                    for (int i = j + 1; i < K; ++i) {
+                        double x = A[i][j];
+                        for (int m = 0; m < j; ++m) x -= A[i][m] * A[j][m];
+                        A[i][j] = x / d;
+                    }
+                }
+                double y[K];
+                for (int i = 0; i < K; ++i) {
+                    double x = b[i];
+                    for (int m = 0; m < i; ++m) x -= A[i][m] * y[m];
+                    y[i] = x / A[i][i];
+                }
+                for (int i = K - 1; i >= 0; --i) {
+                    double x = y[i];
+                    for (int m = i + 1; m < K; ++m) x -= A[m][i] * hs.kappa[m];
+                    hs.kappa[i] = x / A[i][i];
+                }
+            }
+        }
+        __syncthreads();
+    }
+}
 
 // Skip-pass head (every CTA, redundantly): Eq. 2-5 scalar part.
 template <int K>
@@ -110,9 +177,9 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
             const int b = t - kSketch;
             val = sc * (st->cur_S[b] - st->anchor_S[b]) / (sqrt(st->cur_sumsq_anchor / N) + a.prm.eps_nu);
         } else if (t < kOffDepth) {
-            val = a.cam[t - kOffCam];
+            val = (a.prm.flags & WDC_ABL_NO_COND) ? 0.0 : a.cam[t - kOffCam];
         } else if (t < kOffQ) {
-            val = a.depth[t - kOffDepth];
+            val = (a.prm.flags & WDC_ABL_NO_COND) ? 0.0 : a.depth[t - kOffDepth];
         } else if (t == kOffQ) {
             val = a.q_k;
         } else {
@@ -132,6 +199,11 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
         }
         hs.phi[t] = val;
     }
+    if (t == 0) {
+        // Eq. 4: alpha = clip(|q_{t-1}-q_t| / (|q_{a-1}-q_a| + eps), alpha_min, alpha_max)
+        const double raw = fabs(a.q_next - a.q_k) / (fabs(st->q_a_out - st->q_a_in) + a.prm.eps);
+        hs.alpha = fmin(fmax(raw, a.prm.alpha_min), a.prm.alpha_max);
+    }
     __syncthreads();
     if (K == 0) return;
 
@@ -146,6 +218,7 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
     }
     if (t == 0) {
         const double nphi = sqrt(hs.red[K]);
+        const bool filter = !(a.prm.flags & WDC_ABL_NO_SUPPORT);   // w/o support: N_t = whole bank
         int nc = 0;
         double mx = -INFINITY;
         double ell[K > 0 ? K : 1];
@@ -155,7 +228,7 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
             const double s = (nphi == 0.0 || r.n_in == 0.0) ? 0.0 : hs.red[i] / (nphi * r.n_in);
             const double dq = a.q_k - r.q_in;
             hs.sim_in[i] = s;
-            const int c = (s >= a.prm.sim_min) && (fabs(dq) <= a.prm.q_gap_max);
+            const int c = !filter || ((s >= a.prm.sim_min) && (fabs(dq) <= a.prm.q_gap_max));
             hs.compat[i] = c;
             ell[i] = (s - a.prm.gamma_q * dq * dq) / a.prm.tau_in;
             if (c) { ++nc; mx = fmax(mx, ell[i]); }
@@ -169,10 +242,7 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
 #pragma unroll
         for (int i = 0; i < K; ++i) hs.pi[i] = (nc > 0) ? hs.pi[i] / tot : 0.0;
         hs.n_compat = nc;
-        hs.supported = nc >= a.prm.min_support;
-        // Eq. 4: alpha = clip(|q_{t-1}-q_t| / (|q_{a-1}-q_a| + eps), alpha_min, alpha_max)
-        const double raw = fabs(a.q_next - a.q_k) / (fabs(st->q_a_out - st->q_a_in) + a.prm.eps);
-        hs.alpha = fmin(fmax(raw, a.prm.alpha_min), a.prm.alpha_max);
+        hs.supported = filter ? (nc >= a.prm.min_support) : 1;
     }
     __syncthreads();
     // Eq. 4 in summary space, then Eq. 5 similarities with the lifted outputs
@@ -211,6 +281,7 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
         for (int i = 0; i < K; ++i) hs.kappa[i] = e[i] / tot;
     }
     __syncthreads();
+    if (a.prm.flags & WDC_ABL_LINEAR_OBS) linear_readout<K>(a, hs);
 }
 
 struct PassShared {
@@ -234,11 +305,16 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
 
     bool do_stream = true;
     float kap[K > 0 ? K : 1];
+    float alpha_f = 0.f;
     if (MODE == kModeSkip) {
         skip_head<K>(a, hs);
         do_stream = (K > 0) && hs.supported;
 #pragma unroll
         for (int i = 0; i < K; ++i) kap[i] = (float)hs.kappa[i];
+    } else if (MODE == kModeSecant) {
+        skip_head<0>(a, hs);               // lift summary and alpha only: no retrieval
+        do_stream = a.nsrc > 0;
+        alpha_f = (float)hs.alpha;
     } else if (MODE == kModeObserve) {
 #pragma unroll
         for (int i = 0; i < K; ++i) kap[i] = a.kappa[i];
@@ -293,6 +369,17 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                     *reinterpret_cast<float4*>(a.out + base) = zh;
                     o[0] = zh.x; o[1] = zh.y; o[2] = zh.z; o[3] = zh.w;
                     sa[0] = za.x; sa[1] = za.y; sa[2] = za.z; sa[3] = za.w;
+                } else if constexpr (MODE == kModeSecant) {
+                    // native latent secant: z_hat = z_k + alpha (z_a - z_a,in)
+                    const float4 z = __ldg(reinterpret_cast<const float4*>(a.src[0] + base));
+                    const float4 dz = __ldg(reinterpret_cast<const float4*>(a.src[1] + base));
+                    const float4 za = __ldg(reinterpret_cast<const float4*>(a.anchor + base));
+                    float4 zh;
+                    zh.x = fmaf(alpha_f, dz.x, z.x); zh.y = fmaf(alpha_f, dz.y, z.y);
+                    zh.z = fmaf(alpha_f, dz.z, z.z); zh.w = fmaf(alpha_f, dz.w, z.w);
+                    *reinterpret_cast<float4*>(a.out + base) = zh;
+                    o[0] = zh.x; o[1] = zh.y; o[2] = zh.z; o[3] = zh.w;
+                    sa[0] = za.x; sa[1] = za.y; sa[2] = za.z; sa[3] = za.w;
                 } else if constexpr (MODE == kModeAnchor) {
                     // plain loads: z_k / z_a may alias the slot written below (bank capacity 1)
                     const float4 z = *reinterpret_cast<const float4*>(a.src[0] + base);
@@ -302,6 +389,11 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                     ze.x = fmaf(dsig, v.x, z.x); ze.y = fmaf(dsig, v.y, z.y);
                     ze.z = fmaf(dsig, v.z, z.z); ze.w = fmaf(dsig, v.w, z.w);
                     *reinterpret_cast<float4*>(a.out + base) = ze;
+                    if (a.out2) {
+                        float4 dz;
+                        dz.x = ze.x - z.x; dz.y = ze.y - z.y; dz.z = ze.z - z.z; dz.w = ze.w - z.w;
+                        *reinterpret_cast<float4*>(a.out2 + base) = dz;
+                    }
                     o[0] = ze.x; o[1] = ze.y; o[2] = ze.z; o[3] = ze.w;
                     sa[0] = za.x; sa[1] = za.y; sa[2] = za.z; sa[3] = za.w;
                     sb[0] = z.x; sb[1] = z.y; sb[2] = z.z; sb[3] = z.w;
@@ -337,12 +429,18 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                         a.out[idx] = zh;
                         o[e] = zh;
                         sa[e] = a.anchor[idx];
+                    } else if constexpr (MODE == kModeSecant) {
+                        const float zh = fmaf(alpha_f, a.src[1][idx], a.src[0][idx]);
+                        a.out[idx] = zh;
+                        o[e] = zh;
+                        sa[e] = a.anchor[idx];
                     } else if constexpr (MODE == kModeAnchor) {
                         // read z_k and z_a before the store: they may alias the slot
                         const float z = a.src[0][idx];
                         const float za = a.anchor[idx];
                         const float ze = fmaf(dsig, a.v[idx], z);
                         a.out[idx] = ze;
+                        if (a.out2) a.out2[idx] = ze - z;
                         o[e] = ze;
                         sa[e] = za;
                         sb[e] = z;
@@ -362,7 +460,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                 const float d = x - sa[e];
                 const uint32_t idx = (uint32_t)(base + e);
                 sg += signed_term(idx, seed, x);
-                if (MODE == kModeSkip || MODE == kModeObserve) {
+                if (MODE == kModeSkip || MODE == kModeObserve || MODE == kModeSecant) {
                     fac[0] += x * x;
                     fac[1] += d * d;
                     nonfinite += isfinite(x) ? 0 : 1;
@@ -474,9 +572,10 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
         return;
     }
 
-    if (MODE == kModeSkip) {
+    if (MODE == kModeSkip || MODE == kModeSecant) {
         if (t < kSummary) st->s_phi[t] = hs.phi[t];
-        const int supported = (K > 0) && hs.supported;
+        // the secant needs no retrieval: its support term holds with a non-empty bank
+        const int supported = (MODE == kModeSecant) ? (a.nsrc > 0) : ((K > 0) && hs.supported);
         const int finite = supported && (fin[sc0 + 5] == 0.0);
         __shared__ int s_dec;
         if (t == 0) {
@@ -494,20 +593,24 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
             const double pt = p.w_z * d_z + p.w_age * d_age + p.w_phase * d_phase + p.w_cam * sqrt(dc) +
                               p.w_depth * sqrt(dd);
             const double d_hat = st->eta * pt;
-            const double w = fmin(2.0, 1.0 + p.a_cam * sqrt(uc) + p.a_depth * sqrt(ud) + p.a_phase * a.q_k);
+            const double w = (p.flags & WDC_ABL_NO_IMPACT)
+                                 ? 1.0
+                                 : fmin(2.0, 1.0 + p.a_cam * sqrt(uc) + p.a_depth * sqrt(ud) + p.a_phase * a.q_k);
             const double delta = w * d_hat;
             const double R_cand = p.lam * st->R + delta;
             const bool avail = (a.nsrc > 0) && (a.age <= p.max_age) &&
                                (fabs(a.q_k - st->q_a_out) <= p.q_gap_max) && finite && supported &&
                                (a.k >= p.n_init_exact) && (a.k < a.T - p.n_final_exact);
-            const int dec = (avail && R_cand <= p.tau_risk) ? 1 : 0;
+            // Eq. 10, or periodic placement (ablation): at most period - 1 surrogate steps in a row
+            const bool accept = (p.flags & WDC_ABL_PERIODIC) ? (a.age + 1 < p.period) : (R_cand <= p.tau_risk);
+            const int dec = (avail && accept) ? 1 : 0;
             StepOut& o = st->out;
             o.decision = dec;
             o.finite = finite;
             o.supported = supported;
-            o.n_compat = (K > 0) ? hs.n_compat : 0;
+            o.n_compat = (MODE == kModeSecant) ? a.nsrc : ((K > 0) ? hs.n_compat : 0);
             o.q = a.q_k;
-            o.alpha = (K > 0) ? hs.alpha : 0.0;
+            o.alpha = (a.nsrc > 0) ? hs.alpha : 0.0;
             o.p = pt;
             o.d_hat = d_hat;
             o.w = w;
@@ -551,8 +654,10 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
         double d_cf = nan("");
         if (a.zcf != nullptr && st->cand_k == a.k && st->cand_supported && st->cand_finite) {
             d_cf = (fin[sc0 + 0] / N) / (fin[sc0 + 1] / N + p.eps);
-            const double v = p.beta_d * st->eta + (1.0 - p.beta_d) * d_cf / (st->cand_p + p.eps);
-            st->eta = fmin(fmax(v, p.eta_min), p.eta_max);
+            if (!(p.flags & WDC_ABL_NO_CALIB)) {
+                const double v = p.beta_d * st->eta + (1.0 - p.beta_d) * d_cf / (st->cand_p + p.eps);
+                st->eta = fmin(fmax(v, p.eta_min), p.eta_max);
+            }
         }
         st->out.d_cf = d_cf;
         st->out.R = st->R;
@@ -574,9 +679,9 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
             const int b = t - kSketch;
             so = sc * (fin[b] - st->anchor_S[b]) / (s_rms[1] + a.prm.eps_nu);
         } else if (t < kOffDepth) {
-            so = a.cam[t - kOffCam];
+            so = (a.prm.flags & WDC_ABL_NO_COND) ? 0.0 : a.cam[t - kOffCam];
         } else if (t < kOffQ) {
-            so = a.depth[t - kOffDepth];
+            so = (a.prm.flags & WDC_ABL_NO_COND) ? 0.0 : a.depth[t - kOffDepth];
         } else if (t == kOffQ) {
             so = a.q_next;
         } else {
@@ -634,10 +739,13 @@ int pass_grid(const Ctx* c) {
 
 wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s) {
     const int grid = pass_grid(c);
-    LaunchScope ls(c, mode == kModeSkip ? WDC_K_SKIP : (mode == kModeAnchor ? WDC_K_ANCHOR : WDC_K_OTHER), s);
+    LaunchScope ls(c, (mode == kModeSkip || mode == kModeSecant) ? WDC_K_SKIP
+                                                                 : (mode == kModeAnchor ? WDC_K_ANCHOR : WDC_K_OTHER),
+                   s);
     switch (mode) {
         case kModeStats: pass_kernel<kModeStats, 0><<<grid, kThreads, 0, s>>>(a); break;
         case kModeAnchor: pass_kernel<kModeAnchor, 0><<<grid, kThreads, 0, s>>>(a); break;
+        case kModeSecant: pass_kernel<kModeSecant, 0><<<grid, kThreads, 0, s>>>(a); break;
         case kModeSkip:
             switch (a.nsrc) {
                 case 0: launch_skip<0>(a, grid, s); break;
@@ -687,8 +795,11 @@ ParamsDev to_dev_params(const wdc_cache_params& p) {
     d.a_cam = p.a_cam;
     d.a_depth = p.a_depth;
     d.a_phase = p.a_phase;
-    d.lam = p.lambda_;
+    d.lam = (p.flags & WDC_ABL_INSTANT_RISK) ? 0.0 : p.lambda_;   // instantaneous risk: no accumulation
     d.tau_risk = p.tau_risk;
+    d.flags = p.flags;
+    d.period = p.period;
+    d.ridge = p.ridge;
     return d;
 }
 

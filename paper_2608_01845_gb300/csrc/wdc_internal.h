@@ -62,21 +62,25 @@ struct ParamsDev {
     unsigned seed;
     double sim_min, q_gap_max, gamma_q, tau_in, tau_obs, alpha_min, alpha_max, eps, eps_nu;
     double w_z, w_age, w_phase, w_cam, w_depth, eta_min, eta_max, beta_d;
-    double a_cam, a_depth, a_phase, lam, tau_risk;
+    double a_cam, a_depth, a_phase, lam, tau_risk;   // lam = 0 under WDC_ABL_INSTANT_RISK
+    int flags, period;                               // WDC_ABL_* bits; periodic placement
+    double ridge;                                    // linear observation
 };
 
-enum StreamMode { kModeStats = 0, kModeSkip = 1, kModeAnchor = 2, kModeObserve = 3 };
+enum StreamMode { kModeStats = 0, kModeSkip = 1, kModeAnchor = 2, kModeObserve = 3, kModeSecant = 4 };
 
 // Launch arguments of the fused latent-pass kernels (passed by value).
 struct PassArgs {
     long long n;
     int nsrc;                          // skip: records in age order (oldest first)
-    const float* src[kMaxBank];        // skip: bank latents by age; anchor/stats: src[0] = z_k
+    const float* src[kMaxBank];        // skip: bank latents by age; anchor/stats: src[0] = z_k;
+                                       // secant: src[0] = z_k, src[1] = z_a - z_a,in
     int slot[kMaxBank];                // ring slot of each record, by age
     const float* anchor;               // z_a
     const float* v;                    // anchor: velocity
     const float* zcf;                  // anchor: counterfactual candidate or nullptr
     float* out;                        // skip: z_hat; anchor: z_exact (bank slot)
+    float* out2;                       // anchor: z_exact - z_k (secant displacement) or nullptr
     float dsig;                        // anchor: sigma_{k+1} - sigma_k (fp32)
     int k, T, age, ins_slot;
     double q_k, q_next;
@@ -113,6 +117,8 @@ struct Ctx {
     float* cand[2] = {};               // rollout candidate buffers
     float* vbuf = nullptr;
     float* zstage = nullptr;           // host-pointer staging for rollouts
+    float* secant = nullptr;           // WDC_ABL_SECANT: z_a - z_a,in of the latest exact step
+    const float* cur_latent = nullptr; // current latent of the step API (read by the secant)
 
     // host mirror of the discrete state
     int n_bank = 0, head = 0, age = 0;

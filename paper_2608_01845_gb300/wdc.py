@@ -56,7 +56,19 @@ class CacheParams(ctypes.Structure):
                 + [(n, ctypes.c_double) for n in ["w_z", "w_age", "w_phase", "w_cam", "w_depth", "eta_init",
                                                    "eta_min", "eta_max", "beta_d", "a_cam", "a_depth", "a_phase",
                                                    "lambda_", "tau_risk"]]
-                + [(n, ctypes.c_int) for n in ["max_age", "n_init_exact", "n_final_exact", "flags"]])
+                + [(n, ctypes.c_int) for n in ["max_age", "n_init_exact", "n_final_exact", "flags", "period"]]
+                + [("ridge", ctypes.c_double)])
+
+
+# Ablation variants (wdc_cache_params.flags; definitions in include/wdc.h).
+ABL_PERIODIC = 0x01
+ABL_SECANT = 0x02
+ABL_INSTANT_RISK = 0x04
+ABL_NO_IMPACT = 0x08
+ABL_NO_CALIB = 0x10
+ABL_NO_SUPPORT = 0x20
+ABL_LINEAR_OBS = 0x40
+ABL_NO_COND = 0x80
 
 
 class Cond(ctypes.Structure):

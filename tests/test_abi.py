@@ -38,3 +38,35 @@ def test_struct_sizes_match_the_header_layout():
     # wdc_step_info: 7 ints, pad to 8-byte alignment, 12 doubles, 2 x 8 doubles
     assert ctypes.sizeof(wdc.StepInfo) == 8 * 4 + 12 * 8 + 16 * 8
     assert ctypes.sizeof(wdc.Cond) == 8 + 8 * 8
+
+
+def test_ablation_flags_and_defaults_match_the_header():
+    src = open(os.path.join(ROOT, "include", "wdc.h")).read()
+    hdr = {m.group(1): int(m.group(2), 16) for m in re.finditer(r"#define WDC_ABL_([A-Z_]+)\s+0x([0-9A-Fa-f]+)", src)}
+    names = ["PERIODIC", "SECANT", "INSTANT_RISK", "NO_IMPACT", "NO_CALIB", "NO_SUPPORT", "LINEAR_OBS", "NO_COND"]
+    for n in names:
+        assert getattr(wdc, "ABL_" + n) == hdr[n]
+    assert hdr["ALL"] == sum(hdr[n] for n in names)
+    p = wdc.default_params()
+    assert p.period == 8 and p.ridge == 1e-6
+
+
+def test_cache_params_layout_matches_a_c_compiler(tmp_path):
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        import pytest
+        pytest.skip("no C compiler")
+    fields = [f for f, _ in wdc.CacheParams._fields_]
+    prog = tmp_path / "layout.c"
+    prog.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "wdc.h"\nint main(void) {\n'
+                    '  printf("%zu\\n", sizeof(wdc_cache_params));\n'
+                    + "".join(f'  printf("%zu\\n", offsetof(wdc_cache_params, {f}));\n' for f in fields)
+                    + "  return 0;\n}\n")
+    exe = tmp_path / "layout"
+    subprocess.run([cc, "-I", os.path.join(ROOT, "include"), "-I", "/usr/local/cuda/include", str(prog), "-o", str(exe)],
+                   check=True)
+    out = [int(x) for x in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()]
+    assert out[0] == ctypes.sizeof(wdc.CacheParams)
+    assert out[1:] == [getattr(wdc.CacheParams, f).offset for f in fields]
