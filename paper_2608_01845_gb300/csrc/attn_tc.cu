@@ -3,17 +3,25 @@
 // full spatio-temporal attention).  Q, K [H, L, d], V^T [H, d, L], O [L, H*d],
 // bf16 with fp32 softmax and accumulation; d = 64 or 128.
 //
-// One CTA per (head, 256 query rows), 11 (d = 64) or 10 (d = 128) warps:
-//   warp 0      TMA producer: the two 128-row Q tiles once, then K / V^T tiles
+// One CTA per (head, 256 query rows), 12 warps in three warpgroups:
+//   warpgroup 0 (control, registers lowered to 40 / 72 per thread)
+//     warp 0    TMA producer: the two 128-row Q tiles once, then K / V^T tiles
 //               of 128 keys into a shared-memory ring (128-byte swizzle);
-//   warp 1(,10) MMA issuer(s): one thread per query tile (d = 64) or one
+//     warp 1(,2) MMA issuer(s): one thread per query tile (d = 64) or one
 //               thread for both (d = 128):
 //               S(t) = Q(t) K^T into TMEM (128 fp32 columns per tile) and
 //               O(t) += P(t) V into TMEM;
-//   warps 2-5   softmax of query tile 0, warps 6-9 of tile 1 (one thread per
-//               query row = TMEM lane): online max, exp2, row sums, O
-//               rescaling in TMEM when the running max grows by more than 2^8,
-//               final 1/l normalisation and the bf16 store.
+//   warpgroups 1, 2 (softmax of query tile 0, 1; registers raised to 232 / 216)
+//               one thread per query row = TMEM lane: exp2 numerators, row
+//               sums, O rescaling in TMEM when the exponent base moves, final
+//               1/l normalisation and the bf16 store.
+// The exponent base of a row only moves when a tile could produce a numerator
+// above 2^8: each tile is first exponentiated against the running base with
+// no max pass (no max -> exp dependency); only when its row sum exceeds 2^8
+// -- the only way a numerator can -- does the row take the tile max, move the
+// base and recompute (O and l share the base, so the result is unchanged).
+// The first tile sets the base from its own max.  S stays in registers until
+// that check, hence the register split.
 // P (bf16 pairs) is written to tensor memory and read as the TMEM A operand
 // of the PV MMA (shared memory is left to Q, K and V).  Two TMEM layouts:
 //   d = 64   per tile t: S (128 columns), P (64), O (64) = 256 columns, so P
@@ -37,11 +45,16 @@ namespace {
 
 constexpr int BQ = 128;        // query rows per tile (two tiles per CTA)
 constexpr int BKV = 128;       // keys per tile
+// Register split: launch allocation 168 per thread (65536 / 384 rounded
+// down to a multiple of 8); the control warpgroup hands registers to the two
+// softmax warpgroups (d = 64: 128 * 40 + 256 * 232 = 384 * 168; the single
+// d = 128 issuer, which drives both tiles, keeps 72: 128 * 72 + 256 * 216).
+constexpr uint32_t kRegsLaunch = 168;
 
 template <int D>
 struct AttnCfg {
     static constexpr bool P_SEP = D == 64;                  // P in its own TMEM columns, one issuer per tile
-    static constexpr int THREADS = P_SEP ? 352 : 320;       // 11 or 10 warps
+    static constexpr int THREADS = 384;                     // 3 warpgroups
     static constexpr int ISSUERS = P_SEP ? 2 : 1;
     static constexpr int ATOMS = D / 64;                    // 128-byte atoms along d
     static constexpr uint32_t Q_TILE = BQ * D * 2;          // one query tile
@@ -51,11 +64,15 @@ struct AttnCfg {
     static constexpr int STAGES = D == 64 ? 3 : 2;
     static constexpr uint32_t SMEM = 2 * Q_TILE + STAGES * STAGE + 1024 + 256;
     static constexpr uint32_t TMEM_COLS = 512;
+    static constexpr uint32_t REGS_CONTROL = P_SEP ? 40 : 72;
+    static constexpr uint32_t REGS_SOFTMAX = P_SEP ? 232 : 216;
+    static_assert(128 * REGS_CONTROL + 256 * REGS_SOFTMAX <= 384 * kRegsLaunch, "register split exceeds the launch");
     // TMEM column of S, P and O of query tile t
     __device__ static constexpr uint32_t s_col(int t) { return P_SEP ? 256u * t : 128u * t; }
     __device__ static constexpr uint32_t p_col(int t) { return P_SEP ? 256u * t + 128u : 128u * t; }
     __device__ static constexpr uint32_t o_col(int t) { return P_SEP ? 256u * t + 192u : 256u + (uint32_t)D * t; }
 };
+
 
 struct AttnArgs {
     int H, L, n_kv, q_blocks;
@@ -119,9 +136,6 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
                    const __grid_constant__ CUtensorMap tv, const __grid_constant__ AttnArgs g) {
     using C = AttnCfg<D>;
-    // paired-fp32 numerators (fma.f32x2 / add.f32x2) measured faster at
-    // d = 128 and slower at d = 64
-    constexpr bool kPairedExp = D == 128;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sq = smem;                                       // [2 tiles][ATOMS][128 x 128 B]
@@ -173,8 +187,11 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    const int wg = warp >> 2;
 
-    if (warp == 0) {
+    if (wg == 0) {
+      setmaxnreg_dec<C::REGS_CONTROL>();
+      if (warp == 0) {
         if (lane == 0) {
             // Q: two tiles x ATOMS boxes of [128 rows x 64 d]
             mbar_arrive_expect_tx(q_full, 2 * C::Q_TILE);
@@ -209,7 +226,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                 }
             }
         }
-    } else if (warp == 1 || (C::P_SEP && warp == 10)) {
+      } else if (warp == 1 || (C::P_SEP && warp == 2)) {
         if (lane == 0) {
             constexpr uint32_t idesc_s = idesc_bf16(BQ, BKV);
             constexpr uint32_t idesc_o = idesc_bf16(BQ, D);
@@ -242,7 +259,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                 // this thread issues the MMAs of query tile t only; the other
                 // tile has its own issuer, so neither waits behind the other's
                 // softmax
-                const int t = (warp == 1) ? 0 : 1;
+                const int t = warp - 1;
                 for (int j = 0; j < n_kv && ok; ++j) {
                     if (!mbar_wait(&kv_full[stage], phase, abort_flag, g.err)) { ok = false; break; }
                     tc_fence_after();
@@ -301,9 +318,11 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
             while (!mbar_try_wait(mma_done, 0) && globaltimer() - t0 < kWaitLimitNs) {
             }
         }
+      }
     } else {
+        setmaxnreg_inc<C::REGS_SOFTMAX>();
         // softmax warpgroups: t = query tile, quarter = TMEM lane quarter
-        const int t = (warp - 2) >> 2;
+        const int t = wg - 1;
         const int quarter = warp & 3;
         const int row = quarter * 32 + lane;                 // row within the tile = TMEM lane
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
@@ -332,50 +351,58 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                 for (int c = 0; c < BKV; ++c)
                     if (c >= last_valid) s[c] = -INFINITY;
             }
-            // row max with 8 independent partial maxima (short dependency chains)
-            float m8[8];
+            auto tile_max = [&]() {
+                // 8 independent partial maxima (short dependency chains)
+                float m8[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) m8[i] = fmaxf(s[i], s[8 + i]);
+                for (int i = 0; i < 8; ++i) m8[i] = fmaxf(s[i], s[8 + i]);
 #pragma unroll
-            for (int c = 16; c < BKV; c += 16)
+                for (int c = 16; c < BKV; c += 16)
 #pragma unroll
-                for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], s[c + i], s[c + 8 + i]);
-            const float mx = fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
-            // The exponent base only moves when the running max grows by more
-            // than 8 (a factor 256): O and l share the same base, so the result
-            // is unchanged, and most tiles skip the O rescale in TMEM.
-            const float m_cand = fmaxf(m_run, mx * g.scale_log2);
-            const bool grow = m_cand - m_run > 8.0f;
-            const float m_use = grow ? m_cand : m_run;
-            const float corr = grow ? ex2(m_run - m_cand) : 1.0f;
+                    for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], s[c + i], s[c + 8 + i]);
+                return fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
+            };
+            // numerators 2^(s * scale - base) into p (bf16 pairs); returns their sum
             uint32_t p[BKV / 2];
-            float sum;
-            if constexpr (kPairedExp) {
-                // 2^(s * scale - m) in paired-fp32 form; 8 partial sums (4 pairs)
+            auto numerators = [&](float base) {
+                // paired-fp32 form (fma.f32x2, add.f32x2): 8 partial sums in 4 pairs
                 uint64_t sum4[4];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) sum4[i] = 0ull;
-                const uint64_t nm2 = pair(-m_use, -m_use);
+                const uint64_t nm2 = pair(-base, -base);
 #pragma unroll
                 for (int c = 0; c < BKV; c += 2) p[c / 2] = exp2_pair(s[c], s[c + 1], scale2, nm2, sum4[(c / 2) & 3]);
-                sum = (pair_sum(sum4[0]) + pair_sum(sum4[1])) + (pair_sum(sum4[2]) + pair_sum(sum4[3]));
-            } else {
-                float sum8[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) sum8[i] = 0.f;
-                const float nm = -m_use;
-#pragma unroll
-                for (int c = 0; c < BKV; c += 2) {
-                    const float a = ex2(fmaf(s[c], g.scale_log2, nm));
-                    const float b = ex2(fmaf(s[c + 1], g.scale_log2, nm));
-                    sum8[c & 7] += a;
-                    sum8[(c + 1) & 7] += b;
-                    p[c / 2] = pack2(a, b);
+                return (pair_sum(sum4[0]) + pair_sum(sum4[1])) + (pair_sum(sum4[2]) + pair_sum(sum4[3]));
+            };
+            float base = (j == 0) ? tile_max() * g.scale_log2 : m_run;
+            float sum;
+            // A numerator above 2^8 implies a row sum above 2^8 (so does a
+            // non-finite one): only then take the tile max, move the base and
+            // recompute.  d = 64 runs the recompute as a second pass of the
+            // same code; d = 128 (higher register pressure around its single
+            // issuer's schedule) measured faster with a separate copy.
+            if constexpr (C::P_SEP) {
+#pragma unroll 1
+                for (int pass = 0;; ++pass) {
+                    sum = numerators(base);
+                    const bool redo = pass == 0 && !(sum <= 256.0f);
+                    if (!__any_sync(0xffffffffu, redo)) break;
+                    if (redo) base = fmaxf(base, tile_max() * g.scale_log2);
                 }
-                sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
+            } else {
+                sum = numerators(base);
+                const bool redo = !(sum <= 256.0f);
+                if (__any_sync(0xffffffffu, redo)) {
+                    if (redo) {
+                        base = fmaxf(base, tile_max() * g.scale_log2);
+                        sum = numerators(base);
+                    }
+                }
             }
+            const bool moved = base != m_run;
+            const float corr = ex2(m_run - base);     // 1 when the base stays; 0 before the first tile
             l_run = l_run * corr + sum;
-            m_run = m_use;
+            m_run = base;
             if constexpr (C::P_SEP) {
                 // PV(t, j-1) must be done before P(t) is overwritten and O(t) rescaled
                 if (j > 0) {
@@ -383,7 +410,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                     tc_fence_after();
                 }
             }
-            if (j > 0 && __any_sync(0xffffffffu, grow)) {
+            if (j > 0 && __any_sync(0xffffffffu, moved)) {
                 // PV(t, j-1) is complete (p_free, or the commit after S(t, j)): rescale O in place
 #pragma unroll
                 for (int c = 0; c < D; c += 32) {
@@ -444,10 +471,19 @@ template <int D>
 wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, cudaStream_t s) {
     using Cf = AttnCfg<D>;
     static bool attr = false;
+    static bool regs_ok = false;
     if (!attr) {
         cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cf::SMEM);
+        // the warpgroups' register requests must fit the launch allocation,
+        // or setmaxnreg.inc would wait forever: refuse to launch otherwise
+        cudaFuncAttributes fa;
+        regs_ok = cudaFuncGetAttributes(&fa, attn_tc_kernel<D>) == cudaSuccess &&
+                  fa.maxThreadsPerBlock >= Cf::THREADS &&
+                  (uint32_t)fa.numRegs * Cf::THREADS >= 128 * Cf::REGS_CONTROL + 256 * Cf::REGS_SOFTMAX;
+        cudaGetLastError();
         attr = true;
     }
+    if (!regs_ok) return fail(c, WDC_ERR_UNSUPPORTED, "attention kernel's register allocation is below its warpgroup split");
     CUtensorMap tq, tk, tv;
     std::string why;
     const uint64_t row = (uint64_t)D * 2, head = (uint64_t)L * D * 2;
