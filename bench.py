@@ -246,12 +246,16 @@ def traffic_for(kernel_file):
     return e.get("dram_bytes_per_launch")
 
 
-def skip_pass_gbps(torch, wdc, peaks):
+def skip_pass_gbps(torch, wdc, peaks, secant=False):
     """Fused skip pass alone at 2^28 fp32 elements, bank of 4 (reads 4 N,
-    writes N), L2 flushed by a 512 MB write before every launch."""
+    writes N), L2 flushed by a 512 MB write before every launch.  With
+    ``secant`` the native-latent-secant ablation's pass instead (reads z_t,
+    the stored displacement and z_a, writes N)."""
     import numpy as np
     n = SKIP_SWEEP_N
-    ctx = wdc.Context(wdc.make_config(layers=0, width=n), 50, params=wdc.make_params(bank_capacity=4, sim_min=-1.0))
+    flags = wdc.ABL_SECANT if secant else 0
+    ctx = wdc.Context(wdc.make_config(layers=0, width=n), 50,
+                      params=wdc.make_params(bank_capacity=4, sim_min=-1.0, flags=flags))
     dev = torch.device("cuda")
     bank = [torch.randn(n, device=dev) for _ in range(4)]
     st = wdc.StateHost()
@@ -281,12 +285,13 @@ def skip_pass_gbps(torch, wdc, peaks):
         info = ctx.surrogate_step(20, cond, zh)
     prof = ctx.profile_read()
     ms = prof["skip"][0] / prof["skip"][1]
-    gbs = 5 * 4 * n / (ms * 1e-3) / 1e9
+    streams = 4 if secant else 5
+    gbs = streams * 4 * n / (ms * 1e-3) / 1e9
     ctx.close()
     del bank, zc, zh, flush
     torch.cuda.empty_cache()
     return {"gbps": gbs, "ms": ms, "n": n, "bank": 4, "supported": bool(info.supported),
-            "frac_of_measured_copy": gbs / peaks["hbm_gbs"]}
+            "bytes": streams * 4 * n, "frac_of_measured_copy": gbs / peaks["hbm_gbs"]}
 
 
 def block_tflops(torch, ctx, w, peaks):
@@ -310,6 +315,23 @@ def block_tflops(torch, ctx, w, peaks):
     return {"tflops": tf, "ms": ms, "frac_of_measured_burst": tf / peaks["bf16_tflops"]}
 
 
+# Ablation variants of Tables 3-4 for `--ablation NAME` (the periodic
+# controller at period 2 = 25 exact steps of 50, the closest period to the
+# risk controller's 23 of 50: "matched budget").
+ABLATIONS = {
+    "full": dict(flags=0),
+    "periodic+secant": dict(flags=0x01 | 0x02, period=2),
+    "risk+secant": dict(flags=0x02),
+    "periodic+lifted": dict(flags=0x01, period=2),
+    "no_condition": dict(flags=0x80),
+    "linear_obs": dict(flags=0x40),
+    "instantaneous": dict(flags=0x04),
+    "no_impact": dict(flags=0x08),
+    "no_calibration": dict(flags=0x10),
+    "no_support": dict(flags=0x20),
+}
+
+
 def run_gpu(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -318,7 +340,7 @@ def run_gpu(args, rank, world, local_rank):
     w = WORKLOAD_5B
     T = w["T"]
     peaks, peak_src = load_peaks()
-    params = wdc.make_params(tau_risk=w["tau_risk"])
+    params = wdc.make_params(tau_risk=w["tau_risk"], **(ABLATIONS[args.ablation] if args.ablation else {}))
     ctx = wdc.Context(dit_config(w), T, params=params, device=local_rank)
     ctx.init_weights(w["weight_seed"], 0.02)
     zT, ct, desc = inputs(w, rank)
@@ -385,7 +407,8 @@ def run_gpu(args, rank, world, local_rank):
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": w["name"], "T": T, "tau_risk": w["tau_risk"], "bank_capacity": 4,
+            "config": {"workload": w["name"] + (f", ablation {args.ablation}" if args.ablation else ""),
+                       "T": T, "tau_risk": w["tau_risk"], "bank_capacity": 4,
                        "l2": "inputs larger than L2 (10.3 GB of weights per forward)",
                        "parallelism": f"replicas x{world}"},
             "exact_steps_per_rollout": exact, "gpu_launches": launches, "clocks": clk, "roofline": roofline}
@@ -409,12 +432,24 @@ def run_gpu(args, rank, world, local_rank):
     line["e2e"] = {"value": world * T * args.steps / et, "unit": UNIT,
                    "h2d_bytes_per_step": zT.nbytes + ct.nbytes, "d2h_bytes_per_step": zT.nbytes}
 
+    if args.ablation and rank == 0:
+        # mechanics of the variant on the random-init model: final latent
+        # against the uncached rollout of the same inputs
+        cached = out.cpu().numpy().astype("float64")
+        nat = torch.empty_like(zT_d)
+        ctx.native_rollout(zT_d, cond, nat)
+        nat = nat.cpu().numpy().astype("float64")
+        import numpy as np
+        line["ablation"] = {"name": args.ablation, "flags": params.flags, "period": params.period,
+                            "final_rel_l2_vs_native": float(np.linalg.norm(cached - nat) / np.linalg.norm(nat))}
+
     # ---- components named by the metric (rank 0 only)
     if rank == 0:
         line["components"] = {"dit_block": block_tflops(torch, ctx, w, peaks)}
         ctx.close()
         torch.cuda.empty_cache()
         line["components"]["skip_pass"] = skip_pass_gbps(torch, wdc, peaks)
+        line["components"]["secant_pass"] = skip_pass_gbps(torch, wdc, peaks, secant=True)
         line["components"]["peaks"] = {"hbm_gbs": peaks["hbm_gbs"], "bf16_tflops": peaks["bf16_tflops"],
                                        "source": peak_src}
         if world == 1 and not args.no_cpu_baseline:
@@ -453,8 +488,8 @@ def run_op(args):
         mod = 0.1 * torch.randn((2 if w["dual_stream"] else 1) * 6, D, device=dev)
         fn, work, unit = (lambda: ctx.dit_block_forward(0, x, mod)), sum(block_flops(w)), "TFLOP/s"
     else:
-        r = skip_pass_gbps(torch, wdc, peaks)
-        print(json.dumps({"op": "skip", **r}))
+        r = skip_pass_gbps(torch, wdc, peaks, secant=args.op == "secant")
+        print(json.dumps({"op": args.op, **r}))
         return
     for _ in range(2):
         fn()
@@ -478,7 +513,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="wdc", choices=["wdc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--op", choices=["attention", "gemm", "block", "skip"],
+    ap.add_argument("--ablation", choices=sorted(ABLATIONS),
+                    help="run the timed rollout under one ablation variant (Tables 3-4) and report its "
+                         "final latent against the uncached rollout")
+    ap.add_argument("--op", choices=["attention", "gemm", "block", "skip", "secant"],
                     help="time one operator at its 5B-scale shape (profiler captures)")
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="5b",
