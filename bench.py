@@ -315,7 +315,8 @@ def block_tflops(torch, ctx, w, peaks):
     return {"tflops": tf, "ms": ms, "frac_of_measured_burst": tf / peaks["bf16_tflops"]}
 
 
-# Ablation variants of Tables 3-4 for `--ablation NAME` (the periodic
+# Ablation variants of Tables 3-4 (and the residual reading of Eq. 5) for
+# `--ablation NAME` (the periodic
 # controller at period 2 = 25 exact steps of 50, the closest period to the
 # risk controller's 23 of 50: "matched budget").
 ABLATIONS = {
@@ -329,6 +330,7 @@ ABLATIONS = {
     "no_impact": dict(flags=0x08),
     "no_calibration": dict(flags=0x10),
     "no_support": dict(flags=0x20),
+    "residual": dict(flags=0x100),                  # residual reading of Eq. 5 (not an ablation)
 }
 
 

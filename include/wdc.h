@@ -96,7 +96,7 @@ typedef struct wdc_cache_params {
     double lambda_, tau_risk;                     /* decay and threshold (Eq. 9-10) */
     int max_age;                /* pre-decision anchor age limit (Eq. 10 text)   */
     int n_init_exact, n_final_exact;              /* mandatory-exact phases      */
-    int flags;                  /* WDC_ABL_* ablation bits; 0 = the full method  */
+    int flags;                  /* WDC_ABL_* ablation bits, WDC_OBS_RESIDUAL     */
     int period;                 /* WDC_ABL_PERIODIC: exact step every `period`   */
     double ridge;               /* WDC_ABL_LINEAR_OBS: relative ridge            */
 } wdc_cache_params;
@@ -136,6 +136,18 @@ typedef struct wdc_cache_params {
 #define WDC_ABL_LINEAR_OBS   0x40
 #define WDC_ABL_NO_COND      0x80
 #define WDC_ABL_ALL          0xFF
+
+/* Reading flag (also in wdc_cache_params.flags), not an ablation:
+ *   OBS_RESIDUAL  residual reading of Eq. 5's observation: the kernel weights
+ *                 blend the records' exact latent displacements instead of
+ *                 their outputs, z_hat = z_t + sum_i kappa_i (z_out_i - z_in_i).
+ *                 Eq. 5 as printed (the default) is a convex combination of
+ *                 stored exact outputs and so cannot move the latent past the
+ *                 bank; this reading can.  The context keeps one displacement
+ *                 buffer per bank slot (written by the exact-step pass); like
+ *                 the secant's, they are not part of wdc_state_host and
+ *                 wdc_state_set clears them. */
+#define WDC_OBS_RESIDUAL     0x100
 
 /* Model condition c of one step.  tokens: [cond_tokens, cond_dim] fp32, device
  * or host memory (NULL only when layers == 0).  cam/depth: the camera/motion
@@ -265,8 +277,9 @@ wdc_status wdc_state_get(wdc_ctx* ctx, wdc_state_host* out, wdc_stream stream);
  * z_out[0..in->n_bank-1] (device), the anchor = the newest record's latent
  * (or a copy of z_cur when the bank is empty), and recomputes the derived
  * statistics from z_cur (device) and the anchor.  For tests and resume.  The
- * secant displacement of WDC_ABL_SECANT is not part of this state: it is
- * cleared to zero (the secant candidate is z_t until the next exact step). */
+ * exact-step displacements kept for WDC_ABL_SECANT / WDC_OBS_RESIDUAL are not
+ * part of this state: they are cleared to zero (those candidates equal z_t
+ * until exact steps refill them). */
 wdc_status wdc_state_set(wdc_ctx* ctx, const wdc_state_host* in, const float* const* z_out,
                          const float* z_cur, wdc_stream stream);
 

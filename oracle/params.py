@@ -19,6 +19,9 @@ ABL_NO_SUPPORT = 0x20     # w/o support constraint
 ABL_LINEAR_OBS = 0x40     # linear observation instead of Eq. 5's kernel
 ABL_NO_COND = 0x80        # lifted surrogate without condition descriptors
 ABL_ALL = 0xFF
+# Residual reading of Eq. 5 (a reading, not an ablation; see
+# oracle/surrogate.observe_residual).
+OBS_RESIDUAL = 0x100
 
 
 @dataclass
@@ -56,7 +59,7 @@ class CacheParams:
     n_init_exact: int = 1         # mandatory-exact initialisation steps
     n_final_exact: int = 0        # mandatory-exact refinement steps at the end
     # Ablation variants (Tables 3 and 4).
-    flags: int = 0                # ABL_* bits; 0 = the full method
+    flags: int = 0                # ABL_* bits, OBS_RESIDUAL; 0 = the full method as printed
     period: int = 8               # ABL_PERIODIC: one exact step every `period` steps
     ridge: float = 1e-6           # ABL_LINEAR_OBS: ridge, relative to mean diag of the Gram matrix
 

@@ -30,6 +30,7 @@ import numpy as np
 from . import ablation as ab
 from . import controller as ctl
 from . import schedule as sch
+from .params import OBS_RESIDUAL
 from . import summary as sm
 from . import surrogate as sg
 
@@ -106,7 +107,10 @@ def surrogate_step(state, z_k, k, cond, sigmas, p):
             info["margins"].append(abs(p.q_gap_max - abs(head["dq"][i])))
         info["margins"].append(abs(p.q_gap_max - abs(q_k - state.q_a_out)))
         if head["supported"]:
-            z_hat = _f32(sg.observe(head["kappa"], state.bank))
+            if p.has(OBS_RESIDUAL):
+                z_hat = _f32(sg.observe_residual(head["kappa"], state.bank, z_k))
+            else:
+                z_hat = _f32(sg.observe(head["kappa"], state.bank))
             info["finite"] = bool(np.all(np.isfinite(z_hat)))
 
     rms_dz = sm.rms(z_k.astype(np.float64) - state.z_a.astype(np.float64))
@@ -162,7 +166,7 @@ def exact_step(state, z_k, v, z_hat, k, cond, sigmas, p, info):
     lcam, ldepth = ab.lift_descriptors(cam, depth, p)
     s_out = sm.summary_of_state(z_ex, state.z_a, lcam, ldepth, q_next, h, p.eps_nu, p.sketch_seed)
     r = sm.rms(z_ex.astype(np.float64) - z_k.astype(np.float64)) / (sm.rms(z_k) + p.eps)
-    rec = sg.Record(s_in=np.array(s_in), s_out=s_out, s_dphi=s_out - s_in, z_out=z_ex,
+    rec = sg.Record(s_in=np.array(s_in), s_out=s_out, s_dphi=s_out - s_in, z_out=z_ex, z_in=_f32(z_k),
                     q_in=q_k, q_out=q_next, r=r, cam=cam.copy(), depth=depth.copy())
     state.bank.append(rec)
     if len(state.bank) > p.bank_capacity:

@@ -39,6 +39,7 @@ class Record:
     r: float = 0.0              # rms(z_out - z_in) / rms(z_in), feeds h(H)
     cam: np.ndarray = field(default_factory=lambda: np.zeros(4))
     depth: np.ndarray = field(default_factory=lambda: np.zeros(4))
+    z_in: np.ndarray = None     # exact input latent (float32; read only by the residual reading)
 
 
 def _softmax(x):
@@ -104,6 +105,25 @@ def observe(kappa, bank, chunk=1 << 24):
         acc = np.zeros(min(chunk, n - s0), dtype=np.float64)
         for i, rec in enumerate(bank):
             acc += kappa[i] * rec.z_out.reshape(-1)[s0:s0 + chunk].astype(np.float64)
+        out[s0:s0 + chunk] = acc
+    return out
+
+
+def observe_residual(kappa, bank, z_t, chunk=1 << 24):
+    """Residual reading of Eq. 5: z_hat = z_t + sum_i kappa_i (z_out_i - z_in_i),
+    accumulated in fp64.  Eq. 5 as printed blends the stored outputs
+    themselves (``observe``), a convex combination that cannot move past the
+    bank; this reading blends the records' exact displacements and applies
+    them to the current latent."""
+    z_t = np.asarray(z_t).reshape(-1)
+    n = z_t.size
+    out = np.zeros(n, dtype=np.float64)
+    for s0 in range(0, n, chunk):
+        acc = z_t[s0:s0 + chunk].astype(np.float64)
+        for i, rec in enumerate(bank):
+            zo = rec.z_out.reshape(-1)[s0:s0 + chunk].astype(np.float64)
+            zi = rec.z_in.reshape(-1)[s0:s0 + chunk].astype(np.float64)
+            acc = acc + kappa[i] * (zo - zi)
         out[s0:s0 + chunk] = acc
     return out
 

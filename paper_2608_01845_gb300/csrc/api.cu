@@ -106,7 +106,7 @@ wdc_status check_params(Ctx* c, const wdc_cache_params& p) {
     if (!(p.lambda_ >= 0)) return fail(c, WDC_ERR_INVALID_ARG, "lambda must be >= 0");
     if (p.min_support < 0 || p.max_age < 0 || p.n_init_exact < 0 || p.n_final_exact < 0)
         return fail(c, WDC_ERR_INVALID_ARG, "negative integer parameter");
-    if (p.flags & ~WDC_ABL_ALL) return fail(c, WDC_ERR_INVALID_ARG, "unknown ablation flag");
+    if (p.flags & ~(WDC_ABL_ALL | WDC_OBS_RESIDUAL)) return fail(c, WDC_ERR_INVALID_ARG, "unknown flag");
     if ((p.flags & WDC_ABL_PERIODIC) && p.period < 1) return fail(c, WDC_ERR_INVALID_ARG, "period must be >= 1");
     if ((p.flags & WDC_ABL_LINEAR_OBS) && !(p.ridge >= 0 && p.ridge < 1e300))
         return fail(c, WDC_ERR_INVALID_ARG, "ridge must be finite and >= 0");
@@ -158,24 +158,32 @@ void set_cond(PassArgs& a, const wdc_cond* cd) {
 }
 
 // Skip pass + async copy of the step record into `dst` (pinned); no sync.
-// z_cur (the current latent) is read only by the secant ablation.
+bool needs_disp(const Ctx* c) { return c->prm.flags & (WDC_ABL_SECANT | WDC_OBS_RESIDUAL); }
+
+// z_cur (the current latent) is read only by the secant and the residual reading.
 wdc_status enqueue_skip(Ctx* c, int k, const wdc_cond* cd, const float* z_cur, float* z_hat, StepOut* dst,
                         cudaStream_t s) {
     PassArgs a = base_args(c, k);
     set_cond(a, cd);
     a.nsrc = c->n_bank;
     for (int i = 0; i < c->n_bank; ++i) a.slot[i] = slot_of(c, i);
-    const bool secant = c->prm.flags & WDC_ABL_SECANT;
-    if (secant) {
-        if (!z_cur || !c->secant) return fail(c, WDC_ERR_STATE, "secant candidate needs the current latent");
+    int mode = kModeSkip;
+    if (needs_disp(c) && (!z_cur || !c->disp[0]))
+        return fail(c, WDC_ERR_STATE, "this candidate needs the current latent and the displacement buffers");
+    if (c->prm.flags & WDC_ABL_SECANT) {
+        mode = kModeSecant;
         a.src[0] = z_cur;
-        a.src[1] = c->secant;
+        a.src[1] = c->disp[c->n_bank > 0 ? newest_slot(c) : 0];
+    } else if (c->prm.flags & WDC_OBS_RESIDUAL) {
+        mode = kModeResidual;
+        a.zcur = z_cur;
+        for (int i = 0; i < c->n_bank; ++i) a.src[i] = c->disp[a.slot[i]];
     } else {
         for (int i = 0; i < c->n_bank; ++i) a.src[i] = c->bank[a.slot[i]];
     }
     a.anchor = anchor_ptr(c);
     a.out = z_hat;
-    wdc_status st = launch_pass(c, secant ? kModeSecant : kModeSkip, a, s);
+    wdc_status st = launch_pass(c, mode, a, s);
     if (st) return st;
     WDC_CUDA_TRY(c, cudaMemcpyAsync(dst, &c->st->out, sizeof(StepOut), cudaMemcpyDeviceToHost, s));
     return WDC_OK;
@@ -192,7 +200,7 @@ wdc_status enqueue_anchor(Ctx* c, int k, const wdc_cond* cd, const float* z_t, c
     a.zcf = z_cf;
     a.anchor = anchor_ptr(c);
     a.out = c->bank[ins];
-    a.out2 = (c->prm.flags & WDC_ABL_SECANT) ? c->secant : nullptr;
+    a.out2 = needs_disp(c) ? c->disp[ins] : nullptr;
     a.ins_slot = ins;
     a.dsig = (float)(c->sigma[k + 1] - c->sigma[k]);
     wdc_status st = launch_pass(c, kModeAnchor, a, s);
@@ -208,16 +216,20 @@ wdc_status enqueue_anchor(Ctx* c, int k, const wdc_cond* cd, const float* z_t, c
     return WDC_OK;
 }
 
-// The secant ablation's displacement buffer (allocated on first use, zeroed).
-wdc_status ensure_secant(Ctx* c) {
-    if (!(c->prm.flags & WDC_ABL_SECANT) || c->secant) return WDC_OK;
-    WDC_CUDA_TRY(c, cudaMalloc((void**)&c->secant, c->n * sizeof(float)));
-    WDC_CUDA_TRY(c, cudaMemset(c->secant, 0, c->n * sizeof(float)));
+// Per-slot exact-step displacements for the secant and the residual reading
+// (allocated on first use, zeroed).
+wdc_status ensure_disp(Ctx* c) {
+    if (!needs_disp(c) || c->disp[0]) return WDC_OK;
+    for (int i = 0; i < c->prm.bank_capacity; ++i) {
+        WDC_CUDA_TRY(c, cudaMalloc((void**)&c->disp[i], c->n * sizeof(float)));
+        WDC_CUDA_TRY(c, cudaMemset(c->disp[i], 0, c->n * sizeof(float)));
+    }
     return WDC_OK;
 }
 
-wdc_status clear_secant(Ctx* c, cudaStream_t s) {
-    if (c->secant) WDC_CUDA_TRY(c, cudaMemsetAsync(c->secant, 0, c->n * sizeof(float), s));
+wdc_status clear_disp(Ctx* c, cudaStream_t s) {
+    for (int i = 0; i < kMaxBank; ++i)
+        if (c->disp[i]) WDC_CUDA_TRY(c, cudaMemsetAsync(c->disp[i], 0, c->n * sizeof(float), s));
     return WDC_OK;
 }
 
@@ -310,7 +322,7 @@ wdc_status wdc_create(const wdc_dit_config* cfg, const wdc_schedule* sched, cons
     if (!dm((void**)&c->cand[0], lat) || !dm((void**)&c->cand[1], lat)) return bail(WDC_ERR_OOM);
     if (!dm((void**)&c->vbuf, lat)) return bail(WDC_ERR_OOM);
     if (cudaMallocHost((void**)&c->out_host, sizeof(StepOut) * (sched->T + 2)) != cudaSuccess) return bail(WDC_ERR_OOM);
-    if ((st = ensure_secant(c))) return bail(st);
+    if ((st = ensure_disp(c))) return bail(st);
     if (cfg->layers > 0) {
         if ((st = dit_create(c))) return bail(st);
     }
@@ -333,7 +345,7 @@ void wdc_destroy(wdc_ctx* h) {
     cudaFree(c->cand[1]);
     cudaFree(c->vbuf);
     cudaFree(c->zstage);
-    cudaFree(c->secant);
+    for (int i = 0; i < kMaxBank; ++i) cudaFree(c->disp[i]);
     if (c->out_host) cudaFreeHost(c->out_host);
     for (int k = 0; k < WDC_K_COUNT; ++k)
         for (cudaEvent_t e : c->ev[k]) cudaEventDestroy(e);
@@ -349,7 +361,7 @@ wdc_status wdc_set_cache_params(wdc_ctx* h, const wdc_cache_params* params) {
         return fail(c, WDC_ERR_INVALID_ARG, "bank_capacity cannot change after wdc_create");
     c->prm = *params;
     cudaSetDevice(c->device);
-    return ensure_secant(c);
+    return ensure_disp(c);
 }
 
 const char* wdc_last_error(const wdc_ctx* h) {
@@ -475,7 +487,7 @@ wdc_status wdc_state_reset(wdc_ctx* h, const float* z_T, wdc_stream stream) {
     c->anchor_is_init = 1;
     c->last_surrogate_k = -1;
     c->cur_latent = c->z_init;
-    wdc_status cs = clear_secant(c, s);
+    wdc_status cs = clear_disp(c, s);
     if (cs) return cs;
     DevState* hs = nullptr;
     WDC_CUDA_TRY(c, cudaMallocHost((void**)&hs, sizeof(DevState)));
@@ -576,7 +588,7 @@ wdc_status wdc_state_set(wdc_ctx* h, const wdc_state_host* in, const float* cons
     c->age = in->age;
     c->last_surrogate_k = -1;
     c->cur_latent = z_cur;
-    if (wdc_status cs = clear_secant(c, s)) return cs;
+    if (wdc_status cs = clear_disp(c, s)) return cs;
     for (int i = 0; i < in->n_bank; ++i)
         WDC_CUDA_TRY(c, cudaMemcpyAsync(c->bank[i], z_out[i], c->n * sizeof(float), cudaMemcpyDeviceToDevice, s));
     if (in->n_bank == 0) {

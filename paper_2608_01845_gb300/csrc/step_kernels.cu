@@ -12,6 +12,10 @@
 //    decays R and inserts the record (section "Reliability Decision").
 //  * stats pass  (state reset/set): statistics of the current latent and the
 //    anchor.
+//  * variants of the skip pass's stream: the native latent secant (ablation,
+//    z_hat = z_k + alpha (z_a - z_a,in)) and the residual reading of Eq. 5
+//    (z_hat = z_k + sum_i kappa_i (z_out_i - z_in_i)); the anchor pass then
+//    also stores the slot's displacement z_exact - z_k.
 //
 // Summary statistics: because the summary's latent blocks are a linear sketch
 // S of RMS-normalised vectors, S(nu(z)) = S(z)/(rms(z)+eps_nu) and
@@ -306,7 +310,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
     bool do_stream = true;
     float kap[K > 0 ? K : 1];
     float alpha_f = 0.f;
-    if (MODE == kModeSkip) {
+    if (MODE == kModeSkip || MODE == kModeResidual) {
         skip_head<K>(a, hs);
         do_stream = (K > 0) && hs.supported;
 #pragma unroll
@@ -365,6 +369,19 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                     for (int i = 1; i < K; ++i) {
                         zh.x = fmaf(kap[i], x[i].x, zh.x); zh.y = fmaf(kap[i], x[i].y, zh.y);
                         zh.z = fmaf(kap[i], x[i].z, zh.z); zh.w = fmaf(kap[i], x[i].w, zh.w);
+                    }
+                    *reinterpret_cast<float4*>(a.out + base) = zh;
+                    o[0] = zh.x; o[1] = zh.y; o[2] = zh.z; o[3] = zh.w;
+                    sa[0] = za.x; sa[1] = za.y; sa[2] = za.z; sa[3] = za.w;
+                } else if constexpr (MODE == kModeResidual && K > 0) {
+                    // residual reading: z_hat = z_k + sum_i kappa_i (z_out_i - z_in_i)
+                    float4 zh = __ldg(reinterpret_cast<const float4*>(a.zcur + base));
+                    const float4 za = __ldg(reinterpret_cast<const float4*>(a.anchor + base));
+#pragma unroll
+                    for (int i = 0; i < K; ++i) {
+                        const float4 d = __ldg(reinterpret_cast<const float4*>(a.src[i] + base));
+                        zh.x = fmaf(kap[i], d.x, zh.x); zh.y = fmaf(kap[i], d.y, zh.y);
+                        zh.z = fmaf(kap[i], d.z, zh.z); zh.w = fmaf(kap[i], d.w, zh.w);
                     }
                     *reinterpret_cast<float4*>(a.out + base) = zh;
                     o[0] = zh.x; o[1] = zh.y; o[2] = zh.z; o[3] = zh.w;
@@ -429,6 +446,13 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                         a.out[idx] = zh;
                         o[e] = zh;
                         sa[e] = a.anchor[idx];
+                    } else if constexpr (MODE == kModeResidual && K > 0) {
+                        float zh = a.zcur[idx];
+#pragma unroll
+                        for (int i = 0; i < K; ++i) zh = fmaf(kap[i], a.src[i][idx], zh);
+                        a.out[idx] = zh;
+                        o[e] = zh;
+                        sa[e] = a.anchor[idx];
                     } else if constexpr (MODE == kModeSecant) {
                         const float zh = fmaf(alpha_f, a.src[1][idx], a.src[0][idx]);
                         a.out[idx] = zh;
@@ -460,7 +484,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                 const float d = x - sa[e];
                 const uint32_t idx = (uint32_t)(base + e);
                 sg += signed_term(idx, seed, x);
-                if (MODE == kModeSkip || MODE == kModeObserve || MODE == kModeSecant) {
+                if (MODE == kModeSkip || MODE == kModeObserve || MODE == kModeSecant || MODE == kModeResidual) {
                     fac[0] += x * x;
                     fac[1] += d * d;
                     nonfinite += isfinite(x) ? 0 : 1;
@@ -572,7 +596,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
         return;
     }
 
-    if (MODE == kModeSkip || MODE == kModeSecant) {
+    if (MODE == kModeSkip || MODE == kModeSecant || MODE == kModeResidual) {
         if (t < kSummary) st->s_phi[t] = hs.phi[t];
         // the secant needs no retrieval: its support term holds with a non-empty bank
         const int supported = (MODE == kModeSecant) ? (a.nsrc > 0) : ((K > 0) && hs.supported);
@@ -723,8 +747,9 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
 }
 
 template <int K>
-void launch_skip(const PassArgs& a, int grid, cudaStream_t s) {
-    pass_kernel<kModeSkip, K><<<grid, kThreads, 0, s>>>(a);
+void launch_skip(const PassArgs& a, int grid, cudaStream_t s, bool residual) {
+    if (residual) pass_kernel<kModeResidual, K><<<grid, kThreads, 0, s>>>(a);
+    else pass_kernel<kModeSkip, K><<<grid, kThreads, 0, s>>>(a);
 }
 
 }  // namespace
@@ -739,7 +764,8 @@ int pass_grid(const Ctx* c) {
 
 wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s) {
     const int grid = pass_grid(c);
-    LaunchScope ls(c, (mode == kModeSkip || mode == kModeSecant) ? WDC_K_SKIP
+    const bool skip_like = mode == kModeSkip || mode == kModeSecant || mode == kModeResidual;
+    LaunchScope ls(c, skip_like ? WDC_K_SKIP
                                                                  : (mode == kModeAnchor ? WDC_K_ANCHOR : WDC_K_OTHER),
                    s);
     switch (mode) {
@@ -747,19 +773,22 @@ wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s) {
         case kModeAnchor: pass_kernel<kModeAnchor, 0><<<grid, kThreads, 0, s>>>(a); break;
         case kModeSecant: pass_kernel<kModeSecant, 0><<<grid, kThreads, 0, s>>>(a); break;
         case kModeSkip:
+        case kModeResidual: {
+            const bool r = mode == kModeResidual;
             switch (a.nsrc) {
-                case 0: launch_skip<0>(a, grid, s); break;
-                case 1: launch_skip<1>(a, grid, s); break;
-                case 2: launch_skip<2>(a, grid, s); break;
-                case 3: launch_skip<3>(a, grid, s); break;
-                case 4: launch_skip<4>(a, grid, s); break;
-                case 5: launch_skip<5>(a, grid, s); break;
-                case 6: launch_skip<6>(a, grid, s); break;
-                case 7: launch_skip<7>(a, grid, s); break;
-                case 8: launch_skip<8>(a, grid, s); break;
+                case 0: launch_skip<0>(a, grid, s, r); break;
+                case 1: launch_skip<1>(a, grid, s, r); break;
+                case 2: launch_skip<2>(a, grid, s, r); break;
+                case 3: launch_skip<3>(a, grid, s, r); break;
+                case 4: launch_skip<4>(a, grid, s, r); break;
+                case 5: launch_skip<5>(a, grid, s, r); break;
+                case 6: launch_skip<6>(a, grid, s, r); break;
+                case 7: launch_skip<7>(a, grid, s, r); break;
+                case 8: launch_skip<8>(a, grid, s, r); break;
                 default: return fail(c, WDC_ERR_INVALID_ARG, "bank size out of range");
             }
             break;
+        }
         default: return fail(c, WDC_ERR_INVALID_ARG, "unknown pass mode");
     }
     cudaError_t e = cudaGetLastError();

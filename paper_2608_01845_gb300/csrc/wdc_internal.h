@@ -67,20 +67,22 @@ struct ParamsDev {
     double ridge;                                    // linear observation
 };
 
-enum StreamMode { kModeStats = 0, kModeSkip = 1, kModeAnchor = 2, kModeObserve = 3, kModeSecant = 4 };
+enum StreamMode { kModeStats = 0, kModeSkip = 1, kModeAnchor = 2, kModeObserve = 3, kModeSecant = 4, kModeResidual = 5 };
 
 // Launch arguments of the fused latent-pass kernels (passed by value).
 struct PassArgs {
     long long n;
     int nsrc;                          // skip: records in age order (oldest first)
     const float* src[kMaxBank];        // skip: bank latents by age; anchor/stats: src[0] = z_k;
-                                       // secant: src[0] = z_k, src[1] = z_a - z_a,in
+                                       // secant: src[0] = z_k, src[1] = z_a - z_a,in;
+                                       // residual: the records' displacements by age
     int slot[kMaxBank];                // ring slot of each record, by age
     const float* anchor;               // z_a
+    const float* zcur;                 // residual: z_k
     const float* v;                    // anchor: velocity
     const float* zcf;                  // anchor: counterfactual candidate or nullptr
     float* out;                        // skip: z_hat; anchor: z_exact (bank slot)
-    float* out2;                       // anchor: z_exact - z_k (secant displacement) or nullptr
+    float* out2;                       // anchor: z_exact - z_k (the slot's displacement) or nullptr
     float dsig;                        // anchor: sigma_{k+1} - sigma_k (fp32)
     int k, T, age, ins_slot;
     double q_k, q_next;
@@ -117,8 +119,8 @@ struct Ctx {
     float* cand[2] = {};               // rollout candidate buffers
     float* vbuf = nullptr;
     float* zstage = nullptr;           // host-pointer staging for rollouts
-    float* secant = nullptr;           // WDC_ABL_SECANT: z_a - z_a,in of the latest exact step
-    const float* cur_latent = nullptr; // current latent of the step API (read by the secant)
+    float* disp[kMaxBank] = {};        // secant / residual reading: z_out - z_in per bank slot
+    const float* cur_latent = nullptr; // current latent of the step API (read by secant / residual)
 
     // host mirror of the discrete state
     int n_bank = 0, head = 0, age = 0;

@@ -69,6 +69,7 @@ ABL_NO_CALIB = 0x10
 ABL_NO_SUPPORT = 0x20
 ABL_LINEAR_OBS = 0x40
 ABL_NO_COND = 0x80
+OBS_RESIDUAL = 0x100      # residual reading of Eq. 5 (not an ablation)
 
 
 class Cond(ctypes.Structure):

@@ -47,6 +47,8 @@ def test_ablation_flags_and_defaults_match_the_header():
     for n in names:
         assert getattr(wdc, "ABL_" + n) == hdr[n]
     assert hdr["ALL"] == sum(hdr[n] for n in names)
+    m = re.search(r"#define WDC_OBS_RESIDUAL\s+0x([0-9A-Fa-f]+)", src)
+    assert int(m.group(1), 16) == wdc.OBS_RESIDUAL and not (wdc.OBS_RESIDUAL & hdr["ALL"])
     p = wdc.default_params()
     assert p.period == 8 and p.ridge == 1e-6
 

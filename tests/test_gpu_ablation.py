@@ -1,5 +1,5 @@
-"""Ablation variants (section "Ablation Study", Tables 3 and 4) on the GPU
-against the CPU checker: the cfg0 model (2 layers, D=256, latent
+"""Ablation variants (section "Ablation Study", Tables 3 and 4) and the
+residual reading of Eq. 5 on the GPU against the CPU checker: the cfg0 model (2 layers, D=256, latent
 16x4x16x16, fp32 parity mode) rolled out under each variant, one flag at a
 time plus the core factorization (periodic / risk x secant / lifted).  The
 decision sequence must be identical and the final latent within 1e-5
@@ -30,6 +30,8 @@ VARIANTS = {
     "no_support": dict(flags=wdc.ABL_NO_SUPPORT, sim_min=0.3),
     "linear_obs": dict(flags=wdc.ABL_LINEAR_OBS),
     "no_condition": dict(flags=wdc.ABL_NO_COND),
+    "residual": dict(flags=wdc.OBS_RESIDUAL),
+    "residual+linear_obs": dict(flags=wdc.OBS_RESIDUAL | wdc.ABL_LINEAR_OBS),
 }
 
 

@@ -210,3 +210,44 @@ def test_no_condition_drops_descriptors_from_the_lift_only():
         assert np.array_equal(ta["kappa"], tb["kappa"])
         if ta["k"] > 1:
             assert ta["p"] != tb["p"]                          # the controller still sees them
+
+
+# ------------------------------------------------------------------ residual reading of Eq. 5
+def test_residual_observation_closed_forms():
+    g = np.random.default_rng(9)
+    z_t = g.standard_normal(512).astype(np.float32)
+    D = g.standard_normal(512).astype(np.float32)
+    # every record carries the same displacement: z_t + D for any weights summing to 1
+    bank = []
+    for i in range(3):
+        zi = g.standard_normal(512).astype(np.float32)
+        r = _rec(np.zeros(256), (zi.astype(np.float64) + D).astype(np.float32))
+        r.z_in = zi
+        bank.append(r)
+    kap = np.array([0.2, 0.5, 0.3])
+    want = z_t.astype(np.float64) + sum(kap[i] * (bank[i].z_out.astype(np.float64) - bank[i].z_in) for i in range(3))
+    got = sg.observe_residual(kap, bank, z_t)
+    assert np.allclose(got, want, rtol=0, atol=1e-12)
+    assert np.allclose(got, z_t.astype(np.float64) + D, rtol=0, atol=1e-5)
+    # a single record: z_t + (z_out - z_in)
+    one = sg.observe_residual(np.array([1.0]), bank[:1], z_t)
+    assert np.allclose(one, z_t.astype(np.float64) + bank[0].z_out.astype(np.float64) - bank[0].z_in, atol=1e-12)
+
+
+def test_residual_reading_is_exact_for_a_constant_velocity_field():
+    # uniform schedule, v(z) = c: every exact displacement is dsigma c, so
+    # z_t + sum kappa_i (z_out_i - z_in_i) is the exact Euler step whatever
+    # the weights; Eq. 5 as printed instead returns a blend of past latents
+    from oracle.params import OBS_RESIDUAL
+    g = np.random.default_rng(10)
+    c = g.standard_normal(1024)
+    F = lambda z, t, cond, k: c
+    s = sch.sigmas(16)
+    z0 = synth.latent(13, (1024,))
+    p = CacheParams(tau_risk=1e9, sim_min=-1.0, q_gap_max=1.0, flags=OBS_RESIDUAL)
+    zc, dec, _ = ro.cached_rollout(z0, F, {}, s, p)
+    assert sum(dec) >= 10
+    zn = ro.native_rollout(z0, F, {}, s)
+    assert np.max(np.abs(zc - zn)) < 1e-5 * (1 + np.max(np.abs(zn)))
+    zp, dec_p, _ = ro.cached_rollout(z0, F, {}, s, CacheParams(tau_risk=1e9, sim_min=-1.0, q_gap_max=1.0))
+    assert dec_p == dec and np.max(np.abs(zp - zn)) > 0.1        # the printed reading does not advance
