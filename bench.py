@@ -51,7 +51,7 @@ WORKLOAD_13B = dict(
     name="cached rollout, 60-layer dual-stream bf16 DiT 3072/24x128/12288 (~14.7B), latent 16x13x64x64 + 256 cond tokens, T=50",
     layers=60, hidden=3072, heads=24, head_dim=128, mlp=12288, temb_dim=512, freq_dim=256,
     in_ch=16, frames=13, height=64, width=64, patch=2, cond_tokens=256, cond_dim=3072, dual_stream=1,
-    T=50, tau_risk=0.1, target_exact=10, weight_seed=4321, input_seed=91,
+    T=50, tau_risk=0.8, target_exact=10, weight_seed=4321, input_seed=91,
 )
 WORKLOADS = {"5b": WORKLOAD_5B, "13b": WORKLOAD_13B}
 SKIP_SWEEP_N = 1 << 28          # fused skip pass measured at 2^28 fp32 elements, bank of 4
@@ -84,6 +84,13 @@ def block_flops(w):
     gemm = 2 * L * D * 3 * D + 2 * L * D * D + 2 * 2 * L * D * M
     attn = 4 * w["heads"] * L * L * w["head_dim"]
     return gemm, attn
+
+
+def weight_gb(w):
+    """bf16 weight bytes read per forward (block matrices of every stream)."""
+    D, M = w["hidden"], w["mlp"]
+    per_stream = 3 * D * D + D * D + 2 * D * M
+    return w["layers"] * (2 if w["dual_stream"] else 1) * per_stream * 2 / 1e9
 
 
 def forward_flops(w):
@@ -163,6 +170,7 @@ def cpu_sample(w, exact_steps, rows=16):
     cfgd = {k: w[k] for k in ["hidden", "heads", "head_dim", "mlp", "temb_dim", "freq_dim", "in_ch", "frames",
                               "height", "width", "patch", "cond_tokens", "cond_dim", "dual_stream"]}
     cfgd["layers"] = 1
+    cfgd["dual_stream"] = 0      # the timing sample prices flops; a dual-stream block has the same count
     cfg = DiTConfig(**cfgd)
     names = [f"L0.s0.{n}" for n in ["qkv.w", "qkv.b", "o.w", "o.b", "fc1.w", "fc1.b", "fc2.w", "fc2.b"]]
     W = synth.dit_weights(cfgd, 5, bf16=True, names=names)
@@ -208,7 +216,7 @@ def run_reference(args, rank, world):
     """The CPU checker as the reference arm: each step is one bounded sample."""
     if rank != 0:
         return
-    w = WORKLOAD_5B
+    w = WORKLOADS[args.workload]
     vals = []
     desc = ""
     for i in range(args.warmup + args.steps):
@@ -231,15 +239,15 @@ def kernel_hash(path):
     return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
 
 
-def traffic_for(kernel_file):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel's
-    source is unchanged since the counters were taken."""
+def traffic_for(kernel_file, workload):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on this workload's launch and the kernel's source is unchanged since."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
     d = json.load(open(p))
     e = d.get(os.path.basename(kernel_file))
-    if not e:
+    if not e or e.get("bench_workload") != workload:
         return None
     if e.get("source_sha256_16") != kernel_hash(kernel_file):
         return None
@@ -295,10 +303,10 @@ def skip_pass_gbps(torch, wdc, peaks, secant=False):
 
 
 def block_tflops(torch, ctx, w, peaks):
-    """One DiT block (the 5B-scale block operator) in place on [17776, 3072]."""
+    """One DiT block of the workload in place on [L, D]."""
     L, D = tokens(w), w["hidden"]
     x = torch.randn(L, D, device="cuda").bfloat16()
-    mod = 0.1 * torch.randn(6, D, device="cuda")
+    mod = 0.1 * torch.randn((2 if w["dual_stream"] else 1) * 6, D, device="cuda")
     for _ in range(3):
         ctx.dit_block_forward(0, x, mod)
     torch.cuda.synchronize()
@@ -339,7 +347,7 @@ def run_gpu(args, rank, world, local_rank):
     import torch.distributed as dist
     from paper_2608_01845_gb300 import wdc
     torch.cuda.set_device(local_rank)
-    w = WORKLOAD_5B
+    w = WORKLOADS[args.workload]
     T = w["T"]
     peaks, peak_src = load_peaks()
     params = wdc.make_params(tau_risk=w["tau_risk"], **(ABLATIONS[args.ablation] if args.ablation else {}))
@@ -394,16 +402,18 @@ def run_gpu(args, rank, world, local_rank):
         avg_ms = prof["attention"][0] / prof["attention"][1]
         achieved = block_flops(w)[1] / (avg_ms * 1e-3) / 1e12
         kfile = os.path.join(ROOT, "paper_2608_01845_gb300", "csrc", "attn_tc.cu")
-        kname = "attn_tc_kernel<64> (48 heads x 17776 tokens x 64)"
+        kname = f"attn_tc_kernel<{w['head_dim']}> ({w['heads']} heads x {tokens(w)} tokens x {w['head_dim']})"
+        traffic = traffic_for(kfile, args.workload)
     else:
         avg_ms = prof["gemm"][0] / prof["gemm"][1]
         achieved = n_fwd * fwd_gemm / (prof["gemm"][0] * 1e-3) / 1e12
         kfile = os.path.join(ROOT, "paper_2608_01845_gb300", "csrc", "gemm_tc.cu")
-        kname = "gemm_tc_kernel (all denoiser GEMMs)"
+        kname = "gemm_tc2_kernel / gemm_tc_kernel (all denoiser GEMMs)"
+        traffic = None          # an aggregate over several shapes has no per-launch capture
     peak = peaks["bf16_tflops_sustained"]
     roofline = {"bound": "tensor", "kernel": kname, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "peak_source": f"{peak_src} sustained bf16 (kernel timed inside a long step)",
-                "avg_launch_ms": avg_ms, "launches_timed": int(prof[dom][1]), "traffic": traffic_for(kfile),
+                "avg_launch_ms": avg_ms, "launches_timed": int(prof[dom][1]), "traffic": traffic,
                 "time_share": {k: v / sum(cls_time.values()) for k, v in cls_time.items()}}
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -411,7 +421,7 @@ def run_gpu(args, rank, world, local_rank):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": w["name"] + (f", ablation {args.ablation}" if args.ablation else ""),
                        "T": T, "tau_risk": w["tau_risk"], "bank_capacity": 4,
-                       "l2": "inputs larger than L2 (10.3 GB of weights per forward)",
+                       "l2": f"inputs larger than L2 ({weight_gb(w):.1f} GB of weights per forward)",
                        "parallelism": f"replicas x{world}"},
             "exact_steps_per_rollout": exact, "gpu_launches": launches, "clocks": clk, "roofline": roofline}
 
@@ -522,7 +532,8 @@ def main():
                     help="time one operator at its 5B-scale shape (profiler captures)")
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="5b",
-                    help="shape of --op (5b: 48x64 heads, L=17776; 13b: 24x128 heads, L=13568, dual stream)")
+                    help="rollout / --op shape (5b: 42 layers, 48x64 heads, L=17776; 13b: 60 dual-stream layers, "
+                         "24x128 heads, L=13568)")
     args = ap.parse_args()
     if args.op:
         return run_op(args)

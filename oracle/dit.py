@@ -179,27 +179,43 @@ def block(x, Wt, cfg, layer, mod):
 def block_rows(x, Wt, cfg, layer, mod, rows_idx):
     """The same block, evaluated only for the query rows ``rows_idx``.
 
-    Keys and values are computed for every token (attention is joint), queries,
-    attention, out-projection and MLP only for the selected rows.  Single-stream
-    models only.  Returns [len(rows_idx), D].
+    Keys and values are computed for every token (attention is joint), each
+    token with its own stream's weights and modulation; queries, attention,
+    out-projection and MLP only for the selected rows.  Returns
+    [len(rows_idx), D].
     """
-    if cfg.dual_stream:
-        raise NotImplementedError("block_rows: single-stream only")
-    m = mod[0]
-    D = x.shape[1]
-    pre = f"L{layer}.s0."
-    Wqkv = np.asarray(Wt[pre + "qkv.w"], dtype=np.float64)
-    bqkv = np.asarray(Wt[pre + "qkv.b"], dtype=np.float64)
-    h = modulate(layer_norm(x), m[0], m[1])
-    kv = h @ Wqkv[D:].T + bqkv[D:]
-    hq = h[rows_idx]
-    q = hq @ Wqkv[:D].T + bqkv[:D]
-    o = attention(q, kv[:, :D], kv[:, D:], cfg.heads)
-    xr = x[rows_idx].copy()
-    xr += m[2] * linear(o, Wt[pre + "o.w"], Wt[pre + "o.b"])
-    h2 = modulate(layer_norm(xr), m[3], m[4])
-    xr += m[5] * linear(gelu_tanh(linear(h2, Wt[pre + "fc1.w"], Wt[pre + "fc1.b"])), Wt[pre + "fc2.w"], Wt[pre + "fc2.b"])
-    return xr
+    L, D = x.shape
+    rows = _stream_rows(cfg, L)
+    rows_idx = np.asarray(rows_idx)
+    stream_of = np.empty(L, dtype=np.int64)
+    for s, (r0, r1) in enumerate(rows):
+        stream_of[r0:r1] = s
+    h = np.empty_like(x, dtype=np.float64)
+    kv = np.empty((L, 2 * D))
+    for s, (r0, r1) in enumerate(rows):
+        m = mod[s]
+        pre = f"L{layer}.s{s}."
+        Wqkv = np.asarray(Wt[pre + "qkv.w"], dtype=np.float64)
+        bqkv = np.asarray(Wt[pre + "qkv.b"], dtype=np.float64)
+        h[r0:r1] = modulate(layer_norm(x[r0:r1]), m[0], m[1])
+        kv[r0:r1] = h[r0:r1] @ Wqkv[D:].T + bqkv[D:]
+    out = np.empty((len(rows_idx), D))
+    for s, (r0, r1) in enumerate(rows):
+        sel = np.nonzero(stream_of[rows_idx] == s)[0]
+        if sel.size == 0:
+            continue
+        m = mod[s]
+        pre = f"L{layer}.s{s}."
+        Wqkv = np.asarray(Wt[pre + "qkv.w"], dtype=np.float64)
+        bqkv = np.asarray(Wt[pre + "qkv.b"], dtype=np.float64)
+        q = h[rows_idx[sel]] @ Wqkv[:D].T + bqkv[:D]
+        o = attention(q, kv[:, :D], kv[:, D:], cfg.heads)
+        xr = x[rows_idx[sel]].astype(np.float64)
+        xr += m[2] * linear(o, Wt[pre + "o.w"], Wt[pre + "o.b"])
+        h2 = modulate(layer_norm(xr), m[3], m[4])
+        xr += m[5] * linear(gelu_tanh(linear(h2, Wt[pre + "fc1.w"], Wt[pre + "fc1.b"])), Wt[pre + "fc2.w"], Wt[pre + "fc2.b"])
+        out[sel] = xr
+    return out
 
 
 def embed(Wt, cfg, z, cond_tokens):

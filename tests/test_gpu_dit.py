@@ -149,6 +149,39 @@ def test_bf16_block_5b_scale_sampled_rows():
     assert rel_l2(got, want) <= BF16_TOL
 
 
+BLOCK13B = dict(layers=1, hidden=3072, heads=24, head_dim=128, mlp=12288, temb_dim=512, freq_dim=256, in_ch=16,
+                frames=13, height=64, width=64, patch=2, cond_tokens=256, cond_dim=3072, dual_stream=1)
+
+
+def test_bf16_dual_stream_block_13b_scale_sampled_rows():
+    """One dual-stream block at the HunyuanVoyager-13B-like shape (L = 256 +
+    13312 = 13568 tokens, 24 x 128 heads): separate weights and modulation for
+    the condition and video rows, joint attention; 256 seeded rows (both
+    streams) compared with fp64."""
+    cfgd = BLOCK13B
+    ctx = _ctx(cfgd, wdc.BF16)
+    names = [f"L0.s{s}.{n}" for s in range(2) for n in ["qkv.w", "qkv.b", "o.w", "o.b", "fc1.w", "fc1.b", "fc2.w", "fc2.b"]]
+    W = synth.dit_weights(cfgd, 6, std=0.02, bias_std=0.02, bf16=True, names=names)
+    ctx.set_weights(W)
+    L, D = 13568, 3072
+    x = _bf(synth.normal(41, (L, D)))
+    mod = synth.normal(42, (12, D), 0.3)
+    for g in (2, 5, 8, 11):                       # gates of order one in both streams
+        mod[g] = 1.0 + mod[g]
+    xt = _to_dev(x, torch.bfloat16)
+    ctx.dit_block_forward(0, xt, _to_dev(mod))
+    torch.cuda.synchronize()
+    g = np.random.default_rng(43)
+    rows = np.sort(np.concatenate([g.choice(256, 32, replace=False), 256 + g.choice(L - 256, 224, replace=False)]))
+    got = xt.float().cpu().numpy()[rows]
+    mods = [mod[:6].astype(np.float64), mod[6:].astype(np.float64)]
+    want = dit.block_rows(x.astype(np.float64), W, DiTConfig(**cfgd), 0, mods, rows)
+    assert rel_l2(got - x[rows], want - x[rows]) <= BF16_TOL
+    assert rel_l2(got, want) <= BF16_TOL
+    cond = rows < 256
+    assert rel_l2(got[cond] - x[rows][cond], want[cond] - x[rows][cond]) <= BF16_TOL
+
+
 @pytest.mark.parametrize("H,L,d", [(48, 17776, 64), (24, 13568, 128)])
 def test_bf16_attention_full_size_sampled_rows(H, L, d):
     """The attention shapes of the 5B-scale (48 x 64 heads, L = 17776) and

@@ -122,6 +122,17 @@ def test_linear_and_block_rows_consistency():
             assert abs(y[i, o] - (sum(x[i, j] * float(Wl[o, j]) for j in range(cfg.hidden)) + float(b[o]))) < 1e-12
 
 
+def test_dual_stream_block_rows_consistency():
+    # condition rows (stream 1) and video rows (stream 0) against the full block
+    cfg = _tiny_cfg(dual_stream=1)
+    W = synth.dit_weights(cfg.as_dict(), 15, std=0.2, bias_std=0.1)
+    x = np.random.default_rng(15).standard_normal((cfg.tokens, cfg.hidden))
+    mods = [np.random.default_rng(16 + s).standard_normal((6, cfg.hidden)) * 0.3 for s in range(2)]
+    full = dit.block(x, W, cfg, 1, mods)
+    rows = np.array([0, cfg.cond_tokens - 1, cfg.cond_tokens, cfg.tokens - 1])
+    assert np.allclose(dit.block_rows(x, W, cfg, 1, mods, rows), full[rows], atol=1e-12)
+
+
 def test_zero_final_weights_give_bias_field():
     cfg = _tiny_cfg()
     W = synth.dit_weights(cfg.as_dict(), 7, std=0.2, bias_std=0.5)
