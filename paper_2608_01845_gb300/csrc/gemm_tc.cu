@@ -14,8 +14,9 @@
 //               32-lane TMEM quarter = 32 rows), bias / GELU / gated residual /
 //               QKV scatter / unpatchify, 16-byte global stores; then release
 //               the accumulator so the next tile's MMAs overlap this epilogue.
-// Tiles are visited with N fastest: the W matrix (at most 75 MB here) stays
-// in L2 while A and the output stream through once.
+// Tiles are visited N-fastest inside groups of N tiles sized so a group's
+// slab of W stays in L2 (about 40 MB), so W is read from DRAM about once and
+// A once per group.
 // Tails: TMA zero-fills rows past M / N and columns past K; the epilogue
 // masks rows >= M.  Every mbarrier wait is bounded.
 #include "dit_kernels.cuh"
@@ -41,6 +42,7 @@ constexpr size_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
 struct GemmArgs {
     int M, N, K;
     int m_tiles, n_tiles, k_blocks;
+    int group_n;            // pair kernel: N tiles per raster group
     Epi e;
     unsigned* err;
 };
@@ -300,6 +302,19 @@ constexpr uint32_t TMEM2_COLS = 512;
 constexpr uint32_t IDESC2 = idesc_bf16(256, 256);
 constexpr size_t SMEM2_BYTES = STAGES2 * STAGE2_BYTES + 1024 + 512;
 
+// Pair-kernel raster: the N tiles are split into groups of group_n; inside a
+// group the tiles run N-fastest over every 256-row M block.  A group's slab
+// of W (group_n * 256 rows * K) stays in L2 while A streams through once per
+// group, so W is read from DRAM about once and A once per group.
+__device__ __forceinline__ void pair_tile(const GemmArgs& g, int m_pairs, int tile, int& m_blk, int& n_blk) {
+    const int per_group = m_pairs * g.group_n;
+    const int grp = tile / per_group, r = tile - grp * per_group;
+    const int n_first = grp * g.group_n;
+    const int width = min(g.group_n, g.n_tiles - n_first);
+    m_blk = r / width;
+    n_blk = n_first + (r - m_blk * width);
+}
+
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ GemmArgs g) {
@@ -357,8 +372,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             for (int s = 0; s < STAGES2; ++s) armed[s] = false;
             bool ok = true;
             for (int tile = cluster_id; tile < num_tiles && ok; tile += n_clusters) {
-                const int m0 = (tile / g.n_tiles) * 256 + (int)rank * 128;
-                const int n0 = (tile % g.n_tiles) * BN + (int)rank * 128;
+                int mb, nb;
+                pair_tile(g, m_pairs, tile, mb, nb);
+                const int m0 = mb * 256 + (int)rank * 128;
+                const int n0 = nb * BN + (int)rank * 128;
                 for (int kb = 0; kb < g.k_blocks; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
                     if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * STAGE2_BYTES);
@@ -422,8 +439,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int tile = cluster_id; tile < num_tiles; tile += n_clusters) {
-            const int mrow = (tile / g.n_tiles) * 256 + (int)rank * 128;
-            const int n_blk = tile % g.n_tiles;
+            int mb, n_blk;
+            pair_tile(g, m_pairs, tile, mb, n_blk);
+            const int mrow = mb * 256 + (int)rank * 128;
             if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, g.err)) break;
             tc_fence_after();
             const int m = mrow + lg * 32 + lane;
@@ -531,6 +549,21 @@ wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, co
     g.m_tiles = (M + BM - 1) / BM;
     g.n_tiles = (N + BN - 1) / BN;
     g.k_blocks = (K + BK - 1) / BK;
+    {
+        // raster groups: a W slab of at most ~40 MB per group (L2 is 126 MB,
+        // shared with the streamed A and the output), as few groups as that
+        // allows.  For deep K (> 4096) a 256-row slab of A is itself large
+        // and re-reading A per group costs more than it saves (measured on the
+        // 17776 x 3072 x 12288 MLP-down GEMM): plain N-fastest order there.
+        g.group_n = g.n_tiles;
+        if (K <= 4096) {
+            const double slab_per_tile = 256.0 * K * 2.0;
+            int gn = (int)(40.0e6 / slab_per_tile);
+            gn = gn < 1 ? 1 : (gn > g.n_tiles ? g.n_tiles : gn);
+            const int groups = (g.n_tiles + gn - 1) / gn;
+            g.group_n = (g.n_tiles + groups - 1) / groups;  // balance the groups
+        }
+    }
     g.e = e;
     g.err = c->err;
     if (pair) {
