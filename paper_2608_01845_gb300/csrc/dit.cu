@@ -50,6 +50,11 @@ struct DiT {
     void *tok = nullptr, *condx = nullptr, *pe = nullptr;
     float *feat = nullptr, *h1 = nullptr, *temb = nullptr, *mods = nullptr;
     std::vector<void*> allocs;
+    // dual stream: the condition stream's row block runs on a second CUDA
+    // stream forked from and joined back into the caller's, so its small
+    // GEMMs fill the SMs the video GEMMs leave idle in their last wave
+    cudaStream_t aux = nullptr;
+    cudaEvent_t fork[2] = {}, join[2] = {};
 };
 
 namespace {
@@ -484,6 +489,14 @@ wdc_status dit_create(Ctx* c) {
     if ((s = dalloc(c, (void**)&t->h1, (size_t)t->E * sizeof(float)))) return s;
     if ((s = dalloc(c, (void**)&t->temb, (size_t)t->E * sizeof(float)))) return s;
     if ((s = dalloc(c, (void**)&t->mods, t->mod_rows * sizeof(float)))) return s;
+    if (t->S == 2) {
+        if (cudaStreamCreateWithFlags(&t->aux, cudaStreamNonBlocking) != cudaSuccess)
+            return fail(c, WDC_ERR_CUDA, "DiT init: auxiliary stream");
+        for (int i = 0; i < 2; ++i)
+            if (cudaEventCreateWithFlags(&t->fork[i], cudaEventDisableTiming) != cudaSuccess ||
+                cudaEventCreateWithFlags(&t->join[i], cudaEventDisableTiming) != cudaSuccess)
+                return fail(c, WDC_ERR_CUDA, "DiT init: stream events");
+    }
     const long long npe = (long long)t->Lv * t->D;
     LaunchScope ls(c, WDC_K_OTHER, 0);
     if (t->dtype == WDC_BF16)
@@ -498,6 +511,11 @@ wdc_status dit_create(Ctx* c) {
 void dit_destroy(Ctx* c) {
     if (!c->dit) return;
     for (void* p : c->dit->allocs) cudaFree(p);
+    for (int i = 0; i < 2; ++i) {
+        if (c->dit->fork[i]) cudaEventDestroy(c->dit->fork[i]);
+        if (c->dit->join[i]) cudaEventDestroy(c->dit->join[i]);
+    }
+    if (c->dit->aux) cudaStreamDestroy(c->dit->aux);
     delete c->dit;
     c->dit = nullptr;
 }
@@ -624,8 +642,26 @@ static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, cudaSt
     if (t->S == 2) { r0[0] = t->Lc; r1[0] = t->L; r0[1] = 0; r1[1] = t->Lc; }
     else { r0[0] = 0; r1[0] = t->L; }
     wdc_status st;
+    // per-stream CUDA streams: the condition rows (dual stream) on t->aux,
+    // forked before and joined after each half of the block; every buffer
+    // they touch (h, q/k/vt, ao, m, x) is split by rows
+    cudaStream_t ss[2] = {s, t->S == 2 ? t->aux : s};
+    auto fork = [&](int i) -> wdc_status {
+        if (t->S < 2) return WDC_OK;
+        WDC_CUDA_TRY(c, cudaEventRecord(t->fork[i], s));
+        WDC_CUDA_TRY(c, cudaStreamWaitEvent(t->aux, t->fork[i], 0));
+        return WDC_OK;
+    };
+    auto join = [&](int i) -> wdc_status {
+        if (t->S < 2) return WDC_OK;
+        WDC_CUDA_TRY(c, cudaEventRecord(t->join[i], t->aux));
+        WDC_CUDA_TRY(c, cudaStreamWaitEvent(s, t->join[i], 0));
+        return WDC_OK;
+    };
+    if ((st = fork(0))) return st;
     for (int sidx = 0; sidx < t->S; ++sidx) {
         const float* m6 = mod + (size_t)sidx * 6 * D;
+        cudaStream_t s = ss[sidx];
         ln_mod(c, x, t->h, r0[sidx], r1[sidx], m6 + 0 * D, m6 + 1 * D, 0, s);
         const Lin& w = t->qkv[layer * t->S + sidx];
         Epi e{};
@@ -633,9 +669,12 @@ static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, cudaSt
         e.L = t->L; e.H = t->H; e.d = t->d; e.D = D; e.row_off = r0[sidx];
         if ((st = gemm(c, (char*)t->h + (size_t)r0[sidx] * D * es, w.w, r1[sidx] - r0[sidx], 3 * D, D, e, s))) return st;
     }
+    if ((st = join(0))) return st;
     if ((st = attention(c, t->q, t->k, t->vt, t->ao, t->H, t->L, t->d, s))) return st;
+    if ((st = fork(1))) return st;
     for (int sidx = 0; sidx < t->S; ++sidx) {
         const float* m6 = mod + (size_t)sidx * 6 * D;
+        cudaStream_t s = ss[sidx];
         const int rows = r1[sidx] - r0[sidx];
         char* xr = (char*)x + (size_t)r0[sidx] * D * es;
         {
@@ -658,6 +697,7 @@ static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, cudaSt
             if ((st = gemm(c, (char*)t->m + (size_t)r0[sidx] * t->M * es, w.w, rows, D, t->M, e, s))) return st;
         }
     }
+    if ((st = join(1))) return st;
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("block: ") + cudaGetErrorString(e));
     return WDC_OK;
