@@ -234,6 +234,15 @@ unsigned long long wdc_launch_count(const wdc_ctx* ctx);
  * set in the context's error word: 1 = a bounded device-side wait timed out,
  * 4 = the two CTAs of a tensor-core pair saw different tensor-memory bases. */
 wdc_status wdc_device_errors(wdc_ctx* ctx, unsigned* bits);
+/* Self-test of the bounded device-side waits (the paper has no counterpart):
+ * one CTA waits on an mbarrier that nothing completes, through the same
+ * bounded wait the tensor-core kernels use, with a limit of `limit_ns`
+ * (1 us .. 1 s).  When the limit passes the wait gives up, sets bit 1 in the
+ * context's error word and raises the CTA's abort flag, which releases the
+ * CTA's other waiting thread; the kernel then returns normally.  Lets a test
+ * check the timeout path and that the context stays usable afterwards,
+ * without faulting or hanging the GPU.  Asynchronous on `stream`. */
+wdc_status wdc_selftest_wait_timeout(wdc_ctx* ctx, unsigned long long limit_ns, wdc_stream stream);
 
 /* ------------------------------------------------------------------ weights */
 /* Copies one parameter tensor (host fp32, `count` elements, shape as listed in

@@ -8,6 +8,7 @@
 // state (bank ring, anchor age); every continuous quantity of Eq. 2-10 lives
 // in device memory and is updated by the kernels' tails.
 #include "wdc_internal.h"
+#include "ptx.cuh"
 
 #include <cmath>
 #include <cstring>
@@ -67,6 +68,23 @@ __global__ void psi_kernel(const float* __restrict__ z, const float* __restrict_
     } else {
         for (long long i = base; i < n; ++i) out[i] = fmaf(dsig, v[i], z[i]);
     }
+}
+
+// Bounded-wait self-test: an mbarrier that nothing completes (see
+// wdc_selftest_wait_timeout).  Thread 0 gives up after limit_ns; thread 32
+// is released by the abort flag that thread 0 raises.
+__global__ void wait_probe_kernel(unsigned* err, unsigned long long limit_ns) {
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) mbar_wait(&bar, 0, &abort_flag, err, limit_ns);
+    if (threadIdx.x == 32) mbar_wait(&bar, 0, &abort_flag, err, 2 * limit_ns + 1000000ull);
+    __syncthreads();
 }
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -350,6 +368,18 @@ void wdc_destroy(wdc_ctx* h) {
     for (int k = 0; k < WDC_K_COUNT; ++k)
         for (cudaEvent_t e : c->ev[k]) cudaEventDestroy(e);
     delete c;
+}
+
+wdc_status wdc_selftest_wait_timeout(wdc_ctx* h, unsigned long long limit_ns, wdc_stream stream) {
+    Ctx* c = reinterpret_cast<Ctx*>(h);
+    if (!c) return WDC_ERR_INVALID_ARG;
+    if (limit_ns < 1000ull || limit_ns > 1000000000ull) return fail(c, WDC_ERR_INVALID_ARG, "limit_ns must be 1e3..1e9");
+    cudaSetDevice(c->device);
+    LaunchScope ls(c, WDC_K_OTHER, (cudaStream_t)stream);
+    wait_probe_kernel<<<1, 64, 0, (cudaStream_t)stream>>>(c->err, limit_ns);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("wait self-test: ") + cudaGetErrorString(e));
+    return WDC_OK;
 }
 
 wdc_status wdc_set_cache_params(wdc_ctx* h, const wdc_cache_params* params) {

@@ -119,6 +119,7 @@ def _load():
         "wdc_set_cache_params": (I, [P, ctypes.POINTER(CacheParams)]),
         "wdc_profile_enable": (I, [P, I]),
         "wdc_device_errors": (I, [P, ctypes.POINTER(ctypes.c_uint)]),
+        "wdc_selftest_wait_timeout": (I, [P, ctypes.c_ulonglong, P]),
         "wdc_profile_read": (I, [P, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_ulonglong)]),
         "wdc_last_error": (ctypes.c_char_p, [P]),
         "wdc_latent_numel": (S, [P]),
@@ -241,6 +242,10 @@ class Context:
         b = ctypes.c_uint()
         self._check(LIB.wdc_device_errors(self._h, ctypes.byref(b)), "device_errors")
         return b.value
+
+    def selftest_wait_timeout(self, limit_ns, stream=None):
+        """wdc_selftest_wait_timeout: a bounded device wait that must time out."""
+        self._check(LIB.wdc_selftest_wait_timeout(self._h, int(limit_ns), _stream(stream)), "selftest_wait_timeout")
 
     def profile_enable(self, on=True):
         self._check(LIB.wdc_profile_enable(self._h, int(on)), "profile_enable")

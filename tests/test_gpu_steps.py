@@ -176,3 +176,26 @@ def test_scheduler_step_is_one_fma():
     zn, vn = z.cpu().numpy().astype(np.float64), v.cpu().numpy().astype(np.float64)
     want = (zn + float(dsig) * vn)                          # fma: one rounding of the exact value
     assert np.array_equal(out.cpu().numpy(), want.astype(np.float32))
+
+
+def test_bounded_wait_times_out_and_context_stays_usable():
+    """A device wait on an mbarrier that nothing completes gives up after its
+    limit, reports the timeout bit, and the context keeps working (the wait
+    machinery every tensor-core kernel uses; no GPU fault involved)."""
+    import time
+    ctx = _ctx(1 << 16, wdc.make_params(), 50)
+    assert ctx.device_errors() == 0
+    t0 = time.perf_counter()
+    ctx.selftest_wait_timeout(2_000_000)            # 2 ms
+    bits = ctx.device_errors()                     # synchronises
+    assert bits == 1
+    assert time.perf_counter() - t0 < 5.0
+    assert ctx.device_errors() == 0                # cleared by the read
+    with pytest.raises(wdc.WdcError):
+        ctx.selftest_wait_timeout(10)              # limit out of range: rejected before launch
+    # the context still runs a full step afterwards
+    z = torch.randn(1 << 16, device="cuda")
+    ctx.state_reset(z)
+    zh = torch.empty_like(z)
+    info = ctx.surrogate_step(0, wdc.make_cond(), zh)
+    assert info.decision == 0 and ctx.device_errors() == 0
