@@ -486,7 +486,7 @@ def run_op(args):
     if args.op == "attention":
         q = torch.randn(H, L, d, device=dev).bfloat16()
         k = torch.randn(H, L, d, device=dev).bfloat16()
-        vt = torch.randn(H, d, L, device=dev).bfloat16()
+        vt = torch.randn(H, d, L, device=dev).half()           # V^T is fp16 in the bf16 model
         o = torch.empty(L, H * d, device=dev, dtype=torch.bfloat16)
         fn, work, unit = (lambda: ctx.op_attention(q, k, vt, o)), 4 * H * L * L * d, "TFLOP/s"
     elif args.op == "gemm":

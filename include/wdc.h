@@ -359,7 +359,10 @@ wdc_status wdc_op_gemm(wdc_ctx* ctx, const void* A, const void* W, const float* 
                        int M, int N, int K, int gelu, const void* res, const float* gate,
                        wdc_stream stream);
 /* O = softmax(Q K^T / sqrt(d)) V per head, non-causal: q, k [heads, L, d],
- * vt [heads, d, L] (V transposed), o [L, heads*d]; model dtype, device. */
+ * vt [heads, d, L] (V transposed), o [L, heads*d]; device memory.  q, k and
+ * o are in the model dtype; vt is fp32 for an fp32 model and fp16 for a bf16
+ * model (the QKV projection stores V that way so that the PV product takes
+ * the probabilities in fp16). */
 wdc_status wdc_op_attention(wdc_ctx* ctx, const void* q, const void* k, const void* vt, void* o,
                             int heads, int L, int d, wdc_stream stream);
 

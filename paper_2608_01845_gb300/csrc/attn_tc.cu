@@ -1,7 +1,8 @@
 // Non-causal softmax attention on the tcgen05 tensor cores (sm_103a):
 // O = softmax(Q K^T / sqrt(d)) V per head, joint over all L tokens (the DiT's
-// full spatio-temporal attention).  Q, K [H, L, d], V^T [H, d, L], O [L, H*d],
-// bf16 with fp32 softmax and accumulation; d = 64 or 128.
+// full spatio-temporal attention).  Q, K [H, L, d] bf16, V^T [H, d, L] fp16,
+// O [L, H*d] bf16; S = Q K^T in fp32, P in fp16, fp32 accumulation of O;
+// d = 64 or 128.
 //
 // One CTA per (head, 256 query rows), 12 warps in three warpgroups:
 //   warpgroup 0 (control, registers lowered to 40 / 72 per thread)
@@ -22,8 +23,14 @@
 // base and recompute (O and l share the base, so the result is unchanged).
 // The first tile sets the base from its own max.  S stays in registers until
 // that check, hence the register split.
-// P (bf16 pairs) is written to tensor memory and read as the TMEM A operand
-// of the PV MMA (shared memory is left to Q, K and V).  Two TMEM layouts:
+// P (fp16 pairs) is written to tensor memory and read as the TMEM A operand
+// of the PV MMA (shared memory is left to Q, K and V).  The numerators are
+// formed in packed fp16: x = s * scale - base in fp32 (fma.f32x2), one
+// conversion to f16x2 and one ex2.approx.f16x2 per pair, which is already
+// the P word; row sums accumulate per 16 pairs in f16x2 and in fp32 beyond.
+// In fp16, x keeps 11 significant bits (error <= 2^-9 absolute for
+// |x| < 8, below the rounding of P itself where P matters) and P keeps 11
+// (bf16 would keep 8).  Two TMEM layouts:
 //   d = 64   per tile t: S (128 columns), P (64), O (64) = 256 columns, so P
 //            has its own columns: S(t) may be overwritten as soon as the
 //            softmax has loaded it, and the MMA of S(t, j+1) overlaps the
@@ -38,6 +45,8 @@
 // mbarrier wait is bounded.
 #include "dit_kernels.cuh"
 #include "ptx.cuh"
+
+#include <cuda_fp16.h>
 
 namespace wdc {
 
@@ -106,30 +115,28 @@ __device__ __forceinline__ uint64_t pair(float a, float b) {
     return r;
 }
 
-// Two softmax numerators in paired-fp32 form: x = s * scale + nm for both
-// (one fma.f32x2), 2^x, their running row sums acc += (a, b) (one
-// add.f32x2) and the packed bf16 pair of P (lo = first key).
-__device__ __forceinline__ uint32_t exp2_pair(float s0, float s1, uint64_t scale2, uint64_t nm2, uint64_t& acc) {
+// Two softmax numerators: x pair (fma.f32x2) -> f16x2 -> ex2.approx.f16x2
+// (one SFU instruction for both) = the P word; the pair is added into an
+// f16x2 partial sum.
+__device__ __forceinline__ uint32_t exp2_pair_h(float s0, float s1, uint64_t scale2, uint64_t nm2, uint32_t& acc) {
     uint32_t p;
-    asm("{\n .reg .b64 x, e;\n .reg .f32 a, b;\n"
+    asm("{\n .reg .b64 x;\n .reg .f32 a, b;\n .reg .b32 h;\n"
         " mov.b64 x, {%2, %3};\n"
         " fma.rn.f32x2 x, x, %4, %5;\n"
         " mov.b64 {a, b}, x;\n"
-        " ex2.approx.ftz.f32 a, a;\n"
-        " ex2.approx.ftz.f32 b, b;\n"
-        " mov.b64 e, {a, b};\n"
-        " add.rn.f32x2 %1, %1, e;\n"
-        " cvt.rn.bf16x2.f32 %0, b, a;\n}"
-        : "=r"(p), "+l"(acc)
+        " cvt.rn.f16x2.f32 h, b, a;\n"
+        " ex2.approx.f16x2 %0, h;\n"
+        " add.rn.f16x2 %1, %1, %0;\n}"
+        : "=r"(p), "+r"(acc)
         : "f"(s0), "f"(s1), "l"(scale2), "l"(nm2));
     return p;
 }
 
-__device__ __forceinline__ float pair_sum(uint64_t v) {
-    float a, b;
-    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
-    return a + b;
+__device__ __forceinline__ float half2_sum(uint32_t v) {
+    __half2 h = *reinterpret_cast<__half2*>(&v);
+    return __low2float(h) + __high2float(h);
 }
+
 
 template <int D>
 __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
@@ -229,7 +236,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
       } else if (warp == 1 || (C::P_SEP && warp == 2)) {
         if (lane == 0) {
             constexpr uint32_t idesc_s = idesc_bf16(BQ, BKV);
-            constexpr uint32_t idesc_o = idesc_bf16(BQ, D);
+            constexpr uint32_t idesc_o = idesc_f16(BQ, D);       // P (fp16, TMEM) x V (fp16, shared memory)
             const uint32_t sq0 = smem_u32(sq);
             bool ok = mbar_wait(q_full, 0, abort_flag, g.err);
             int stage = 0, prev = 0;
@@ -365,14 +372,13 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
             // numerators 2^(s * scale - base) into p (bf16 pairs); returns their sum
             uint32_t p[BKV / 2];
             auto numerators = [&](float base) {
-                // paired-fp32 form (fma.f32x2, add.f32x2): 8 partial sums in 4 pairs
-                uint64_t sum4[4];
+                uint32_t sum4[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) sum4[i] = 0ull;
+                for (int i = 0; i < 4; ++i) sum4[i] = 0u;
                 const uint64_t nm2 = pair(-base, -base);
 #pragma unroll
-                for (int c = 0; c < BKV; c += 2) p[c / 2] = exp2_pair(s[c], s[c + 1], scale2, nm2, sum4[(c / 2) & 3]);
-                return (pair_sum(sum4[0]) + pair_sum(sum4[1])) + (pair_sum(sum4[2]) + pair_sum(sum4[3]));
+                for (int c = 0; c < BKV; c += 2) p[c / 2] = exp2_pair_h(s[c], s[c + 1], scale2, nm2, sum4[(c / 2) & 3]);
+                return (half2_sum(sum4[0]) + half2_sum(sum4[1])) + (half2_sum(sum4[2]) + half2_sum(sum4[3]));
             };
             float base = (j == 0) ? tile_max() * g.scale_log2 : m_run;
             float sum;
@@ -489,7 +495,7 @@ wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o,
     const uint64_t row = (uint64_t)D * 2, head = (uint64_t)L * D * 2;
     if (!encode_tmap_3d(&tq, q, D, L, H, row, head, 64, BQ, 1, &why) ||
         !encode_tmap_3d(&tk, k, D, L, H, row, head, 64, BKV, 1, &why) ||
-        !encode_tmap_3d(&tv, vt, L, D, H, (uint64_t)L * 2, (uint64_t)L * D * 2, 64, D, 1, &why))
+        !encode_tmap_3d(&tv, vt, L, D, H, (uint64_t)L * 2, (uint64_t)L * D * 2, 64, D, 1, &why, true))
         return fail(c, WDC_ERR_CUDA, why);
     AttnArgs g;
     g.H = H;

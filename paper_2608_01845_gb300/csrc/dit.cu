@@ -294,9 +294,9 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
 
 // ---------------------------------------------------------------- SIMT attention
 // One thread per query row, online softmax over key tiles staged in shared memory.
-template <typename T, int HD>
+template <typename T, typename TV, int HD>
 __global__ void __launch_bounds__(128) attn_simt_kernel(const T* __restrict__ q, const T* __restrict__ k,
-                                                         const T* __restrict__ vt, T* __restrict__ o, int H, int L,
+                                                         const TV* __restrict__ vt, T* __restrict__ o, int H, int L,
                                                          float scale) {
     constexpr int KT = HD <= 64 ? 64 : 32;
     __shared__ float Ks[KT][HD + 1];
@@ -315,7 +315,7 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const T* __restrict__ q,
             const int jj = i / HD, dd = i % HD;
             Ks[jj][dd] = (j0 + jj < L) ? ld_act<T>(k + ((size_t)h * L + j0 + jj) * HD + dd) : 0.f;
             const int dv = i / KT, jv = i % KT;
-            Vs[jv][dv] = (j0 + jv < L) ? ld_act<T>(vt + ((size_t)h * HD + dv) * L + j0 + jv) : 0.f;
+            Vs[jv][dv] = (j0 + jv < L) ? ld_act<TV>(vt + ((size_t)h * HD + dv) * L + j0 + jv) : 0.f;
         }
         __syncthreads();
         const int nk = min(KT, L - j0);
@@ -393,16 +393,17 @@ static wdc_status attention(Ctx* c, const void* q, const void* k, const void* vt
     const float scale = 1.0f / sqrtf((float)d);
     if (c->cfg.dtype == WDC_BF16) {
         using T = __nv_bfloat16;
+        using TV = __half;          // V^T is fp16 in the bf16 model (the PV product takes P in fp16)
         if (d == 64)
-            attn_simt_kernel<T, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+            attn_simt_kernel<T, TV, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const TV*)vt, (T*)o, H, L, scale);
         else
-            attn_simt_kernel<T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+            attn_simt_kernel<T, TV, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const TV*)vt, (T*)o, H, L, scale);
     } else {
         using T = float;
         if (d == 64)
-            attn_simt_kernel<T, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+            attn_simt_kernel<T, T, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
         else
-            attn_simt_kernel<T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+            attn_simt_kernel<T, T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
     }
     return WDC_OK;
 }

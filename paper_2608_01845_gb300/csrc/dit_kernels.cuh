@@ -5,11 +5,20 @@
 
 #include "wdc_internal.h"
 
+#include <cuda_fp16.h>
+
 namespace wdc {
 
 template <typename T> __device__ __forceinline__ float ld_act(const T* p);
 template <> __device__ __forceinline__ float ld_act<float>(const float* p) { return *p; }
 template <> __device__ __forceinline__ float ld_act<__nv_bfloat16>(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+template <> __device__ __forceinline__ float ld_act<__half>(const __half* p) { return __half2float(*p); }
+
+// V^T of the bf16 model is stored in fp16 (10-bit mantissa, range +-65504,
+// saturated) so that the attention's PV product can take P in fp16.
+__device__ __forceinline__ __half to_vt_half(float v) {
+    return __float2half_rn(fminf(fmaxf(v, -65504.0f), 65504.0f));
+}
 
 template <typename T> __device__ __forceinline__ T to_act(float v);
 template <> __device__ __forceinline__ float to_act<float>(float v) { return v; }
@@ -62,6 +71,8 @@ __device__ __forceinline__ void epi_apply(const Epi& e, int m, int n, float acc)
                 reinterpret_cast<T*>(e.q)[((size_t)h * e.L + tok) * e.d + dd] = to_act<T>(x);
             else if (which == 1)
                 reinterpret_cast<T*>(e.k)[((size_t)h * e.L + tok) * e.d + dd] = to_act<T>(x);
+            else if constexpr (sizeof(T) == 2)
+                reinterpret_cast<__half*>(e.vt)[((size_t)h * e.d + dd) * e.L + tok] = to_vt_half(x);
             else
                 reinterpret_cast<T*>(e.vt)[((size_t)h * e.d + dd) * e.L + tok] = to_act<T>(x);
             break;

@@ -136,9 +136,9 @@ __device__ __forceinline__ void epilogue_chunk(const Epi& e, int m, int col0, co
                 o4[q] = w;
             }
         } else {
-            __nv_bfloat16* base = reinterpret_cast<__nv_bfloat16*>(e.vt) + ((size_t)h * e.d + dd0) * e.L + tok;
+            __half* base = reinterpret_cast<__half*>(e.vt) + ((size_t)h * e.d + dd0) * e.L + tok;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) base[(size_t)j * e.L] = __float2bfloat16_rn(v[j]);
+            for (int j = 0; j < 32; ++j) base[(size_t)j * e.L] = to_vt_half(v[j]);
         }
         return;
     }
@@ -506,14 +506,15 @@ bool encode_tmap_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t
 }
 
 bool encode_tmap_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1_bytes,
-                    uint64_t s2_bytes, uint32_t b0, uint32_t b1, uint32_t b2, std::string* why) {
+                    uint64_t s2_bytes, uint32_t b0, uint32_t b1, uint32_t b2, std::string* why, bool f16) {
     auto fn = get_encode();
     if (!fn) { if (why) *why = "cuTensorMapEncodeTiled unavailable"; return false; }
     cuuint64_t dims[3] = {d0, d1, d2};
     cuuint64_t strides[2] = {s1_bytes, s2_bytes};
     cuuint32_t box[3] = {b0, b1, b2};
     cuuint32_t es[3] = {1, 1, 1};
-    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+    CUresult r = fn(map, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                    const_cast<void*>(base), dims, strides, box, es,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) { if (why) *why = "cuTensorMapEncodeTiled failed: " + std::to_string((int)r); return false; }

@@ -180,6 +180,13 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
            | ((uint32_t)(M >> 4) << 24);   // M / 16
 }
 
+// Instruction descriptor of kind::f16 with fp16 A and B, fp32 accumulation.
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N) {
+    return (1u << 4)                       // D format: f32 (A, B format 0: f16)
+           | ((uint32_t)(N >> 3) << 17)    // N / 8
+           | ((uint32_t)(M >> 4) << 24);   // M / 16
+}
+
 __device__ __forceinline__ void tmem_alloc(uint32_t* smem_result, uint32_t ncols) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(smem_result)),
                  "r"(ncols)
@@ -272,6 +279,7 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 bool encode_tmap_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
                     uint32_t box_inner, uint32_t box_outer, std::string* why);
 bool encode_tmap_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1_bytes,
-                    uint64_t s2_bytes, uint32_t b0, uint32_t b1, uint32_t b2, std::string* why);
+                    uint64_t s2_bytes, uint32_t b0, uint32_t b1, uint32_t b2, std::string* why,
+                    bool f16 = false);
 
 }  // namespace wdc

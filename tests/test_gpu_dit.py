@@ -62,6 +62,11 @@ def _bf(a):
     return synth.bf16_round(np.asarray(a, dtype=np.float32))
 
 
+def _h(a):
+    """fp16-rounded values (V^T of the bf16 model is stored in fp16)."""
+    return np.asarray(a, dtype=np.float32).astype(np.float16).astype(np.float32)
+
+
 @pytest.mark.parametrize("M,N,K", [(300, 384, 320), (128, 256, 64), (1000, 768, 1024), (17, 64, 128)])
 @pytest.mark.parametrize("mode", ["store", "gelu", "resid"])
 def test_bf16_gemm_matches_oracle(M, N, K, mode):
@@ -97,10 +102,10 @@ def test_bf16_attention_matches_oracle(H, L, d):
     ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
     q = _bf(synth.normal(11, (H, L, d)))
     k = _bf(synth.normal(12, (H, L, d)))
-    v = _bf(synth.normal(13, (H, L, d)))
+    v = _h(synth.normal(13, (H, L, d)))
     o = torch.empty(L, H * d, dtype=torch.bfloat16, device="cuda")
     ctx.op_attention(_to_dev(q, torch.bfloat16), _to_dev(k, torch.bfloat16),
-                     _to_dev(np.ascontiguousarray(v.transpose(0, 2, 1)), torch.bfloat16), o)
+                     _to_dev(np.ascontiguousarray(v.transpose(0, 2, 1)), torch.float16), o)
     torch.cuda.synchronize()
     qf = q.transpose(1, 0, 2).reshape(L, H * d).astype(np.float64)
     kf = k.transpose(1, 0, 2).reshape(L, H * d).astype(np.float64)
@@ -191,10 +196,10 @@ def test_bf16_attention_full_size_sampled_rows(H, L, d):
     g = np.random.default_rng(44)
     q = _bf(g.standard_normal((H, L, d), dtype=np.float32))
     k = _bf(g.standard_normal((H, L, d), dtype=np.float32))
-    v = _bf(g.standard_normal((H, L, d), dtype=np.float32))
+    v = _h(g.standard_normal((H, L, d), dtype=np.float32))
     o = torch.empty(L, H * d, dtype=torch.bfloat16, device="cuda")
     ctx.op_attention(_to_dev(q, torch.bfloat16), _to_dev(k, torch.bfloat16),
-                     _to_dev(np.ascontiguousarray(v.transpose(0, 2, 1)), torch.bfloat16), o)
+                     _to_dev(np.ascontiguousarray(v.transpose(0, 2, 1)), torch.float16), o)
     torch.cuda.synchronize()
     got = o.float().cpu().numpy()
     rows = np.sort(g.choice(L, 96, replace=False))
