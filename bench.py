@@ -499,6 +499,35 @@ def run_op(args):
         x = torch.randn(L, D, device=dev).bfloat16()
         mod = 0.1 * torch.randn((2 if w["dual_stream"] else 1) * 6, D, device=dev)
         fn, work, unit = (lambda: ctx.dit_block_forward(0, x, mod)), sum(block_flops(w)), "TFLOP/s"
+    elif args.op == "gemms":
+        # the block's four GEMMs with their epilogues, one line per shape
+        M = L
+        out = {}
+        for name, N, K, kw in [("qkv", 3 * D, D, {}), ("out", D, D, {"resid": True}),
+                               ("mlp_up", w["mlp"], D, {"gelu": True}), ("mlp_down", D, w["mlp"], {"resid": True})]:
+            A = torch.randn(M, K, device=dev).bfloat16()
+            Wt = (0.02 * torch.randn(N, K, device=dev)).bfloat16()
+            C = torch.randn(M, N, device=dev).bfloat16()
+            b = torch.zeros(N, device=dev)
+            gate = torch.ones(N, device=dev)
+            extra = {"gelu": True} if kw.get("gelu") else ({"res": C, "gate": gate} if kw.get("resid") else {})
+            f = lambda: ctx.op_gemm(A, Wt, C, bias=b, **extra)
+            for _ in range(3):
+                f()
+            torch.cuda.synchronize()
+            ts = []
+            for _ in range(args.reps):
+                a, e = ev(), ev()
+                a.record()
+                f()
+                e.record()
+                torch.cuda.synchronize()
+                ts.append(a.elapsed_time(e))
+            ms = statistics.median(ts)
+            out[f"{name} {M}x{N}x{K}"] = {"ms": ms, "TFLOP/s": 2 * M * N * K / (ms * 1e-3) / 1e12}
+            del A, Wt, C
+        print(json.dumps({"op": "gemms", "workload": args.workload, **out}))
+        return
     else:
         r = skip_pass_gbps(torch, wdc, peaks, secant=args.op == "secant")
         print(json.dumps({"op": args.op, **r}))
@@ -528,7 +557,7 @@ def main():
     ap.add_argument("--ablation", choices=sorted(ABLATIONS),
                     help="run the timed rollout under one ablation variant (Tables 3-4) and report its "
                          "final latent against the uncached rollout")
-    ap.add_argument("--op", choices=["attention", "gemm", "block", "skip", "secant"],
+    ap.add_argument("--op", choices=["attention", "gemm", "gemms", "block", "skip", "secant"],
                     help="time one operator at its 5B-scale shape (profiler captures)")
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="5b",
