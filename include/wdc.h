@@ -326,6 +326,19 @@ wdc_status wdc_risk_update(wdc_ctx* ctx, int k, const wdc_cond* c, const float* 
  * NULL.  Synchronises the stream once per step. */
 wdc_status wdc_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* conds, int n_cond,
                        float* z_out, int* decisions, wdc_step_info* trace, wdc_stream stream);
+/* The cached rollout of wdc_rollout with device-side control flow (the
+ * paper has no counterpart; it changes where the per-step bookkeeping runs,
+ * not what is computed): one CUDA graph with a WHILE node over the T steps,
+ * a SWITCH node on the bank size selecting the fused skip pass, and IF nodes
+ * on the decision, which the skip pass's last CTA sets on the device; so there
+ * is no host synchronisation between steps.  Same decisions and latents as
+ * wdc_rollout with one condition `cond` for every step.  z_T / z_out and the
+ * condition tokens may be host or device memory.  The graph is built on the
+ * first call (and again when the pass mode flags WDC_ABL_SECANT /
+ * WDC_OBS_RESIDUAL change); the event profiler must be off.  Afterwards the
+ * context's step-API state is that of the rollout's end. */
+wdc_status wdc_rollout_graph(wdc_ctx* ctx, const float* z_T, const wdc_cond* cond, float* z_out,
+                             int* decisions, wdc_step_info* trace, wdc_stream stream);
 /* The uncached rollout: wdc_dit_forward + wdc_scheduler_step at every step. */
 wdc_status wdc_native_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* conds, int n_cond,
                               float* z_out, wdc_stream stream);

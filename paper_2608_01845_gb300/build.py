@@ -15,7 +15,7 @@ ROOT = os.path.dirname(HERE)
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libwdc.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "step_kernels.cu", "dit.cu", "gemm_tc.cu", "attn_tc.cu"]
+SOURCES = ["api.cu", "step_kernels.cu", "dit.cu", "gemm_tc.cu", "attn_tc.cu", "graph_rollout.cu"]
 
 
 def nvcc():

@@ -22,6 +22,22 @@ wdc_status fail(Ctx* c, wdc_status s, const std::string& msg) {
     return s;
 }
 
+void fill_info(const StepOut& o, int k, int n_bank, int age, wdc_step_info* info) {
+    if (!info) return;
+    info->k = k;
+    info->decision = o.decision;
+    info->finite = o.finite;
+    info->supported = o.supported;
+    info->n_compat = o.n_compat;
+    info->n_bank = n_bank;
+    info->age = age;
+    info->q = o.q; info->alpha = o.alpha; info->p = o.p; info->d_hat = o.d_hat; info->w = o.w;
+    info->delta = o.delta; info->R_cand = o.R_cand; info->R = o.R; info->eta = o.eta;
+    info->d_cf = o.d_cf; info->d_z = o.d_z; info->r = o.r;
+    for (int i = 0; i < WDC_MAX_BANK; ++i) { info->kappa[i] = o.kappa[i]; info->pi[i] = o.pi[i]; }
+}
+
+
 static cudaEvent_t next_event(Ctx* c, int cls) {
     auto& v = c->ev[cls];
     if (c->ev_used[cls] == v.size()) {
@@ -131,20 +147,6 @@ wdc_status check_params(Ctx* c, const wdc_cache_params& p) {
     return WDC_OK;
 }
 
-void fill_info(const StepOut& o, int k, int n_bank, int age, wdc_step_info* info) {
-    if (!info) return;
-    info->k = k;
-    info->decision = o.decision;
-    info->finite = o.finite;
-    info->supported = o.supported;
-    info->n_compat = o.n_compat;
-    info->n_bank = n_bank;
-    info->age = age;
-    info->q = o.q; info->alpha = o.alpha; info->p = o.p; info->d_hat = o.d_hat; info->w = o.w;
-    info->delta = o.delta; info->R_cand = o.R_cand; info->R = o.R; info->eta = o.eta;
-    info->d_cf = o.d_cf; info->d_z = o.d_z; info->r = o.r;
-    for (int i = 0; i < WDC_MAX_BANK; ++i) { info->kappa[i] = o.kappa[i]; info->pi[i] = o.pi[i]; }
-}
 
 int slot_of(const Ctx* c, int age_idx) { return (c->head + age_idx) % c->prm.bank_capacity; }
 int newest_slot(const Ctx* c) { return slot_of(c, c->n_bank - 1); }
@@ -351,6 +353,7 @@ wdc_status wdc_create(const wdc_dit_config* cfg, const wdc_schedule* sched, cons
 void wdc_destroy(wdc_ctx* h) {
     Ctx* c = reinterpret_cast<Ctx*>(h);
     if (!c) return;
+    graph_rollout_destroy(c);
     cudaSetDevice(c->device);
     dit_destroy(c);
     cudaFree(c->st);
@@ -763,6 +766,21 @@ wdc_status wdc_rollout(wdc_ctx* h, const float* z_T, const wdc_cond* conds, int 
     if (!c) return WDC_ERR_INVALID_ARG;
     cudaSetDevice(c->device);
     return rollout_impl(c, z_T, conds, n_cond, z_out, decisions, trace, (cudaStream_t)stream, true);
+}
+
+wdc_status wdc_rollout_graph(wdc_ctx* h, const float* z_T, const wdc_cond* cond, float* z_out, int* decisions,
+                             wdc_step_info* trace, wdc_stream stream) {
+    Ctx* c = reinterpret_cast<Ctx*>(h);
+    if (!c) return WDC_ERR_INVALID_ARG;
+    if (!z_T || !z_out || !cond) return fail(c, WDC_ERR_INVALID_ARG, "null pointer");
+    if (!c->dit) return fail(c, WDC_ERR_UNSUPPORTED, "rollout needs a denoiser (layers > 0)");
+    const size_t cond_elems = (size_t)c->cfg.cond_tokens * c->cfg.cond_dim;
+    if (cond_elems && !cond->tokens) return fail(c, WDC_ERR_INVALID_ARG, "condition tokens required");
+    cudaSetDevice(c->device);
+    const bool in_dev = is_device_ptr(z_T), out_dev = is_device_ptr(z_out);
+    const bool tok_dev = cond_elems && is_device_ptr(cond->tokens);
+    return graph_rollout(c, z_T, in_dev, cond, tok_dev ? cond->tokens : nullptr, z_out, out_dev, decisions, trace,
+                         (cudaStream_t)stream);
 }
 
 wdc_status wdc_native_rollout(wdc_ctx* h, const float* z_T, const wdc_cond* conds, int n_cond, float* z_out,

@@ -55,14 +55,19 @@ struct DiT {
     // GEMMs fill the SMs the video GEMMs leave idle in their last wave
     cudaStream_t aux = nullptr;
     cudaEvent_t fork[2] = {}, join[2] = {};
+    // set while a graph rollout captures the forward: the timestep comes from
+    // device memory at replay time
+    const float* t_src = nullptr;
 };
 
 namespace {
 
 // ---------------------------------------------------------------- small kernels
-__global__ void features_kernel(float t, int half, float* out) {
+// t_src (device, or null): the timestep is read there instead (graph rollout).
+__global__ void features_kernel(float t, const float* t_src, int half, float* out) {
     const int j = threadIdx.x + blockIdx.x * blockDim.x;
     if (j >= half) return;
+    if (t_src) t = *t_src;
     const double w = exp(-log(10000.0) * (double)j / (double)half);
     const double a = (double)t * w;
     out[j] = (float)cos(a);
@@ -615,7 +620,7 @@ wdc_status dit_modulation(Ctx* c, float t_model, float* mod_out, cudaStream_t s)
     const int half = t->Fd / 2;
     {
         LaunchScope ls(c, WDC_K_OTHER, s);
-        features_kernel<<<blocks_for(half, 128), 128, 0, s>>>(t_model, half, t->feat);
+        features_kernel<<<blocks_for(half, 128), 128, 0, s>>>(t_model, t->t_src, half, t->feat);
     }
     auto gv = [&](const void* W, const float* x, const float* b, float* y, int rows, int cols, int act) {
         const unsigned grid = blocks_for((long long)rows * 32, 256);
@@ -702,6 +707,10 @@ static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, cudaSt
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("block: ") + cudaGetErrorString(e));
     return WDC_OK;
+}
+
+void dit_set_timestep_source(Ctx* c, const float* t_src) {
+    if (c->dit) c->dit->t_src = t_src;
 }
 
 wdc_status dit_block(Ctx* c, int layer, void* x, const float* mod6, cudaStream_t s) {

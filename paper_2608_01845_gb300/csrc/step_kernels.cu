@@ -296,7 +296,7 @@ struct PassShared {
 };
 
 template <int MODE, int K>
-__global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant__ PassArgs a) {
+__device__ __forceinline__ void pass_body(const PassArgs& a) {
     __shared__ HeadShared hs;
     __shared__ PassShared ps;
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
@@ -406,6 +406,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                     ze.x = fmaf(dsig, v.x, z.x); ze.y = fmaf(dsig, v.y, z.y);
                     ze.z = fmaf(dsig, v.z, z.z); ze.w = fmaf(dsig, v.w, z.w);
                     *reinterpret_cast<float4*>(a.out + base) = ze;
+                    if (a.out3) *reinterpret_cast<float4*>(a.out3 + base) = ze;
                     if (a.out2) {
                         float4 dz;
                         dz.x = ze.x - z.x; dz.y = ze.y - z.y; dz.z = ze.z - z.z; dz.w = ze.w - z.w;
@@ -464,6 +465,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                         const float za = a.anchor[idx];
                         const float ze = fmaf(dsig, a.v[idx], z);
                         a.out[idx] = ze;
+                        if (a.out3) a.out3[idx] = ze;
                         if (a.out2) a.out2[idx] = ze - z;
                         o[e] = ze;
                         sa[e] = za;
@@ -648,6 +650,11 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
                 o.pi[i] = (i < K) ? hs.pi[i] : 0.0;
             }
             if (dec) st->R = R_cand;
+            if (a.graph) {
+                // device-side control flow: exactly one of the two branches runs
+                cudaGraphSetConditional((cudaGraphConditionalHandle)a.h_exact, dec ? 0u : 1u);
+                cudaGraphSetConditional((cudaGraphConditionalHandle)a.h_accept, dec ? 1u : 0u);
+            }
             o.R = st->R;
             o.eta = st->eta;
             st->cand_k = a.k;
@@ -746,6 +753,17 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
     }
 }
 
+// Launch forms: arguments by value (the host-driven calls) or read from
+// device memory (graph rollout: a planning kernel writes them each step).
+template <int MODE, int K>
+__global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant__ PassArgs a) {
+    pass_body<MODE, K>(a);
+}
+template <int MODE, int K>
+__global__ void __launch_bounds__(kThreads, 1) pass_kernel_p(const PassArgs* __restrict__ pa) {
+    pass_body<MODE, K>(*pa);
+}
+
 template <int K>
 void launch_skip(const PassArgs& a, int grid, cudaStream_t s, bool residual) {
     if (residual) pass_kernel<kModeResidual, K><<<grid, kThreads, 0, s>>>(a);
@@ -760,6 +778,36 @@ int pass_grid(const Ctx* c) {
     if (g > c->num_sms) g = c->num_sms;
     if (g < 1) g = 1;
     return (int)g;
+}
+
+// Pointer-argument launch (graph capture); K selects the bank-size
+// specialisation of the skip / residual passes.
+wdc_status launch_pass_ptr(Ctx* c, int mode, int K, const PassArgs* pa, cudaStream_t s) {
+    const int grid = pass_grid(c);
+    switch (mode) {
+        case kModeAnchor: pass_kernel_p<kModeAnchor, 0><<<grid, kThreads, 0, s>>>(pa); break;
+        case kModeSecant: pass_kernel_p<kModeSecant, 0><<<grid, kThreads, 0, s>>>(pa); break;
+        case kModeSkip:
+        case kModeResidual: {
+            const bool r = mode == kModeResidual;
+#define WDC_SKIP_P(KK)                                                                       \
+    case KK:                                                                                 \
+        if (r) pass_kernel_p<kModeResidual, KK><<<grid, kThreads, 0, s>>>(pa);              \
+        else pass_kernel_p<kModeSkip, KK><<<grid, kThreads, 0, s>>>(pa);                    \
+        break;
+            switch (K) {
+                WDC_SKIP_P(0) WDC_SKIP_P(1) WDC_SKIP_P(2) WDC_SKIP_P(3) WDC_SKIP_P(4)
+                WDC_SKIP_P(5) WDC_SKIP_P(6) WDC_SKIP_P(7) WDC_SKIP_P(8)
+                default: return fail(c, WDC_ERR_INVALID_ARG, "bank size out of range");
+            }
+#undef WDC_SKIP_P
+            break;
+        }
+        default: return fail(c, WDC_ERR_INVALID_ARG, "unsupported pass mode for the graph rollout");
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("latent pass launch: ") + cudaGetErrorString(e));
+    return WDC_OK;
 }
 
 wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s) {

@@ -55,6 +55,10 @@ struct DevState {
     double cand_p;
     double cand_S[kSketch], cand_sumsq, cand_sumsq_anchor;
     StepOut out;
+    // discrete state of the graph rollout (device-resident mirror of the
+    // host's ring head, bank size and age)
+    int g_k, g_n_bank, g_head, g_age;
+    float g_t_model;                   // 1000 * sigma_k for the denoiser's timestep path
 };
 
 struct ParamsDev {
@@ -94,9 +98,15 @@ struct PassArgs {
     unsigned* err;
     float kappa[kMaxBank];             // observe: caller-given weights
     double* stats_out;                 // observe: caller-given statistics output
+    // graph rollout (device-side control flow)
+    int graph;                         // skip tail sets the branch conditions below
+    unsigned long long h_exact, h_accept;   // cudaGraphConditionalHandle values
+    float* out3;                       // anchor: z_exact also into the graph's current latent
 };
 
 // ---------------------------------------------------------------- context
+struct GraphRollout;
+
 struct Ctx {
     wdc_dit_config cfg{};
     wdc_schedule sched{};
@@ -130,6 +140,9 @@ struct Ctx {
     // denoiser
     struct DiT* dit = nullptr;
 
+    // graph rollout (device-side control flow), built on first use
+    GraphRollout* grollout = nullptr;
+
     // optional per-class event timing (wdc_profile_enable)
     bool prof = false;
     std::vector<cudaEvent_t> ev[WDC_K_COUNT];      // begin/end pairs
@@ -158,11 +171,18 @@ struct LaunchScope {
     } while (0)
 
 wdc_status fail(Ctx* c, wdc_status s, const std::string& msg);
+void fill_info(const StepOut& o, int k, int n_bank, int age, wdc_step_info* info);
+
+// graph_rollout.cu
+wdc_status graph_rollout(Ctx* c, const float* z_T, bool z_dev, const wdc_cond* cd, const float* tokens_dev,
+                         float* z_out, bool out_dev, int* decisions, wdc_step_info* trace, cudaStream_t s);
+void graph_rollout_destroy(Ctx* c);
 
 // step_kernels.cu
 constexpr int kPartials = 2 * kSketch + 8;     // per-block partial sums
 int pass_grid(const Ctx* c);
 wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s);
+wdc_status launch_pass_ptr(Ctx* c, int mode, int K, const PassArgs* pa, cudaStream_t s);
 ParamsDev to_dev_params(const wdc_cache_params& p);
 
 // dit.cu
@@ -171,6 +191,7 @@ void dit_destroy(Ctx* c);
 wdc_status dit_set_tensor(Ctx* c, int id, int layer, int stream, const float* host, size_t count);
 wdc_status dit_init_weights(Ctx* c, unsigned long long seed, float std);
 wdc_status dit_forward(Ctx* c, const float* z, float t, const float* cond, float* v, cudaStream_t s);
+void dit_set_timestep_source(Ctx* c, const float* t_src);   // null: the t argument of dit_forward
 wdc_status dit_block(Ctx* c, int layer, void* x, const float* mod6, cudaStream_t s);
 wdc_status dit_modulation(Ctx* c, float t, float* mod_out, cudaStream_t s);
 wdc_status op_gemm(Ctx* c, const void* A, const void* W, const float* bias, void* C, int M, int N, int K,

@@ -136,6 +136,7 @@ def _load():
         "wdc_surrogate_step": (I, [P, I, ctypes.POINTER(Cond), P, ctypes.POINTER(StepInfo), P]),
         "wdc_risk_update": (I, [P, I, ctypes.POINTER(Cond), P, P, P, ctypes.POINTER(P), ctypes.POINTER(StepInfo), P]),
         "wdc_rollout": (I, [P, P, ctypes.POINTER(Cond), I, P, ctypes.POINTER(I), ctypes.POINTER(StepInfo), P]),
+        "wdc_rollout_graph": (I, [P, P, ctypes.POINTER(Cond), P, ctypes.POINTER(I), ctypes.POINTER(StepInfo), P]),
         "wdc_native_rollout": (I, [P, P, ctypes.POINTER(Cond), I, P, P]),
         "wdc_op_gemm": (I, [P, P, P, P, P, I, I, I, I, P, P, P]),
         "wdc_op_attention": (I, [P, P, P, P, P, I, I, I, P]),
@@ -325,6 +326,15 @@ class Context:
         tr = (StepInfo * T)() if trace else None
         self._check(LIB.wdc_rollout(self._h, _ptr(z_T), carr, len(conds), _ptr(z_out), dec, tr, _stream(stream)),
                     "rollout")
+        return list(dec), ([tr[k].as_dict() for k in range(T)] if trace else None)
+
+    def rollout_graph(self, z_T, cond, z_out, trace=True, stream=None):
+        """wdc_rollout_graph: the cached rollout with device-side control flow (one condition)."""
+        T = self.sched.T
+        dec = (ctypes.c_int * T)()
+        tr = (StepInfo * T)() if trace else None
+        self._check(LIB.wdc_rollout_graph(self._h, _ptr(z_T), ctypes.byref(cond), _ptr(z_out), dec, tr,
+                                          _stream(stream)), "rollout_graph")
         return list(dec), ([tr[k].as_dict() for k in range(T)] if trace else None)
 
     def native_rollout(self, z_T, conds, z_out, stream=None):

@@ -99,3 +99,63 @@ def test_age_convention_budget_on_gpu():
     dec, _ = ctx.rollout(torch.from_numpy(z0.ravel().copy()).cuda(), c, out)
     assert [k for k, d in enumerate(dec) if d == 0] == gold["exact_steps"]
     assert torch.isfinite(out).all()
+
+
+@pytest.mark.parametrize("flags", [0, wdc.ABL_SECANT, wdc.OBS_RESIDUAL])
+def test_graph_rollout_equals_host_rollout(flags):
+    """wdc_rollout_graph (device-side control flow: WHILE / SWITCH / IF graph
+    nodes, decisions set on the device) against the host-driven rollout of
+    the same context: identical decisions and trace, bitwise-identical latent;
+    a second call reuses the graph."""
+    T = 10
+    op, cp, W, ctx, z0, ct, desc = _setup(T, tau_risk=0.5, flags=flags)
+    c = wdc.make_cond(torch.from_numpy(ct).cuda(), desc["cam"], desc["depth"])
+    zT = torch.from_numpy(z0.ravel().copy()).cuda()
+    out_h = torch.empty(z0.size, dtype=torch.float32, device="cuda")
+    dec_h, tr_h = ctx.rollout(zT, c, out_h)
+    assert 0 < sum(dec_h) < T
+    for rep in range(2):
+        out_g = torch.empty_like(out_h)
+        dec_g, tr_g = ctx.rollout_graph(zT, c, out_g)
+        assert dec_g == dec_h
+        assert torch.equal(out_g, out_h)
+        for a, b in zip(tr_g, tr_h):
+            for key in ["decision", "n_bank", "age", "p", "d_hat", "w", "R_cand", "R", "eta", "alpha"]:
+                assert a[key] == b[key], (rep, a["k"], key)
+    assert ctx.device_errors() == 0
+
+
+def test_graph_rollout_all_exact_is_native_and_host_buffers():
+    T = 6
+    op, cp, W, ctx, z0, ct, desc = _setup(T, tau_risk=-1.0)
+    c = wdc.make_cond(torch.from_numpy(ct).cuda(), desc["cam"], desc["depth"])
+    zT = torch.from_numpy(z0.ravel().copy()).cuda()
+    nat = torch.empty_like(zT)
+    ctx.native_rollout(zT, c, nat)
+    zh = torch.from_numpy(z0.ravel().copy()).pin_memory()
+    outh = torch.empty_like(zh).pin_memory()
+    ch = wdc.make_cond(torch.from_numpy(ct).pin_memory(), desc["cam"], desc["depth"])
+    dec, _ = ctx.rollout_graph(zh, ch, outh)
+    assert dec == [0] * T
+    assert torch.equal(outh, nat.cpu())
+
+
+def test_graph_rollout_dual_stream_bf16_equals_host():
+    """bf16 dual-stream model: the captured forward forks the condition rows
+    onto a second stream; graph and host rollouts agree bitwise."""
+    T = 8
+    cfg = dict(CFG0, dual_stream=1)
+    W = synth.dit_weights(cfg, 0, std=0.02)
+    _, cp = params_for_both(tau_risk=0.5)
+    ctx = wdc.Context(wdc.make_config(dtype=wdc.BF16, **cfg), T, params=cp)
+    ctx.set_weights(W)
+    z0 = synth.latent(1, (16, 4, 16, 16))
+    ct = synth.cond_tokens(2, 16, 256)
+    desc = synth.cond_descriptors(3)
+    c = wdc.make_cond(torch.from_numpy(ct).cuda(), desc["cam"], desc["depth"])
+    zT = torch.from_numpy(z0.ravel().copy()).cuda()
+    out_h = torch.empty_like(zT)
+    dec_h, _ = ctx.rollout(zT, c, out_h)
+    out_g = torch.empty_like(zT)
+    dec_g, _ = ctx.rollout_graph(zT, c, out_g)
+    assert dec_g == dec_h and torch.equal(out_g, out_h)
