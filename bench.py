@@ -444,6 +444,17 @@ def run_gpu(args, rank, world, local_rank):
     line["e2e"] = {"value": world * T * args.steps / et, "unit": UNIT,
                    "h2d_bytes_per_step": zT.nbytes + ct.nbytes, "d2h_bytes_per_step": zT.nbytes}
 
+    # device-side control flow on the same workload (graph built by a first call)
+    if rank == 0 and not args.ablation:
+        ctx.rollout_graph(zT_d, cond, out, trace=False)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        dec_g, _ = ctx.rollout_graph(zT_d, cond, out, trace=False)
+        torch.cuda.synchronize()
+        gt = time.perf_counter() - t0
+        line["graph_rollout"] = {"steps_per_s": T / gt, "exact_steps": T - sum(dec_g),
+                                 "note": "wdc_rollout_graph: no host synchronisation between steps"}
+
     if args.ablation and rank == 0:
         # mechanics of the variant on the random-init model: final latent
         # against the uncached rollout of the same inputs
@@ -499,6 +510,39 @@ def run_op(args):
         x = torch.randn(L, D, device=dev).bfloat16()
         mod = 0.1 * torch.randn((2 if w["dual_stream"] else 1) * 6, D, device=dev)
         fn, work, unit = (lambda: ctx.dit_block_forward(0, x, mod)), sum(block_flops(w)), "TFLOP/s"
+    elif args.op == "control":
+        # host-driven vs device-side control flow (wdc_rollout vs
+        # wdc_rollout_graph) on the 2-layer D=256 parity model, T = 50,
+        # where the per-step host synchronisation is visible
+        from paper_2608_01845_gb300 import synth
+        small = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16,
+                     frames=4, height=16, width=16, patch=2, cond_tokens=16, cond_dim=256, dual_stream=0)
+        T = 50
+        res = {}
+        for dt, name in [(wdc.F32, "fp32"), (wdc.BF16, "bf16")]:
+            cx = wdc.Context(wdc.make_config(dtype=dt, **small), T, params=wdc.make_params(tau_risk=0.5))
+            cx.init_weights(3, 0.02)
+            zT = torch.from_numpy(synth.latent(1, (16 * 4 * 16 * 16,))).cuda()
+            cd = wdc.make_cond(torch.from_numpy(synth.cond_tokens(2, 16, 256)).cuda(), [0.1] * 4, [0.05] * 4)
+            out = torch.empty_like(zT)
+            row = {}
+            for mode, fn in [("host", lambda: cx.rollout(zT, cd, out, trace=False)),
+                             ("graph", lambda: cx.rollout_graph(zT, cd, out, trace=False))]:
+                for _ in range(3):
+                    dec, _ = fn()
+                torch.cuda.synchronize()
+                ts = []
+                for _ in range(max(args.reps, 5)):
+                    t0 = time.perf_counter()
+                    fn()
+                    torch.cuda.synchronize()
+                    ts.append(time.perf_counter() - t0)
+                ms = 1e3 * statistics.median(ts)
+                row[mode] = {"ms_per_rollout": ms, "steps_per_s": T / (ms * 1e-3), "exact_steps": T - sum(dec)}
+            res[name] = row
+            cx.close()
+        print(json.dumps({"op": "control", "model": "2-layer D=256 (parity model shape), T=50", **res}))
+        return
     elif args.op == "gemms":
         # the block's four GEMMs with their epilogues, one line per shape
         M = L
@@ -557,7 +601,7 @@ def main():
     ap.add_argument("--ablation", choices=sorted(ABLATIONS),
                     help="run the timed rollout under one ablation variant (Tables 3-4) and report its "
                          "final latent against the uncached rollout")
-    ap.add_argument("--op", choices=["attention", "gemm", "gemms", "block", "skip", "secant"],
+    ap.add_argument("--op", choices=["attention", "gemm", "gemms", "block", "skip", "secant", "control"],
                     help="time one operator at its 5B-scale shape (profiler captures)")
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="5b",

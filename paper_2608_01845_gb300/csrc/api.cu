@@ -342,6 +342,7 @@ wdc_status wdc_create(const wdc_dit_config* cfg, const wdc_schedule* sched, cons
     if (!dm((void**)&c->cand[0], lat) || !dm((void**)&c->cand[1], lat)) return bail(WDC_ERR_OOM);
     if (!dm((void**)&c->vbuf, lat)) return bail(WDC_ERR_OOM);
     if (cudaMallocHost((void**)&c->out_host, sizeof(StepOut) * (sched->T + 2)) != cudaSuccess) return bail(WDC_ERR_OOM);
+    if (cudaMallocHost((void**)&c->st_host, sizeof(DevState)) != cudaSuccess) return bail(WDC_ERR_OOM);
     if ((st = ensure_disp(c))) return bail(st);
     if (cfg->layers > 0) {
         if ((st = dit_create(c))) return bail(st);
@@ -368,6 +369,7 @@ void wdc_destroy(wdc_ctx* h) {
     cudaFree(c->zstage);
     for (int i = 0; i < kMaxBank; ++i) cudaFree(c->disp[i]);
     if (c->out_host) cudaFreeHost(c->out_host);
+    if (c->st_host) cudaFreeHost(c->st_host);
     for (int k = 0; k < WDC_K_COUNT; ++k)
         for (cudaEvent_t e : c->ev[k]) cudaEventDestroy(e);
     delete c;
@@ -522,8 +524,7 @@ wdc_status wdc_state_reset(wdc_ctx* h, const float* z_T, wdc_stream stream) {
     c->cur_latent = c->z_init;
     wdc_status cs = clear_disp(c, s);
     if (cs) return cs;
-    DevState* hs = nullptr;
-    WDC_CUDA_TRY(c, cudaMallocHost((void**)&hs, sizeof(DevState)));
+    DevState* hs = c->st_host;           // pinned staging owned by the context
     std::memset(hs, 0, sizeof(DevState));
     hs->R = 0.0;
     hs->eta = c->prm.eta_init;
@@ -531,7 +532,6 @@ wdc_status wdc_state_reset(wdc_ctx* h, const float* z_T, wdc_stream stream) {
     hs->cand_k = -1;
     cudaError_t e = cudaMemcpyAsync(c->st, hs, sizeof(DevState), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-    cudaFreeHost(hs);
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("state_reset: ") + cudaGetErrorString(e));
     return stats_pass(c, c->z_init, s);
 }
@@ -540,12 +540,10 @@ wdc_status wdc_state_get(wdc_ctx* h, wdc_state_host* out, wdc_stream stream) {
     Ctx* c = reinterpret_cast<Ctx*>(h);
     if (!c || !out) return WDC_ERR_INVALID_ARG;
     cudaSetDevice(c->device);
-    DevState* hs = nullptr;
-    WDC_CUDA_TRY(c, cudaMallocHost((void**)&hs, sizeof(DevState)));
+    DevState* hs = c->st_host;           // pinned staging owned by the context
     cudaError_t e = cudaMemcpyAsync(hs, c->st, sizeof(DevState), cudaMemcpyDeviceToHost, (cudaStream_t)stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) {
-        cudaFreeHost(hs);
         return fail(c, WDC_ERR_CUDA, std::string("state_get: ") + cudaGetErrorString(e));
     }
     std::memset(out, 0, sizeof(*out));
@@ -574,7 +572,6 @@ wdc_status wdc_state_get(wdc_ctx* h, wdc_state_host* out, wdc_stream stream) {
     out->cand_supported = hs->cand_supported;
     out->cand_finite = hs->cand_finite;
     out->cand_p = hs->cand_p;
-    cudaFreeHost(hs);
     return WDC_OK;
 }
 
@@ -590,8 +587,7 @@ wdc_status wdc_state_set(wdc_ctx* h, const wdc_state_host* in, const float* cons
         if (!z_out[i] || !aligned16(z_out[i])) return fail(c, WDC_ERR_INVALID_ARG, "bank latents must be 16-byte aligned device pointers");
     cudaSetDevice(c->device);
     cudaStream_t s = (cudaStream_t)stream;
-    DevState* hs = nullptr;
-    WDC_CUDA_TRY(c, cudaMallocHost((void**)&hs, sizeof(DevState)));
+    DevState* hs = c->st_host;           // pinned staging owned by the context
     std::memset(hs, 0, sizeof(DevState));
     hs->R = in->R;
     hs->eta = in->eta;
@@ -614,7 +610,6 @@ wdc_status wdc_state_set(wdc_ctx* h, const wdc_state_host* in, const float* cons
     }
     cudaError_t e = cudaMemcpyAsync(c->st, hs, sizeof(DevState), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-    cudaFreeHost(hs);
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("state_set: ") + cudaGetErrorString(e));
     c->head = 0;
     c->n_bank = in->n_bank;

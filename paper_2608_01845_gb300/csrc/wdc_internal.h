@@ -124,6 +124,7 @@ struct Ctx {
     unsigned* counter = nullptr;
     unsigned* err = nullptr;
     StepOut* out_host = nullptr;       // pinned
+    DevState* st_host = nullptr;       // pinned staging of the device state (reset / get / set)
     float* bank[kMaxBank] = {};
     float* z_init = nullptr;           // anchor before the first exact step
     float* cand[2] = {};               // rollout candidate buffers
