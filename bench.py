@@ -384,6 +384,7 @@ def run_gpu(args, rank, world, local_rank):
     barrier()
     clk = clocks.stop()
     prof = ctx.profile_read()
+    ctx.profile_enable(False)
     launches = ctx.launches - launches0
     ms = e0.elapsed_time(e1)
     if world > 1:
