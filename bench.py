@@ -13,7 +13,7 @@ metric: denoising steps per second of the whole job (N replicas, one rollout
 each per step: weak scaling).  Extra fields: the dominant kernel's roofline
 (live CUDA-event durations inside the timed region), the DiT-block TFLOP/s,
 the fused skip-pass GB/s at 2^28 fp32 elements (L2 flushed), the end-to-end
-number through the C ABI with host buffers, the CPU checker's baseline and the
+number through the C ABI with host buffers, the CPU oracle's baseline and the
 clocks seen during the timed region.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
@@ -154,11 +154,11 @@ class ClockSampler:
                 "samples": len(rows)}
 
 
-# ------------------------------------------------------------------ CPU checker timing
+# ------------------------------------------------------------------ CPU oracle timing
 def cpu_sample(w, exact_steps, rows=16):
-    """Times the CPU checker on a bounded sample of the workload and scales it
+    """Times the CPU oracle on a bounded sample of the workload and scales it
     to steps/s: one DiT block evaluated for `rows` sampled query rows (keys and
-    values for all 17776 tokens) gives the checker's flop rate, which prices an
+    values for all 17776 tokens) gives the oracle's flop rate, which prices an
     exact forward; one surrogate step and one anchor step at the full latent
     size price the rest.  Returns (steps/s estimate, description, seconds)."""
     import numpy as np
@@ -205,7 +205,7 @@ def cpu_sample(w, exact_steps, rows=16):
     ro.exact_step(st, z1, v, zh, 4, {}, sig, p, info)
     t_anchor = time.perf_counter() - t0
     per_rollout = exact_steps * (t_exact_fwd + t_skip + t_anchor) + (T - exact_steps) * t_skip
-    desc = (f"CPU checker (fp64 numpy, {os.cpu_count()} BLAS threads): one DiT block for {rows} sampled query rows "
+    desc = (f"CPU oracle (fp64 numpy, {os.cpu_count()} BLAS threads): one DiT block for {rows} sampled query rows "
             f"({t_blk:.1f} s, {rate / 1e9:.1f} GFLOP/s) priced {exact_steps} exact forwards; one surrogate step "
             f"({t_skip:.2f} s) and one anchor step ({t_anchor:.2f} s) at {n} latent elements priced the rest; "
             f"scaled to a {T}-step rollout")
@@ -213,7 +213,7 @@ def cpu_sample(w, exact_steps, rows=16):
 
 
 def run_reference(args, rank, world):
-    """The CPU checker as the reference arm: each step is one bounded sample."""
+    """The CPU oracle as the reference arm: each step is one bounded sample."""
     if rank != 0:
         return
     w = WORKLOADS[args.workload]
@@ -492,8 +492,8 @@ def run_op(args):
     peaks, _ = load_peaks()
     L, D, H, d = tokens(w), w["hidden"], w["heads"], w["head_dim"]
     dev = torch.device("cuda")
-    cfg1 = dict(w, layers=1)
-    ctx = wdc.Context(dit_config(cfg1), w["T"])
+    one_layer = dict(w, layers=1)
+    ctx = wdc.Context(dit_config(one_layer), w["T"])
     ev = lambda: torch.cuda.Event(enable_timing=True)
     if args.op == "attention":
         q = torch.randn(H, L, d, device=dev).bfloat16()

@@ -39,7 +39,7 @@ typedef enum wdc_status {
     WDC_OK = 0,
     WDC_ERR_INVALID_ARG = 1,   /* bad pointer, size, alignment or config        */
     WDC_ERR_CUDA = 2,          /* a CUDA runtime/driver call failed              */
-    WDC_ERR_UNSUPPORTED = 3,   /* valid request this build does not implement    */
+    WDC_ERR_UNSUPPORTED = 3,   /* valid request this library does not implement    */
     WDC_ERR_TIMEOUT = 4,       /* a bounded device-side wait gave up             */
     WDC_ERR_NONFINITE = 5,     /* reserved: non-finite data where it is an error */
     WDC_ERR_STATE = 6,         /* call out of order for the context's state      */

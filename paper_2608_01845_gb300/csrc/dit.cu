@@ -2,7 +2,7 @@
 // tokens, and its orchestration on one GPU.
 //
 // Layer layout (the paper takes F_theta from its backbone; this is the DiT
-// reading shared with the CPU checker):
+// reading shared with the CPU oracle):
 //   x = [Linear(cond tokens); Linear(patchify(z)) + sinusoidal position]
 //   per block: x += gate1 * (W_o Attn(LN(x)(1+scale1)+shift1) + b_o)
 //              x += gate2 * (W_2 GELU_tanh(W_1 (LN(x)(1+scale2)+shift2) + b_1) + b_2)

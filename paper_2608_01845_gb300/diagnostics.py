@@ -119,7 +119,7 @@ def _sigmas(T, shift=1.0):
 def downstream_impact(ctx, z_T, conds, cond_tokens, steps=None, tau_d=0.025, tau_D=0.06):
     """Single-injection diagnostics on the GPU (module docstring).  The
     context's tau_risk must be negative.  Returns the same dict layout as the
-    CPU checker's ``downstream_impact``."""
+    CPU oracle's ``downstream_impact``."""
     assert ctx.params.tau_risk < 0
     torch = __import__("torch")
     T = ctx.sched.T

@@ -2,7 +2,7 @@
 weights, bank contents).
 
 This module holds no arithmetic of the method: it only draws numbers.  Tests
-feed the same arrays to the CUDA path and to the CPU checker, and ``bench.py``
+feed the same arrays to the CUDA path and to the CPU oracle, and ``bench.py``
 uses it to build its workloads.  It imports neither of them.
 
 Every generator is a pure function of its seed (numpy PCG64).

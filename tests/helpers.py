@@ -1,4 +1,4 @@
-"""Test helpers: move state between the CPU checker's representation and the
+"""Test helpers: move state between the CPU oracle's representation and the
 C ABI's host structs; comparison utilities."""
 import numpy as np
 

@@ -1,5 +1,5 @@
 """Ablation variants (section "Ablation Study", Tables 3 and 4) and the
-residual reading of Eq. 5 on the GPU against the CPU checker: the cfg0 model (2 layers, D=256, latent
+residual reading of Eq. 5 on the GPU against the CPU oracle: the 2-layer parity model (D=256, latent
 16x4x16x16, fp32 parity mode) rolled out under each variant, one flag at a
 time plus the core factorization (periodic / risk x secant / lifted).  The
 decision sequence must be identical and the final latent within 1e-5
@@ -16,7 +16,7 @@ from oracle.params import DiTConfig
 from paper_2608_01845_gb300 import synth, wdc
 
 pytestmark = pytest.mark.gpu
-CFG0 = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
+PARITY_MODEL = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
             height=16, width=16, patch=2, cond_tokens=16, cond_dim=256, dual_stream=0)
 T = 10
 
@@ -37,11 +37,11 @@ VARIANTS = {
 
 @pytest.fixture(scope="module")
 def model():
-    W = synth.dit_weights(CFG0, 0, std=0.02)
+    W = synth.dit_weights(PARITY_MODEL, 0, std=0.02)
     z0 = synth.latent(1, (16, 4, 16, 16))
     ct = synth.cond_tokens(2, 16, 256)
     desc = synth.cond_descriptors(3)
-    cfg = DiTConfig(**CFG0)
+    cfg = DiTConfig(**PARITY_MODEL)
     cache = {}
 
     def F(z, t, c, k):
@@ -54,8 +54,8 @@ def model():
 
 
 def _oracle_with_margin(kw, z0, desc, F):
-    """The first threshold for which the checker's rollout takes both
-    decisions with every tie margin above 1e-4 (chosen from the checker only)."""
+    """The first threshold for which the oracle's rollout takes both
+    decisions with every tie margin above 1e-4 (chosen from the oracle only)."""
     for tau in (0.5, 0.3, 0.8, 1.2, 0.2):
         op, cp = params_for_both(tau_risk=tau, **kw)
         zf, dec, tr = ro.cached_rollout(z0, F, desc, sch.sigmas(T), op)
@@ -70,7 +70,7 @@ def _oracle_with_margin(kw, z0, desc, F):
 def test_ablation_rollout_matches_oracle(model, name):
     W, z0, ct, desc, F = model
     op, cp, zf_o, dec_o, tr_o = _oracle_with_margin(VARIANTS[name], z0, desc, F)
-    ctx = wdc.Context(wdc.make_config(dtype=wdc.F32, **CFG0), T, params=cp)
+    ctx = wdc.Context(wdc.make_config(dtype=wdc.F32, **PARITY_MODEL), T, params=cp)
     ctx.set_weights(W)
     c = wdc.make_cond(torch.from_numpy(ct).cuda(), desc["cam"], desc["depth"])
     out = torch.empty(z0.size, dtype=torch.float32, device="cuda")
@@ -90,7 +90,7 @@ def test_periodic_placement_pattern_on_gpu(model):
     # tau_risk < 0: only the period places surrogate steps
     W, z0, ct, desc, F = model
     _, cp = params_for_both(tau_risk=-1.0, q_gap_max=1.0, sim_min=-1.0, flags=wdc.ABL_PERIODIC, period=4)
-    ctx = wdc.Context(wdc.make_config(dtype=wdc.F32, **CFG0), T, params=cp)
+    ctx = wdc.Context(wdc.make_config(dtype=wdc.F32, **PARITY_MODEL), T, params=cp)
     ctx.set_weights(W)
     c = wdc.make_cond(torch.from_numpy(ct).cuda(), desc["cam"], desc["depth"])
     out = torch.empty(z0.size, dtype=torch.float32, device="cuda")
@@ -100,7 +100,7 @@ def test_periodic_placement_pattern_on_gpu(model):
 
 def test_linear_readout_weights_match_oracle_at_larger_bank():
     # the surrogate step alone, bank of 6 records, linear observation: the
-    # readout coefficients (reported as kappa) against the checker's solve
+    # readout coefficients (reported as kappa) against the oracle's solve
     from helpers import make_state, state_to_host
     from oracle import surrogate as sg
     n, K, k = 1 << 16, 6, 20

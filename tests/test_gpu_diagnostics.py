@@ -1,5 +1,5 @@
 """Synthetic diagnostics (Fig. 2, Fig. 3a readings) on the GPU against the
-CPU checker's, on the cfg0 model (2 layers, D=256, latent 16x4x16x16, fp32
+CPU oracle's, on the 2-layer parity model (D=256, latent 16x4x16x16, fp32
 parity mode): single-injection local and downstream defects, the
 predicted / counterfactual defect pairs, and the direction error per streak
 position."""
@@ -16,24 +16,24 @@ from paper_2608_01845_gb300 import diagnostics as gdg
 from paper_2608_01845_gb300 import synth, wdc
 
 pytestmark = pytest.mark.gpu
-CFG0 = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
+PARITY_MODEL = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
             height=16, width=16, patch=2, cond_tokens=16, cond_dim=256, dual_stream=0)
 T = 10
 
 
 @pytest.fixture(scope="module")
 def model():
-    W = synth.dit_weights(CFG0, 0, std=0.02)
+    W = synth.dit_weights(PARITY_MODEL, 0, std=0.02)
     z0 = synth.latent(1, (16, 4, 16, 16)).reshape(-1)
     ct = synth.cond_tokens(2, 16, 256)
     desc = synth.cond_descriptors(3)
-    cfg = DiTConfig(**CFG0)
+    cfg = DiTConfig(**PARITY_MODEL)
     F = lambda z, t, c, k: dit.forward(W, cfg, np.asarray(z).reshape(16, 4, 16, 16), t, ct)
     return W, z0, ct, desc, F
 
 
 def _ctx(W, cp):
-    ctx = wdc.Context(wdc.make_config(dtype=wdc.F32, **CFG0), T, params=cp)
+    ctx = wdc.Context(wdc.make_config(dtype=wdc.F32, **PARITY_MODEL), T, params=cp)
     ctx.set_weights(W)
     return ctx
 

@@ -1,4 +1,4 @@
-"""Parity of the denoiser F_theta's CUDA kernels with the CPU checker.
+"""Parity of the denoiser F_theta's CUDA kernels with the CPU oracle.
 
 fp32 mode: full forward of the 2-layer D=256 model (and a dual-stream
 variant), rel L2 <= 1e-5 against fp64.  bf16 mode: the GEMM and attention
@@ -17,7 +17,7 @@ from paper_2608_01845_gb300 import synth, wdc
 pytestmark = pytest.mark.gpu
 BF16_TOL = 2e-2
 
-CFG0 = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
+PARITY_MODEL = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
             height=16, width=16, patch=2, cond_tokens=16, cond_dim=256, dual_stream=0)
 
 
@@ -32,7 +32,7 @@ def _to_dev(a, dtype=torch.float32):
 
 @pytest.mark.parametrize("dual", [0, 1])
 def test_fp32_forward_matches_oracle(dual):
-    cfgd = dict(CFG0, dual_stream=dual, layers=2 if not dual else 1)
+    cfgd = dict(PARITY_MODEL, dual_stream=dual, layers=2 if not dual else 1)
     W = synth.dit_weights(cfgd, 7, std=0.02, bias_std=0.02)
     ctx = _ctx(cfgd, wdc.F32)
     ctx.set_weights(W)
@@ -46,14 +46,14 @@ def test_fp32_forward_matches_oracle(dual):
 
 
 def test_fp32_modulation_matches_oracle():
-    W = synth.dit_weights(CFG0, 8, std=0.05, bias_std=0.02)
-    ctx = _ctx(CFG0, wdc.F32)
+    W = synth.dit_weights(PARITY_MODEL, 8, std=0.05, bias_std=0.02)
+    ctx = _ctx(PARITY_MODEL, wdc.F32)
     ctx.set_weights(W)
     D = 256
     out = torch.empty(2 * 6 * D + 2 * D, dtype=torch.float32, device="cuda")
     ctx.dit_modulation(250.0, out)
     torch.cuda.synchronize()
-    _, mods, fm = dit.conditioning(W, DiTConfig(**CFG0), 250.0)
+    _, mods, fm = dit.conditioning(W, DiTConfig(**PARITY_MODEL), 250.0)
     want = np.concatenate([mods[(0, 0)].ravel(), mods[(1, 0)].ravel(), fm.ravel()])
     assert rel_l2(out.cpu().numpy(), want) <= 1e-5
 
@@ -70,7 +70,7 @@ def _h(a):
 @pytest.mark.parametrize("M,N,K", [(300, 384, 320), (128, 256, 64), (1000, 768, 1024), (17, 64, 128)])
 @pytest.mark.parametrize("mode", ["store", "gelu", "resid"])
 def test_bf16_gemm_matches_oracle(M, N, K, mode):
-    ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
+    ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.BF16)
     A = _bf(synth.normal(1, (M, K)))
     W = _bf(synth.normal(2, (N, K), 0.05))
     b = synth.normal(3, (N,), 0.1)
@@ -99,7 +99,7 @@ def test_bf16_gemm_matches_oracle(M, N, K, mode):
 def test_bf16_attention_matches_oracle(H, L, d):
     """L % 8 == 0 runs the tcgen05 kernel (ragged against its 128-key and
     256-query tiles); other L the SIMT kernel."""
-    ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
+    ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.BF16)
     q = _bf(synth.normal(11, (H, L, d)))
     k = _bf(synth.normal(12, (H, L, d)))
     v = _h(synth.normal(13, (H, L, d)))
@@ -116,7 +116,7 @@ def test_bf16_attention_matches_oracle(H, L, d):
 
 @pytest.mark.parametrize("H,L,d", [(2, 300, 64), (2, 257, 128)])
 def test_fp32_attention_matches_oracle(H, L, d):
-    ctx = _ctx(dict(CFG0, layers=1), wdc.F32)
+    ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.F32)
     q, k, v = (synth.normal(s, (H, L, d)) for s in (21, 22, 23))
     o = torch.empty(L, H * d, dtype=torch.float32, device="cuda")
     ctx.op_attention(_to_dev(q), _to_dev(k), _to_dev(np.ascontiguousarray(v.transpose(0, 2, 1))), o)
@@ -192,7 +192,7 @@ def test_bf16_attention_full_size_sampled_rows(H, L, d):
     """The attention shapes of the 5B-scale (48 x 64 heads, L = 17776) and
     13B-scale (24 x 128 heads, L = 13568) models; 96 sampled query rows per
     head compared with fp64."""
-    ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
+    ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.BF16)
     g = np.random.default_rng(44)
     q = _bf(g.standard_normal((H, L, d), dtype=np.float32))
     k = _bf(g.standard_normal((H, L, d), dtype=np.float32))
@@ -213,7 +213,7 @@ def test_bf16_attention_full_size_sampled_rows(H, L, d):
 def test_bf16_gemm_sampled_full_size_and_no_device_errors(M, N, K):
     """Full 5B-scale QKV shape (the CTA-pair kernel) checked on 64 sampled rows;
     no kernel reported a timeout or a tensor-memory pair mismatch."""
-    ctx = _ctx(dict(CFG0, layers=1), wdc.BF16)
+    ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.BF16)
     g = np.random.default_rng(55)
     A = _bf(g.standard_normal((M, K), dtype=np.float32))
     W = _bf(0.05 * g.standard_normal((N, K), dtype=np.float32))

@@ -1,4 +1,4 @@
-"""Cached rollout on the GPU against the CPU checker (2-layer D=256 model,
+"""Cached rollout on the GPU against the CPU oracle (2-layer D=256 model,
 latent 16x4x16x16, fp32 parity mode): the anchor/skip decision sequence must
 be identical and the final latent within 1e-4 relative L2 (fp32 kernels vs
 fp64).  Plus the invariants: all-exact == native bitwise, host-pointer API ==
@@ -19,14 +19,14 @@ from paper_2608_01845_gb300 import synth, wdc
 
 pytestmark = pytest.mark.gpu
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
-CFG0 = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
+PARITY_MODEL = dict(layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
             height=16, width=16, patch=2, cond_tokens=16, cond_dim=256, dual_stream=0)
 
 
 def _setup(T, **pkw):
     op, cp = params_for_both(**pkw)
-    W = synth.dit_weights(CFG0, 0, std=0.02)
-    ctx = wdc.Context(wdc.make_config(dtype=wdc.F32, **CFG0), T, params=cp)
+    W = synth.dit_weights(PARITY_MODEL, 0, std=0.02)
+    ctx = wdc.Context(wdc.make_config(dtype=wdc.F32, **PARITY_MODEL), T, params=cp)
     ctx.set_weights(W)
     z0 = synth.latent(1, (16, 4, 16, 16))
     ct = synth.cond_tokens(2, 16, 256)
@@ -35,7 +35,7 @@ def _setup(T, **pkw):
 
 
 def _oracle(op, W, z0, ct, desc, T):
-    cfg = DiTConfig(**CFG0)
+    cfg = DiTConfig(**PARITY_MODEL)
     F = lambda z, t, c, k: dit.forward(W, cfg, np.asarray(z).reshape(16, 4, 16, 16), t, ct)
     return ro.cached_rollout(z0, F, desc, sch.sigmas(T), op)
 
@@ -144,7 +144,7 @@ def test_graph_rollout_dual_stream_bf16_equals_host():
     """bf16 dual-stream model: the captured forward forks the condition rows
     onto a second stream; graph and host rollouts agree bitwise."""
     T = 8
-    cfg = dict(CFG0, dual_stream=1)
+    cfg = dict(PARITY_MODEL, dual_stream=1)
     W = synth.dit_weights(cfg, 0, std=0.02)
     _, cp = params_for_both(tau_risk=0.5)
     ctx = wdc.Context(wdc.make_config(dtype=wdc.BF16, **cfg), T, params=cp)

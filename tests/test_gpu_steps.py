@@ -1,5 +1,5 @@
 """Parity of the fused step kernels (skip pass: Eq. 2-6, 9, 10; anchor pass:
-Eq. 1, 7, 8 and the bank insertion) with the CPU checker, element by element,
+Eq. 1, 7, 8 and the bank insertion) with the CPU oracle, element by element,
 on seeded synthetic banks with smooth drift.  Tolerance: 1e-5 relative for the
 fp32 latents and the reduced statistics; decisions and integer fields exact."""
 import copy

@@ -145,16 +145,16 @@ def test_zero_final_weights_give_bias_field():
 
 
 def test_dual_stream_with_equal_weights_equals_single_stream():
-    cfg1 = _tiny_cfg(layers=1)
-    cfg2 = _tiny_cfg(layers=1, dual_stream=1)
-    W2 = synth.dit_weights(cfg2.as_dict(), 9, std=0.2, bias_std=0.1)
+    cfg_single = _tiny_cfg(layers=1)
+    cfg_dual = _tiny_cfg(layers=1, dual_stream=1)
+    W2 = synth.dit_weights(cfg_dual.as_dict(), 9, std=0.2, bias_std=0.1)
     for key in list(W2):
         if key.startswith("L0.s1."):
             W2[key] = W2["L0.s0." + key[len("L0.s1."):]]
     W1 = {k: v for k, v in W2.items() if not k.startswith("L0.s1.")}
     z = np.random.default_rng(9).standard_normal((4, 2, 4, 4))
     c = np.random.default_rng(10).standard_normal((3, 32))
-    assert np.allclose(dit.forward(W1, cfg1, z, 300.0, c), dit.forward(W2, cfg2, z, 300.0, c), atol=1e-13)
+    assert np.allclose(dit.forward(W1, cfg_single, z, 300.0, c), dit.forward(W2, cfg_dual, z, 300.0, c), atol=1e-13)
 
 
 # ------------------------------------------------------------------ rollouts
