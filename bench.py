@@ -492,6 +492,8 @@ def run_op(args):
     peaks, _ = load_peaks()
     L, D, H, d = tokens(w), w["hidden"], w["heads"], w["head_dim"]
     dev = torch.device("cuda")
+    if args.op == "batch":
+        return run_batch(args, w, peaks)
     one_layer = dict(w, layers=1)
     ctx = wdc.Context(dit_config(one_layer), w["T"])
     ev = lambda: torch.cuda.Event(enable_timing=True)
@@ -592,6 +594,54 @@ def run_op(args):
     print(json.dumps({"op": args.op, "workload": args.workload, "ms": ms, unit: work / (ms * 1e-3) / 1e12}))
 
 
+def run_batch(args, w, peaks):
+    """Batched cached rollout (wdc_rollout_batch) of --batch samples of the
+    workload, each from its own latent, against the same samples rolled out
+    one at a time (a batch of one each).  With --cfg every exact step runs the
+    guided velocity (conditional + null-condition forward in one batch)."""
+    import torch
+    from paper_2608_01845_gb300 import wdc
+    B = args.batch
+    cfg = dit_config(w)
+    cfg.max_batch = 2 * B if args.cfg else B
+    T = w["T"]
+    prm = lambda: wdc.make_params(tau_risk=w["tau_risk"])
+    ctxs = [wdc.Context(cfg, T, params=prm())]
+    ctxs[0].init_weights(w["weight_seed"], 0.02)
+    lat = wdc.make_config(in_ch=w["in_ch"], frames=w["frames"], height=w["height"], width=w["width"])
+    ctxs += [wdc.Context(lat, T, params=prm()) for _ in range(1, B)]
+    _, ct, desc = inputs(w, 0)
+    ct = torch.from_numpy(ct).cuda()
+    zs = [torch.from_numpy(inputs(w, b)[0]).cuda() for b in range(B)]
+    conds = [wdc.make_cond(ct, desc["cam"], desc["depth"]) for _ in range(B)]
+    outs = [torch.empty_like(z) for z in zs]
+    kw = dict(cfg=args.cfg, guidance=args.guidance, trace=False)
+
+    def batched():
+        return wdc.rollout_batch(ctxs, zs, conds, outs, **kw)[0]
+
+    def sequential():
+        return [wdc.rollout_batch([ctxs[0]], [zs[b]], [conds[b]], [outs[b]], **kw)[0][0] for b in range(B)]
+
+    res = {}
+    for name, fn in [("batched", batched), ("sequential", sequential)]:
+        decs = fn()                                   # warm-up (and the decisions)
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(args.reps):
+            t0 = time.perf_counter()
+            fn()
+            torch.cuda.synchronize()
+            ts.append(time.perf_counter() - t0)
+        sec = statistics.median(ts)
+        res[name] = {"s": sec, "samples_per_s": B / sec, "steps_per_s": B * T / sec,
+                     "exact_steps": [T - sum(d) for d in decs]}
+    res["batched"]["exact_batches"] = sum(1 for k in range(T) if any(d[k] == 0 for d in decs))
+    print(json.dumps({"op": "batch", "workload": args.workload, "B": B, "cfg": bool(args.cfg),
+                      "guidance": args.guidance if args.cfg else None, **res,
+                      "speedup": res["sequential"]["s"] / res["batched"]["s"]}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -602,8 +652,12 @@ def main():
     ap.add_argument("--ablation", choices=sorted(ABLATIONS),
                     help="run the timed rollout under one ablation variant (Tables 3-4) and report its "
                          "final latent against the uncached rollout")
-    ap.add_argument("--op", choices=["attention", "gemm", "gemms", "block", "skip", "secant", "control"],
-                    help="time one operator at its 5B-scale shape (profiler captures)")
+    ap.add_argument("--op", choices=["attention", "gemm", "gemms", "block", "skip", "secant", "control", "batch"],
+                    help="time one operator at its 5B-scale shape (profiler captures); batch: the batched "
+                         "cached rollout against one-at-a-time rollouts")
+    ap.add_argument("--batch", type=int, default=2, help="--op batch: samples per batch")
+    ap.add_argument("--cfg", action="store_true", help="--op batch: classifier-free guidance on every exact step")
+    ap.add_argument("--guidance", type=float, default=5.0, help="--op batch: guidance scale with --cfg")
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="5b",
                     help="rollout / --op shape (5b: 42 layers, 48x64 heads, L=17776; 13b: 60 dual-stream layers, "

@@ -49,6 +49,7 @@ typedef enum wdc_status {
 enum { WDC_F32 = 0, WDC_BF16 = 1 };
 
 #define WDC_MAX_BANK 8          /* largest supported bank capacity K           */
+#define WDC_MAX_BATCH 16        /* most latents one batched forward may hold   */
 #define WDC_SUMMARY_DIM 256     /* the fixed summary s(.) (section "Kernelized Nonlinear Observation") */
 #define WDC_SKETCH 120          /* buckets of each latent block of s(.)        */
 
@@ -70,6 +71,10 @@ typedef struct wdc_dit_config {
     int cond_tokens, cond_dim;
     int dual_stream;            /* 1: separate block weights for condition tokens */
     int dtype;                  /* WDC_F32 (fp32 parity mode) or WDC_BF16          */
+    int max_batch;              /* latents one batched forward may hold, counting
+                                   both halves of a guided pair (0 or 1: single;
+                                   at most WDC_MAX_BATCH); activation buffers
+                                   are sized for it */
 } wdc_dit_config;
 
 /* Flow-matching Euler schedule: sigma_k = 1 - k/T, shifted by
@@ -260,6 +265,26 @@ wdc_status wdc_init_weights(wdc_ctx* ctx, unsigned long long seed, float std);
  * output.  Asynchronous. */
 wdc_status wdc_dit_forward(wdc_ctx* ctx, const float* z_t, float t, const float* cond_tokens,
                            float* v, wdc_stream stream);
+/* Batched F_theta (the paper runs one trajectory at a time and is silent on
+ * batching and on classifier-free guidance; both are serving extensions that
+ * do not change what one sample computes).  B latents z_t[b] (device fp32,
+ * 16-byte aligned) at the same model timestep t, each with its own condition
+ * tokens cond_tokens[b] (device fp32 [cond_tokens, cond_dim]; the array may
+ * be NULL when the model has no condition tokens).  One forward holds all of
+ * them: every GEMM and row-wise kernel runs once over all samples' tokens,
+ * the attention once over all samples' heads (each sample attends to its own
+ * tokens only).  Writes v[b] (device fp32, 16-byte aligned, latent-shaped).
+ *   cfg == 0: v[b] = F(z_t[b], t, c_b); needs B <= max_batch.
+ *   cfg == 1: guided velocity v[b] = F(z, t, 0) + guidance (F(z, t, c_b) -
+ *             F(z, t, 0)), where 0 is the all-zero token set (the null
+ *             condition); the 2B forwards share one batch, so 2B <= max_batch.
+ * A sample's velocity is bitwise the same as that of wdc_dit_forward on it
+ * alone.  Host arrays z_t, cond_tokens and v hold B pointers each.  Errors:
+ * WDC_ERR_INVALID_ARG for B < 1, B (2B) > max_batch or a null / unaligned
+ * pointer.  Asynchronous. */
+wdc_status wdc_dit_forward_batch(wdc_ctx* ctx, int B, const float* const* z_t, float t,
+                                 const float* const* cond_tokens, int cfg, float guidance,
+                                 float* const* v, wdc_stream stream);
 /* One DiT block in place on the token sequence x (device, model dtype,
  * [cond_tokens + video_tokens, hidden]) with modulation mod6 (device fp32,
  * [streams][6][hidden] = shift1, scale1, gate1, shift2, scale2, gate2). */
@@ -339,6 +364,27 @@ wdc_status wdc_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* conds, in
  * context's step-API state is that of the rollout's end. */
 wdc_status wdc_rollout_graph(wdc_ctx* ctx, const float* z_T, const wdc_cond* cond, float* z_out,
                              int* decisions, wdc_step_info* trace, wdc_stream stream);
+/* B independent cached rollouts advanced in lockstep (the paper's method per
+ * sample; batching itself has no counterpart in the paper).  ctxs[b] holds
+ * sample b's cache state and controller parameters; ctxs[0] also owns the
+ * denoiser that every sample's exact steps run through (its max_batch must
+ * cover the largest exact batch: B, or 2B with cfg), the others may be
+ * created with layers == 0.  All contexts must be distinct, on one device,
+ * with the same latent size and schedule.  At step k every sample's skip pass
+ * runs and decides (one stream synchronisation for all), then the samples
+ * that decided Exact share one batched forward (wdc_dit_forward_batch, with
+ * cfg / guidance as there) and each runs its anchor pass.  z_T[b] and z_out[b]
+ * may be device or host pointers; conds holds B * n_cond entries (sample-major,
+ * n_cond 1 or T) whose tokens must be device pointers when the model has
+ * condition tokens.  decisions (host int[B*T]) and trace (host
+ * wdc_step_info[B*T]), sample-major, may be NULL.  Each sample's decisions,
+ * trace and final latent equal those of wdc_rollout on that sample alone
+ * (with cfg, of the guided velocity).  Argument errors are reported on
+ * ctxs[0]; an error inside one sample's step pass on that sample's context. */
+wdc_status wdc_rollout_batch(wdc_ctx* const* ctxs, int B, const float* const* z_T,
+                             const wdc_cond* conds, int n_cond, int cfg, float guidance,
+                             float* const* z_out, int* decisions, wdc_step_info* trace,
+                             wdc_stream stream);
 /* The uncached rollout: wdc_dit_forward + wdc_scheduler_step at every step. */
 wdc_status wdc_native_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* conds, int n_cond,
                               float* z_out, wdc_stream stream);

@@ -118,6 +118,7 @@ wdc_status check_cfg(Ctx* c, const wdc_dit_config& g) {
     if (g.in_ch <= 0 || g.frames <= 0 || g.height <= 0 || g.width <= 0)
         return fail(c, WDC_ERR_INVALID_ARG, "latent shape must be positive");
     if (g.layers < 0) return fail(c, WDC_ERR_INVALID_ARG, "layers must be >= 0");
+    if (g.max_batch < 0 || g.max_batch > WDC_MAX_BATCH) return fail(c, WDC_ERR_INVALID_ARG, "max_batch must be 0..16");
     if (g.layers == 0) return WDC_OK;
     if (g.dtype != WDC_F32 && g.dtype != WDC_BF16) return fail(c, WDC_ERR_INVALID_ARG, "dtype must be WDC_F32 or WDC_BF16");
     if (g.head_dim != 64 && g.head_dim != 128) return fail(c, WDC_ERR_UNSUPPORTED, "head_dim must be 64 or 128");
@@ -476,6 +477,15 @@ wdc_status wdc_dit_forward(wdc_ctx* h, const float* z_t, float t, const float* c
     return dit_forward(c, z_t, t, cond_tokens, v, (cudaStream_t)stream);
 }
 
+wdc_status wdc_dit_forward_batch(wdc_ctx* h, int B, const float* const* z_t, float t, const float* const* cond_tokens,
+                                 int cfg, float guidance, float* const* v, wdc_stream stream) {
+    Ctx* c = reinterpret_cast<Ctx*>(h);
+    if (!c) return WDC_ERR_INVALID_ARG;
+    if (B < 1 || B > WDC_MAX_BATCH) return fail(c, WDC_ERR_INVALID_ARG, "B must be 1..16");
+    cudaSetDevice(c->device);
+    return dit_forward_guided(c, B, z_t, t, cond_tokens, cfg ? 1 : 0, guidance, v, (cudaStream_t)stream);
+}
+
 wdc_status wdc_dit_block_forward(wdc_ctx* h, int layer, void* x, const float* mod6, wdc_stream stream) {
     Ctx* c = reinterpret_cast<Ctx*>(h);
     if (!c) return WDC_ERR_INVALID_ARG;
@@ -776,6 +786,114 @@ wdc_status wdc_rollout_graph(wdc_ctx* h, const float* z_T, const wdc_cond* cond,
     const bool tok_dev = cond_elems && is_device_ptr(cond->tokens);
     return graph_rollout(c, z_T, in_dev, cond, tok_dev ? cond->tokens : nullptr, z_out, out_dev, decisions, trace,
                          (cudaStream_t)stream);
+}
+
+wdc_status wdc_rollout_batch(wdc_ctx* const* hs, int B, const float* const* z_T, const wdc_cond* conds, int n_cond,
+                             int cfg, float guidance, float* const* z_out, int* decisions, wdc_step_info* trace,
+                             wdc_stream stream) {
+    if (!hs || !hs[0]) return WDC_ERR_INVALID_ARG;
+    Ctx* c0 = reinterpret_cast<Ctx*>(hs[0]);
+    cudaSetDevice(c0->device);
+    cudaStream_t s = (cudaStream_t)stream;
+    const int T = c0->sched.T;
+    if (B < 1 || B > WDC_MAX_BATCH) return fail(c0, WDC_ERR_INVALID_ARG, "B must be 1..16");
+    if (!c0->dit) return fail(c0, WDC_ERR_UNSUPPORTED, "ctxs[0] must own a denoiser (layers > 0)");
+    const int max_batch = c0->cfg.max_batch > 1 ? c0->cfg.max_batch : 1;
+    if ((cfg ? 2 * B : B) > max_batch) return fail(c0, WDC_ERR_INVALID_ARG, "batch larger than ctxs[0]'s max_batch");
+    if (!z_T || !z_out || !conds) return fail(c0, WDC_ERR_INVALID_ARG, "null pointer array");
+    if (n_cond != 1 && n_cond != T) return fail(c0, WDC_ERR_INVALID_ARG, "n_cond must be 1 or T");
+    const size_t cond_elems = (size_t)c0->cfg.cond_tokens * c0->cfg.cond_dim;
+    std::vector<Ctx*> cs(B);
+    for (int b = 0; b < B; ++b) {
+        Ctx* cb = reinterpret_cast<Ctx*>(hs[b]);
+        if (!cb) return fail(c0, WDC_ERR_INVALID_ARG, "null context");
+        for (int a = 0; a < b; ++a)
+            if (cs[a] == cb) return fail(c0, WDC_ERR_INVALID_ARG, "every sample needs its own context");
+        if (cb->device != c0->device || cb->n != c0->n || cb->sched.T != T || cb->sigma != c0->sigma)
+            return fail(c0, WDC_ERR_INVALID_ARG, "contexts differ in device, latent size or schedule");
+        if (!z_T[b] || !z_out[b]) return fail(c0, WDC_ERR_INVALID_ARG, "null latent");
+        for (int i = 0; i < n_cond && cond_elems; ++i)
+            if (!conds[b * n_cond + i].tokens || !is_device_ptr(conds[b * n_cond + i].tokens))
+                return fail(c0, WDC_ERR_INVALID_ARG, "condition tokens must be device pointers");
+        cs[b] = cb;
+    }
+    const size_t bytes = c0->n * sizeof(float);
+    std::vector<float*> cur(B);
+    std::vector<int> cur_cand(B, 0);
+    wdc_status st;
+    for (int b = 0; b < B; ++b) {
+        Ctx* cb = cs[b];
+        const bool in_dev = is_device_ptr(z_T[b]);
+        if (in_dev && !aligned16(z_T[b])) return fail(c0, WDC_ERR_INVALID_ARG, "z_T must be 16-byte aligned");
+        WDC_CUDA_TRY(c0, cudaMemcpyAsync(cb->cand[0], z_T[b], bytes, in_dev ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s));
+        cur[b] = cb->cand[0];
+        if ((st = wdc_state_reset(reinterpret_cast<wdc_ctx*>(cb), cur[b], s))) return st;
+    }
+    std::vector<int> ex;
+    std::vector<float*> zh(B);
+    std::vector<const float*> zs, toks;
+    std::vector<float*> vs;
+    for (int k = 0; k < T; ++k) {
+        const int ci = n_cond == 1 ? 0 : k;
+        std::vector<int> nb(B), age(B);
+        for (int b = 0; b < B; ++b) {
+            Ctx* cb = cs[b];
+            zh[b] = cb->cand[cur_cand[b] == 0 ? 1 : 0];
+            nb[b] = cb->n_bank;
+            age[b] = cb->age;
+            if ((st = enqueue_skip(cb, k, &conds[b * n_cond + ci], cur[b], zh[b], &cb->out_host[k], s))) return st;
+        }
+        if ((st = sync(c0, s))) return st;
+        ex.clear(); zs.clear(); toks.clear(); vs.clear();
+        for (int b = 0; b < B; ++b) {
+            Ctx* cb = cs[b];
+            const StepOut& o = cb->out_host[k];
+            cb->last_surrogate_k = k;
+            if (decisions) decisions[b * T + k] = o.decision;
+            if (trace) fill_info(o, k, nb[b], age[b], &trace[b * T + k]);
+            if (o.decision) {
+                cb->age++;
+                cur[b] = zh[b];
+                cur_cand[b] = cur_cand[b] == 0 ? 1 : 0;
+            } else {
+                ex.push_back(b);
+                zs.push_back(cur[b]);
+                toks.push_back(cond_elems ? conds[b * n_cond + ci].tokens : nullptr);
+                vs.push_back(cb->vbuf);
+            }
+        }
+        if (ex.empty()) continue;
+        if ((st = dit_forward_guided(c0, (int)ex.size(), zs.data(), (float)(1000.0 * c0->sigma[k]), toks.data(), cfg ? 1 : 0,
+                                     guidance, vs.data(), s)))
+            return st;
+        for (int b : ex) {
+            Ctx* cb = cs[b];
+            const StepOut& o = cb->out_host[k];
+            const bool cf = o.supported && o.finite;
+            const float* zn = nullptr;
+            if ((st = enqueue_anchor(cb, k, &conds[b * n_cond + ci], cur[b], cb->vbuf, cf ? zh[b] : nullptr, &zn,
+                                     &cb->out_host[T], s)))
+                return st;
+            cur[b] = const_cast<float*>(zn);
+            cur_cand[b] = -1;
+        }
+        if (trace) {
+            if ((st = sync(c0, s))) return st;
+            for (int b : ex) {
+                const StepOut& o = cs[b]->out_host[T];
+                wdc_step_info& ti = trace[b * T + k];
+                ti.d_cf = o.d_cf;
+                ti.R = o.R;
+                ti.eta = o.eta;
+                ti.r = o.r;
+            }
+        }
+    }
+    for (int b = 0; b < B; ++b) {
+        const bool out_dev = is_device_ptr(z_out[b]);
+        WDC_CUDA_TRY(c0, cudaMemcpyAsync(z_out[b], cur[b], bytes, out_dev ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost, s));
+    }
+    return sync(c0, s);
 }
 
 wdc_status wdc_native_rollout(wdc_ctx* h, const float* z_T, const wdc_cond* conds, int n_cond, float* z_out,

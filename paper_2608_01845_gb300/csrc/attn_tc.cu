@@ -85,6 +85,7 @@ struct AttnCfg {
 
 struct AttnArgs {
     int H, L, n_kv, q_blocks;
+    int Hs, nb, Lc;           // heads per sample, samples, condition tokens (output row mapping)
     float scale_log2;
     __nv_bfloat16* o;
     unsigned* err;
@@ -451,7 +452,11 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                 tmem_ld32(o_addr + c, o);
                 tmem_ld_wait();
                 if (tok < g.L) {
-                    uint4* dst = reinterpret_cast<uint4*>(g.o + (size_t)tok * g.H * D + (size_t)h * D + c);
+                    // head h = (sample, head within the sample); O row of
+                    // (sample, token) in the batch's stream-major token rows
+                    const int b = h / g.Hs, hs = h - b * g.Hs;
+                    const size_t orow = (size_t)batch_row(b, tok, g.nb, g.Lc, g.L);
+                    uint4* dst = reinterpret_cast<uint4*>(g.o + orow * g.Hs * D + (size_t)hs * D + c);
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
                         uint4 w;
@@ -474,7 +479,8 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
 }
 
 template <int D>
-wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, cudaStream_t s) {
+wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int Hs, int Lc,
+                  cudaStream_t s) {
     using Cf = AttnCfg<D>;
     static bool attr = false;
     static bool regs_ok = false;
@@ -500,6 +506,9 @@ wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o,
     AttnArgs g;
     g.H = H;
     g.L = L;
+    g.Hs = Hs;
+    g.nb = H / Hs;
+    g.Lc = Lc;
     g.n_kv = (L + BKV - 1) / BKV;
     g.q_blocks = (L + 2 * BQ - 1) / (2 * BQ);
     g.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
@@ -516,10 +525,11 @@ wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o,
 bool tc_attention_supported(int L, int d) { return L > 0 && L % 8 == 0 && (d == 64 || d == 128); }
 
 wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
-                        cudaStream_t s) {
+                        int Hs, int Lc, cudaStream_t s) {
     if (((uintptr_t)q | (uintptr_t)k | (uintptr_t)vt | (uintptr_t)o) & 15)
         return fail(c, WDC_ERR_INVALID_ARG, "attention operands must be 16-byte aligned");
-    return d == 64 ? launch<64>(c, q, k, vt, o, H, L, s) : launch<128>(c, q, k, vt, o, H, L, s);
+    if (Hs <= 0 || H % Hs || Lc < 0 || Lc >= L) return fail(c, WDC_ERR_INVALID_ARG, "bad attention batch layout");
+    return d == 64 ? launch<64>(c, q, k, vt, o, H, L, Hs, Lc, s) : launch<128>(c, q, k, vt, o, H, L, Hs, Lc, s);
 }
 
 }  // namespace wdc

@@ -27,7 +27,7 @@ bool tc_gemm_supported(int M, int N, int K);
 wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, const Epi& e, cudaStream_t s);
 bool tc_attention_supported(int L, int d);
 wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
-                        cudaStream_t s);
+                        int Hs, int Lc, cudaStream_t s);
 
 struct Lin {
     void* w = nullptr;
@@ -40,6 +40,7 @@ struct DiT {
     size_t esz = 4;
     int S = 1;                            // weight streams (2 with dual_stream)
     int D = 0, H = 0, d = 0, M = 0, E = 0, Fd = 0, P = 0, Lc = 0, Lv = 0, L = 0, Dc = 0, layers = 0;
+    int B = 1;                            // most samples one forward holds (activation buffers sized for it)
     Lin patch, cond, t1, t2, fin;
     void* modW = nullptr;                 // [(layers*S*6 + 2) * D, E]
     float* modB = nullptr;
@@ -49,6 +50,7 @@ struct DiT {
     void *x = nullptr, *h = nullptr, *q = nullptr, *k = nullptr, *vt = nullptr, *ao = nullptr, *m = nullptr;
     void *tok = nullptr, *condx = nullptr, *pe = nullptr;
     float *feat = nullptr, *h1 = nullptr, *temb = nullptr, *mods = nullptr;
+    float* vb = nullptr;                  // [B, latent] velocities of a batched forward (B > 1)
     std::vector<void*> allocs;
     // dual stream: the condition stream's row block runs on a second CUDA
     // stream forked from and joined back into the caller's, so its small
@@ -187,24 +189,53 @@ __global__ void ln_mod_vec_kernel(const __nv_bfloat16* __restrict__ x, __nv_bflo
     }
 }
 
-// tok[(f, h', w'), (c, ph, pw)] = z[c, f, h'*p+ph, w'*p+pw]
+// Per-sample device pointers of a batch, passed by value.
+struct BatchPtrs {
+    const float* p[WDC_MAX_BATCH];
+};
+
+// tok[b][(f, h', w'), (c, ph, pw)] = z_b[c, f, h'*p+ph, w'*p+pw]
 template <typename T>
-__global__ void patchify_kernel(const float* __restrict__ z, T* __restrict__ tok, int C, int F, int Hh, int Ww, int p) {
+__global__ void patchify_kernel(BatchPtrs z, int nb, T* __restrict__ tok, int C, int F, int Hh, int Ww, int p) {
     const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     const int P = C * p * p, hp = Hh / p, wp = Ww / p;
-    const long long total = (long long)F * hp * wp * P;
-    if (i >= total) return;
-    const int col = (int)(i % P);
-    const long long m = i / P;
+    const long long per = (long long)F * hp * wp * P;
+    if (i >= per * nb) return;
+    const int b = (int)(i / per);
+    const long long ii = i - b * per;
+    const int col = (int)(ii % P);
+    const long long m = ii / P;
     const int f = (int)(m / (hp * wp)), rem = (int)(m % (hp * wp)), h2 = rem / wp, w2 = rem % wp;
     const int c = col / (p * p), r2 = col % (p * p), ph = r2 / p, pw = r2 % p;
-    tok[i] = to_act<T>(z[(((size_t)c * F + f) * Hh + h2 * p + ph) * Ww + w2 * p + pw]);
+    tok[i] = to_act<T>(z.p[b][(((size_t)c * F + f) * Hh + h2 * p + ph) * Ww + w2 * p + pw]);
 }
 
+// dst[b][i] = src_b[i] in the model dtype; a null src_b is the all-zero set.
 template <typename T>
-__global__ void convert_kernel(const float* __restrict__ src, T* __restrict__ dst, long long n) {
+__global__ void convert_kernel(BatchPtrs src, int nb, T* __restrict__ dst, long long per) {
     const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i < n) dst[i] = to_act<T>(src[i]);
+    if (i >= per * nb) return;
+    const int b = (int)(i / per);
+    const float* sp = src.p[b];
+    dst[i] = to_act<T>(sp ? sp[i - b * per] : 0.0f);
+}
+
+// Guided velocity (cfg) or plain scatter of a batched forward's [nb, n]
+// velocities into the callers' buffers: cfg: rows (2b, 2b+1) = (conditional,
+// null-condition) forwards of sample b, v_b = v_u + g (v_c - v_u).
+__global__ void guide_kernel(const float* __restrict__ vb, long long n, int B, int cfg, float g, BatchPtrs dst) {
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n * B) return;
+    const int b = (int)(i / n);
+    const long long j = i - b * n;
+    float v;
+    if (cfg) {
+        const float vc = vb[(2 * b) * n + j], vu = vb[(2 * b + 1) * n + j];
+        v = fmaf(g, vc - vu, vu);
+    } else {
+        v = vb[i];
+    }
+    const_cast<float*>(dst.p[b])[j] = v;
 }
 
 template <typename T>
@@ -301,8 +332,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
 // One thread per query row, online softmax over key tiles staged in shared memory.
 template <typename T, typename TV, int HD>
 __global__ void __launch_bounds__(128) attn_simt_kernel(const T* __restrict__ q, const T* __restrict__ k,
-                                                         const TV* __restrict__ vt, T* __restrict__ o, int H, int L,
-                                                         float scale) {
+                                                         const TV* __restrict__ vt, T* __restrict__ o, int Hs, int nb,
+                                                         int Lc, int L, float scale) {
     constexpr int KT = HD <= 64 ? 64 : 32;
     __shared__ float Ks[KT][HD + 1];
     __shared__ float Vs[KT][HD + 1];
@@ -345,8 +376,10 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const T* __restrict__ q,
     }
     if (qi < L) {
         const float inv = 1.0f / l;
+        const int b = h / Hs, hs = h - b * Hs;
+        const size_t orow = (size_t)batch_row(b, qi, nb, Lc, L);
 #pragma unroll
-        for (int dd = 0; dd < HD; ++dd) o[(size_t)qi * H * HD + h * HD + dd] = to_act<T>(acc[dd] * inv);
+        for (int dd = 0; dd < HD; ++dd) o[orow * Hs * HD + hs * HD + dd] = to_act<T>(acc[dd] * inv);
     }
 }
 
@@ -390,25 +423,29 @@ static wdc_status gemm(Ctx* c, const void* A, const void* W, int M, int N, int K
     return WDC_OK;
 }
 
+// H heads in all = nb samples x Hs heads; sample b's output rows follow the
+// batch's stream-major token layout (Lc condition tokens per sample).
 static wdc_status attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
-                            cudaStream_t s) {
+                            int Hs, int Lc, cudaStream_t s) {
     LaunchScope ls(c, WDC_K_ATTN, s);
-    if (c->cfg.dtype == WDC_BF16 && tc_attention_supported(L, d)) return tc_attention(c, q, k, vt, o, H, L, d, s);
+    if (c->cfg.dtype == WDC_BF16 && tc_attention_supported(L, d))
+        return tc_attention(c, q, k, vt, o, H, L, d, Hs, Lc, s);
     dim3 grid(blocks_for(L, 128), H);
     const float scale = 1.0f / sqrtf((float)d);
+    const int nb = H / Hs;
     if (c->cfg.dtype == WDC_BF16) {
         using T = __nv_bfloat16;
         using TV = __half;          // V^T is fp16 in the bf16 model (the PV product takes P in fp16)
         if (d == 64)
-            attn_simt_kernel<T, TV, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const TV*)vt, (T*)o, H, L, scale);
+            attn_simt_kernel<T, TV, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const TV*)vt, (T*)o, Hs, nb, Lc, L, scale);
         else
-            attn_simt_kernel<T, TV, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const TV*)vt, (T*)o, H, L, scale);
+            attn_simt_kernel<T, TV, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const TV*)vt, (T*)o, Hs, nb, Lc, L, scale);
     } else {
         using T = float;
         if (d == 64)
-            attn_simt_kernel<T, T, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+            attn_simt_kernel<T, T, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, Hs, nb, Lc, L, scale);
         else
-            attn_simt_kernel<T, T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, H, L, scale);
+            attn_simt_kernel<T, T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, Hs, nb, Lc, L, scale);
     }
     return WDC_OK;
 }
@@ -460,6 +497,7 @@ wdc_status dit_create(Ctx* c) {
     t->L = t->Lc + t->Lv;
     t->Dc = g.cond_dim;
     t->layers = g.layers;
+    t->B = g.max_batch > 1 ? g.max_batch : 1;
     wdc_status s;
     if ((s = alloc_lin(c, t->patch, t->D, t->P))) return s;
     if ((s = alloc_lin(c, t->cond, t->D, t->Dc > 0 ? t->Dc : 1))) return s;
@@ -480,16 +518,17 @@ wdc_status dit_create(Ctx* c) {
         if ((s = alloc_lin(c, t->fc1[i], t->M, t->D))) return s;
         if ((s = alloc_lin(c, t->fc2[i], t->D, t->M))) return s;
     }
-    const size_t LD = (size_t)t->L * t->D * t->esz;
+    const size_t LD = (size_t)t->B * t->L * t->D * t->esz;
     if ((s = dalloc(c, &t->x, LD))) return s;
     if ((s = dalloc(c, &t->h, LD))) return s;
     if ((s = dalloc(c, &t->q, LD))) return s;
     if ((s = dalloc(c, &t->k, LD))) return s;
     if ((s = dalloc(c, &t->vt, LD))) return s;
     if ((s = dalloc(c, &t->ao, LD))) return s;
-    if ((s = dalloc(c, &t->m, (size_t)t->L * t->M * t->esz))) return s;
-    if ((s = dalloc(c, &t->tok, (size_t)t->Lv * t->P * t->esz))) return s;
-    if ((s = dalloc(c, &t->condx, (size_t)(t->Lc > 0 ? t->Lc : 1) * (t->Dc > 0 ? t->Dc : 1) * t->esz))) return s;
+    if ((s = dalloc(c, &t->m, (size_t)t->B * t->L * t->M * t->esz))) return s;
+    if ((s = dalloc(c, &t->tok, (size_t)t->B * t->Lv * t->P * t->esz))) return s;
+    if ((s = dalloc(c, &t->condx, (size_t)t->B * (t->Lc > 0 ? t->Lc : 1) * (t->Dc > 0 ? t->Dc : 1) * t->esz))) return s;
+    if (t->B > 1 && (s = dalloc(c, (void**)&t->vb, (size_t)t->B * c->n * sizeof(float)))) return s;
     if ((s = dalloc(c, &t->pe, (size_t)t->Lv * t->D * t->esz))) return s;
     if ((s = dalloc(c, (void**)&t->feat, (size_t)t->Fd * sizeof(float)))) return s;
     if ((s = dalloc(c, (void**)&t->h1, (size_t)t->E * sizeof(float)))) return s;
@@ -638,15 +677,16 @@ wdc_status dit_modulation(Ctx* c, float t_model, float* mod_out, cudaStream_t s)
     return WDC_OK;
 }
 
-// One block on x (device, [L, D]) with mod (device fp32, [S][6][D]).
-static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, cudaStream_t s) {
+// One block on x (device, [nb*L, D], stream-major batch rows) with mod
+// (device fp32, [S][6][D]).
+static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, int nb, cudaStream_t s) {
     DiT* t = c->dit;
     const int D = t->D;
     const size_t es = t->esz;
-    // stream s rows: s = 0 video [Lc, L), s = 1 cond [0, Lc); single stream: all rows
+    // stream s rows: s = 0 video [nb*Lc, nb*L), s = 1 cond [0, nb*Lc); single stream: all rows
     int r0[2], r1[2];
-    if (t->S == 2) { r0[0] = t->Lc; r1[0] = t->L; r0[1] = 0; r1[1] = t->Lc; }
-    else { r0[0] = 0; r1[0] = t->L; }
+    if (t->S == 2) { r0[0] = nb * t->Lc; r1[0] = nb * t->L; r0[1] = 0; r1[1] = nb * t->Lc; }
+    else { r0[0] = 0; r1[0] = nb * t->L; }
     wdc_status st;
     // per-stream CUDA streams: the condition rows (dual stream) on t->aux,
     // forked before and joined after each half of the block; every buffer
@@ -672,11 +712,11 @@ static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, cudaSt
         const Lin& w = t->qkv[layer * t->S + sidx];
         Epi e{};
         e.mode = kEpiQKV; e.bias = w.b; e.q = t->q; e.k = t->k; e.vt = t->vt;
-        e.L = t->L; e.H = t->H; e.d = t->d; e.D = D; e.row_off = r0[sidx];
+        e.L = t->L; e.H = t->H; e.d = t->d; e.D = D; e.row_off = r0[sidx]; e.nb = nb; e.Lc = t->Lc;
         if ((st = gemm(c, (char*)t->h + (size_t)r0[sidx] * D * es, w.w, r1[sidx] - r0[sidx], 3 * D, D, e, s))) return st;
     }
     if ((st = join(0))) return st;
-    if ((st = attention(c, t->q, t->k, t->vt, t->ao, t->H, t->L, t->d, s))) return st;
+    if ((st = attention(c, t->q, t->k, t->vt, t->ao, nb * t->H, t->L, t->d, t->H, t->Lc, s))) return st;
     if ((st = fork(1))) return st;
     for (int sidx = 0; sidx < t->S; ++sidx) {
         const float* m6 = mod + (size_t)sidx * 6 * D;
@@ -717,56 +757,112 @@ wdc_status dit_block(Ctx* c, int layer, void* x, const float* mod6, cudaStream_t
     if (!c->dit) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
     if (layer < 0 || layer >= c->dit->layers) return fail(c, WDC_ERR_INVALID_ARG, "layer out of range");
     if (!x || !mod6) return fail(c, WDC_ERR_INVALID_ARG, "null pointer");
-    return run_block(c, layer, x, mod6, s);
+    return run_block(c, layer, x, mod6, 1, s);
 }
 
-wdc_status dit_forward(Ctx* c, const float* z, float t_model, const float* cond, float* v, cudaStream_t s) {
+// nb samples at one timestep: z[b] (device fp32 latents), cond[b] (device
+// fp32 condition tokens, null = the all-zero set); velocities into v
+// ([nb, latent], device fp32).
+wdc_status dit_forward_batch(Ctx* c, int nb, const float* const* z, float t_model, const float* const* cond,
+                             float* v, cudaStream_t s) {
     DiT* t = c->dit;
     if (!t) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
-    if (!z || !v || (t->Lc > 0 && !cond)) return fail(c, WDC_ERR_INVALID_ARG, "null pointer");
+    if (nb < 1 || nb > t->B) return fail(c, WDC_ERR_INVALID_ARG, "batch larger than the context's max_batch");
+    if (!z || !v) return fail(c, WDC_ERR_INVALID_ARG, "null pointer");
+    BatchPtrs zp{}, cp{};
+    for (int b = 0; b < nb; ++b) {
+        if (!z[b]) return fail(c, WDC_ERR_INVALID_ARG, "null latent");
+        zp.p[b] = z[b];
+        cp.p[b] = cond ? cond[b] : nullptr;
+    }
     wdc_status st;
     if ((st = dit_modulation(c, t_model, nullptr, s))) return st;
     const int D = t->D;
     const size_t es = t->esz;
     const wdc_dit_config& g = c->cfg;
-    // embed: condition tokens, then patches + position
+    // embed: condition tokens (rows [0, nb*Lc)), then patches + position
+    // (rows [nb*Lc, nb*L))
     if (t->Lc > 0) {
-        const long long nc = (long long)t->Lc * t->Dc;
+        const long long per = (long long)t->Lc * t->Dc;
         {
             LaunchScope ls(c, WDC_K_OTHER, s);
             if (t->dtype == WDC_BF16)
-                convert_kernel<__nv_bfloat16><<<blocks_for(nc, 256), 256, 0, s>>>(cond, (__nv_bfloat16*)t->condx, nc);
+                convert_kernel<__nv_bfloat16><<<blocks_for(per * nb, 256), 256, 0, s>>>(cp, nb, (__nv_bfloat16*)t->condx, per);
             else
-                convert_kernel<float><<<blocks_for(nc, 256), 256, 0, s>>>(cond, (float*)t->condx, nc);
+                convert_kernel<float><<<blocks_for(per * nb, 256), 256, 0, s>>>(cp, nb, (float*)t->condx, per);
         }
         Epi e{};
         e.mode = kEpiStore; e.bias = t->cond.b; e.out = t->x; e.ldo = D;
-        if ((st = gemm(c, t->condx, t->cond.w, t->Lc, D, t->Dc, e, s))) return st;
+        if ((st = gemm(c, t->condx, t->cond.w, nb * t->Lc, D, t->Dc, e, s))) return st;
     }
     {
-        const long long nt = (long long)t->Lv * t->P;
+        const long long nt = (long long)t->Lv * t->P * nb;
         {
             LaunchScope ls(c, WDC_K_OTHER, s);
             if (t->dtype == WDC_BF16)
-                patchify_kernel<__nv_bfloat16><<<blocks_for(nt, 256), 256, 0, s>>>(z, (__nv_bfloat16*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
+                patchify_kernel<__nv_bfloat16><<<blocks_for(nt, 256), 256, 0, s>>>(zp, nb, (__nv_bfloat16*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
             else
-                patchify_kernel<float><<<blocks_for(nt, 256), 256, 0, s>>>(z, (float*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
+                patchify_kernel<float><<<blocks_for(nt, 256), 256, 0, s>>>(zp, nb, (float*)t->tok, g.in_ch, g.frames, g.height, g.width, g.patch);
         }
         Epi e{};
-        char* xv = (char*)t->x + (size_t)t->Lc * D * es;
-        e.mode = kEpiResid; e.bias = t->patch.b; e.out = xv; e.res = t->pe; e.ldo = D; e.gate = nullptr;
-        if ((st = gemm(c, t->tok, t->patch.w, t->Lv, D, t->P, e, s))) return st;
+        char* xv = (char*)t->x + (size_t)nb * t->Lc * D * es;
+        e.mode = kEpiResid; e.bias = t->patch.b; e.out = xv; e.res = t->pe; e.res_rows = t->Lv; e.ldo = D; e.gate = nullptr;
+        if ((st = gemm(c, t->tok, t->patch.w, nb * t->Lv, D, t->P, e, s))) return st;
     }
     for (int l = 0; l < t->layers; ++l)
-        if ((st = run_block(c, l, t->x, t->mods + (size_t)l * t->S * 6 * D, s))) return st;
+        if ((st = run_block(c, l, t->x, t->mods + (size_t)l * t->S * 6 * D, nb, s))) return st;
     // final layer on the video tokens, unpatchified into v (fp32)
     const float* fm = t->mods + (size_t)t->layers * t->S * 6 * D;
-    ln_mod(c, t->x, t->h, t->Lc, t->L, fm, fm + D, t->Lc, s);
+    ln_mod(c, t->x, t->h, nb * t->Lc, nb * t->L, fm, fm + D, nb * t->Lc, s);
     Epi e{};
     e.mode = kEpiUnpatch; e.bias = t->fin.b; e.v = v; e.C = g.in_ch; e.F = g.frames; e.Hh = g.height; e.Ww = g.width; e.p = g.patch;
-    if ((st = gemm(c, t->h, t->fin.w, t->Lv, t->P, D, e, s))) return st;
+    if ((st = gemm(c, t->h, t->fin.w, nb * t->Lv, t->P, D, e, s))) return st;
     cudaError_t ce = cudaGetLastError();
     if (ce != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("forward: ") + cudaGetErrorString(ce));
+    return WDC_OK;
+}
+
+wdc_status dit_forward(Ctx* c, const float* z, float t_model, const float* cond, float* v, cudaStream_t s) {
+    if (!c->dit) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
+    if (!z || !v || (c->dit->Lc > 0 && !cond)) return fail(c, WDC_ERR_INVALID_ARG, "null pointer");
+    return dit_forward_batch(c, 1, &z, t_model, &cond, v, s);
+}
+
+// Batched, optionally guided forward into the callers' velocity buffers
+// (the ABI's wdc_dit_forward_batch): z, cond, v hold B entries; cfg doubles
+// the batch as (conditional, null condition) pairs.
+wdc_status dit_forward_guided(Ctx* c, int B, const float* const* z, float t_model, const float* const* cond, int cfg,
+                              float guidance, float* const* v, cudaStream_t s) {
+    DiT* t = c->dit;
+    if (!t) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
+    const int nb = cfg ? 2 * B : B;
+    if (B < 1 || nb > t->B) return fail(c, WDC_ERR_INVALID_ARG, "batch larger than the context's max_batch");
+    if (!z || !v || (t->Lc > 0 && !cond)) return fail(c, WDC_ERR_INVALID_ARG, "null pointer array");
+    BatchPtrs out{};
+    const float* zz[WDC_MAX_BATCH];
+    const float* cc[WDC_MAX_BATCH];
+    for (int b = 0; b < B; ++b) {
+        if (!z[b] || !v[b] || (t->Lc > 0 && !cond[b])) return fail(c, WDC_ERR_INVALID_ARG, "null pointer");
+        if (((uintptr_t)z[b] | (uintptr_t)v[b]) & 15) return fail(c, WDC_ERR_INVALID_ARG, "latents must be 16-byte aligned");
+        out.p[b] = v[b];
+        const int i = cfg ? 2 * b : b;
+        zz[i] = z[b];
+        cc[i] = t->Lc > 0 ? cond[b] : nullptr;
+        if (cfg) {
+            zz[i + 1] = z[b];
+            cc[i + 1] = nullptr;
+        }
+    }
+    if (nb == 1) return dit_forward_batch(c, 1, zz, t_model, cc, v[0], s);
+    wdc_status st = dit_forward_batch(c, nb, zz, t_model, cc, t->vb, s);
+    if (st) return st;
+    const long long n = (long long)c->n;
+    {
+        LaunchScope ls(c, WDC_K_OTHER, s);
+        guide_kernel<<<blocks_for(n * B, 256), 256, 0, s>>>(t->vb, n, B, cfg, guidance, out);
+    }
+    cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("guidance: ") + cudaGetErrorString(ce));
     return WDC_OK;
 }
 
@@ -787,7 +883,7 @@ wdc_status op_attention(Ctx* c, const void* q, const void* k, const void* vt, vo
                         cudaStream_t s) {
     if (!q || !k || !vt || !o || H <= 0 || L <= 0 || (d != 64 && d != 128))
         return fail(c, WDC_ERR_INVALID_ARG, "bad attention arguments");
-    wdc_status st = attention(c, q, k, vt, o, H, L, d, s);
+    wdc_status st = attention(c, q, k, vt, o, H, L, d, H, 0, s);
     if (st) return st;
     cudaError_t ce = cudaGetLastError();
     if (ce != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("attention: ") + cudaGetErrorString(ce));

@@ -40,6 +40,27 @@ __device__ __forceinline__ float gelu_tanh_f(float x) {
 
 enum EpiMode { kEpiStore = 0, kEpiResid = 1, kEpiQKV = 2, kEpiUnpatch = 3 };
 
+// Token rows of a batch of nb samples (L tokens each, the first Lc of them
+// condition tokens) are laid out stream-major: rows [0, nb*Lc) hold the
+// condition tokens of samples 0..nb-1, rows [nb*Lc, nb*L) their video tokens.
+// Row-wise kernels and the GEMMs see one [nb*L, D] matrix; the dual-stream
+// row blocks stay contiguous.  nb == 1 is the single-sample sequence.
+__host__ __device__ __forceinline__ void batch_token(int row, int nb, int Lc, int L, int& b, int& tok) {
+    if (nb <= 1) { b = 0; tok = row; return; }
+    const int cond_rows = nb * Lc;
+    if (row < cond_rows) {
+        b = row / Lc;
+        tok = row - b * Lc;
+    } else {
+        const int j = row - cond_rows, Lv = L - Lc;
+        b = j / Lv;
+        tok = Lc + (j - b * Lv);
+    }
+}
+__host__ __device__ __forceinline__ int batch_row(int b, int tok, int nb, int Lc, int L) {
+    return tok < Lc ? b * Lc + tok : nb * Lc + b * (L - Lc) + (tok - Lc);
+}
+
 // Epilogue of C = A W^T on one output element (row m of this GEMM, column n).
 struct Epi {
     int mode;
@@ -49,10 +70,13 @@ struct Epi {
     int ldo;
     const void* res;          // kEpiResid: [M, ldo] (may equal out)
     const float* gate;        // kEpiResid: [N] or null (= 1)
-    // kEpiQKV: q, k [H, L, d], vt [H, d, L]; token = row_off + m
+    int res_rows;             // kEpiResid: > 0 reads residual row m % res_rows
+    // kEpiQKV: q, k [nb*H, L, d], vt [nb*H, d, L]; (sample, token) of batch
+    // row row_off + m (batch_token); head of sample b = b*H + h
     void* q; void* k; void* vt;
-    int L, H, d, D, row_off;
-    // kEpiUnpatch: v fp32 [C, F, Hh, Ww]; token m = (f, h', w'), column = (c, ph, pw)
+    int L, H, d, D, row_off, nb, Lc;
+    // kEpiUnpatch: v fp32 [nb][C, F, Hh, Ww]; row m = (sample, f, h', w'),
+    // column = (c, ph, pw)
     float* v;
     int C, F, Hh, Ww, p;
 };
@@ -67,29 +91,34 @@ __device__ __forceinline__ void epi_apply(const Epi& e, int m, int n, float acc)
             break;
         case kEpiResid: {
             const size_t idx = (size_t)m * e.ldo + n;
-            const float r = ld_act<T>(reinterpret_cast<const T*>(e.res) + idx);
+            const size_t ridx = (size_t)(e.res_rows > 0 ? m % e.res_rows : m) * e.ldo + n;
+            const float r = ld_act<T>(reinterpret_cast<const T*>(e.res) + ridx);
             const float g = e.gate ? e.gate[n] : 1.0f;
             reinterpret_cast<T*>(e.out)[idx] = to_act<T>(fmaf(g, x, r));
             break;
         }
         case kEpiQKV: {
-            const int which = n / e.D, c = n % e.D, h = c / e.d, dd = c % e.d;
-            const int tok = e.row_off + m;
+            const int which = n / e.D, c = n % e.D, dd = c % e.d;
+            int b, tok;
+            batch_token(e.row_off + m, e.nb, e.Lc, e.L, b, tok);
+            const size_t h = (size_t)b * e.H + c / e.d;
             if (which == 0)
-                reinterpret_cast<T*>(e.q)[((size_t)h * e.L + tok) * e.d + dd] = to_act<T>(x);
+                reinterpret_cast<T*>(e.q)[(h * e.L + tok) * e.d + dd] = to_act<T>(x);
             else if (which == 1)
-                reinterpret_cast<T*>(e.k)[((size_t)h * e.L + tok) * e.d + dd] = to_act<T>(x);
+                reinterpret_cast<T*>(e.k)[(h * e.L + tok) * e.d + dd] = to_act<T>(x);
             else if constexpr (sizeof(T) == 2)
-                reinterpret_cast<__half*>(e.vt)[((size_t)h * e.d + dd) * e.L + tok] = to_vt_half(x);
+                reinterpret_cast<__half*>(e.vt)[(h * e.d + dd) * e.L + tok] = to_vt_half(x);
             else
-                reinterpret_cast<T*>(e.vt)[((size_t)h * e.d + dd) * e.L + tok] = to_act<T>(x);
+                reinterpret_cast<T*>(e.vt)[(h * e.d + dd) * e.L + tok] = to_act<T>(x);
             break;
         }
         case kEpiUnpatch: {
-            const int hp = e.Hh / e.p, wp = e.Ww / e.p;
-            const int f = m / (hp * wp), rem = m % (hp * wp), h2 = rem / wp, w2 = rem % wp;
+            const int hp = e.Hh / e.p, wp = e.Ww / e.p, Lv = e.F * hp * wp;
+            const int b = m / Lv, mm = m - b * Lv;
+            const int f = mm / (hp * wp), rem = mm % (hp * wp), h2 = rem / wp, w2 = rem % wp;
             const int c = n / (e.p * e.p), r2 = n % (e.p * e.p), ph = r2 / e.p, pw = r2 % e.p;
-            e.v[(((size_t)c * e.F + f) * e.Hh + h2 * e.p + ph) * e.Ww + w2 * e.p + pw] = x;
+            e.v[(size_t)b * e.C * e.F * e.Hh * e.Ww +
+                (((size_t)c * e.F + f) * e.Hh + h2 * e.p + ph) * e.Ww + w2 * e.p + pw] = x;
             break;
         }
     }

@@ -81,8 +81,9 @@ __device__ __forceinline__ void epilogue_chunk(const Epi& e, int m, int col0, co
         __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(e.out) + (size_t)m * e.ldo + col0;
         uint4* o4 = reinterpret_cast<uint4*>(out);
         if (e.mode == kEpiResid) {
+            const int rm = e.res_rows > 0 ? m % e.res_rows : m;
             const uint4* r4 = reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(e.res) +
-                                                             (size_t)m * e.ldo + col0);
+                                                             (size_t)rm * e.ldo + col0);
             float g[32];
             if (e.gate) {
                 const float4* g4 = reinterpret_cast<const float4*>(e.gate + col0);
@@ -120,11 +121,13 @@ __device__ __forceinline__ void epilogue_chunk(const Epi& e, int m, int col0, co
         return;
     }
     if (e.mode == kEpiQKV) {
-        const int which = col0 / e.D, c = col0 % e.D, h = c / e.d, dd0 = c % e.d;
-        const int tok = e.row_off + m;
+        const int which = col0 / e.D, c = col0 % e.D, dd0 = c % e.d;
+        int b, tok;
+        batch_token(e.row_off + m, e.nb, e.Lc, e.L, b, tok);
+        const size_t h = (size_t)b * e.H + c / e.d;
         if (which < 2) {
             __nv_bfloat16* base = reinterpret_cast<__nv_bfloat16*>(which == 0 ? e.q : e.k) +
-                                  ((size_t)h * e.L + tok) * e.d + dd0;
+                                  (h * e.L + tok) * e.d + dd0;
             uint4* o4 = reinterpret_cast<uint4*>(base);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -136,7 +139,7 @@ __device__ __forceinline__ void epilogue_chunk(const Epi& e, int m, int col0, co
                 o4[q] = w;
             }
         } else {
-            __half* base = reinterpret_cast<__half*>(e.vt) + ((size_t)h * e.d + dd0) * e.L + tok;
+            __half* base = reinterpret_cast<__half*>(e.vt) + (h * e.d + dd0) * e.L + tok;
 #pragma unroll
             for (int j = 0; j < 32; ++j) base[(size_t)j * e.L] = to_vt_half(v[j]);
         }

@@ -192,6 +192,10 @@ void dit_destroy(Ctx* c);
 wdc_status dit_set_tensor(Ctx* c, int id, int layer, int stream, const float* host, size_t count);
 wdc_status dit_init_weights(Ctx* c, unsigned long long seed, float std);
 wdc_status dit_forward(Ctx* c, const float* z, float t, const float* cond, float* v, cudaStream_t s);
+// B latents at one timestep through one batched forward; cfg doubles the
+// batch with null-condition twins and writes the guided velocity.
+wdc_status dit_forward_guided(Ctx* c, int B, const float* const* z, float t, const float* const* cond, int cfg,
+                              float guidance, float* const* v, cudaStream_t s);
 void dit_set_timestep_source(Ctx* c, const float* t_src);   // null: the t argument of dit_forward
 wdc_status dit_block(Ctx* c, int layer, void* x, const float* mod6, cudaStream_t s);
 wdc_status dit_modulation(Ctx* c, float t, float* mod_out, cudaStream_t s);

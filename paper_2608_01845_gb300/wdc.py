@@ -12,6 +12,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libwdc.so")
 
 MAX_BANK = 8
+MAX_BATCH = 16
 SUMMARY_DIM = 256
 SKETCH = 120
 F32, BF16 = 0, 1
@@ -41,7 +42,7 @@ class WdcError(RuntimeError):
 class DitConfig(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in
                 ["layers", "hidden", "heads", "head_dim", "mlp", "temb_dim", "freq_dim", "in_ch", "frames",
-                 "height", "width", "patch", "cond_tokens", "cond_dim", "dual_stream", "dtype"]]
+                 "height", "width", "patch", "cond_tokens", "cond_dim", "dual_stream", "dtype", "max_batch"]]
 
 
 class Schedule(ctypes.Structure):
@@ -127,6 +128,7 @@ def _load():
         "wdc_set_tensor": (I, [P, I, I, I, P, S]),
         "wdc_init_weights": (I, [P, ctypes.c_ulonglong, F]),
         "wdc_dit_forward": (I, [P, P, F, P, P, P]),
+        "wdc_dit_forward_batch": (I, [P, I, ctypes.POINTER(P), F, ctypes.POINTER(P), I, F, ctypes.POINTER(P), P]),
         "wdc_dit_block_forward": (I, [P, I, P, P, P]),
         "wdc_dit_modulation": (I, [P, F, P, P]),
         "wdc_scheduler_step": (I, [P, I, P, P, P, P]),
@@ -137,6 +139,8 @@ def _load():
         "wdc_risk_update": (I, [P, I, ctypes.POINTER(Cond), P, P, P, ctypes.POINTER(P), ctypes.POINTER(StepInfo), P]),
         "wdc_rollout": (I, [P, P, ctypes.POINTER(Cond), I, P, ctypes.POINTER(I), ctypes.POINTER(StepInfo), P]),
         "wdc_rollout_graph": (I, [P, P, ctypes.POINTER(Cond), P, ctypes.POINTER(I), ctypes.POINTER(StepInfo), P]),
+        "wdc_rollout_batch": (I, [ctypes.POINTER(P), I, ctypes.POINTER(P), ctypes.POINTER(Cond), I, I, F,
+                                  ctypes.POINTER(P), ctypes.POINTER(I), ctypes.POINTER(StepInfo), P]),
         "wdc_native_rollout": (I, [P, P, ctypes.POINTER(Cond), I, P, P]),
         "wdc_op_gemm": (I, [P, P, P, P, P, I, I, I, I, P, P, P]),
         "wdc_op_attention": (I, [P, P, P, P, P, I, I, I, P]),
@@ -168,9 +172,9 @@ def make_params(**overrides):
 
 
 def make_config(layers=0, hidden=0, heads=0, head_dim=0, mlp=0, temb_dim=0, freq_dim=256, in_ch=1, frames=1,
-                height=1, width=1, patch=1, cond_tokens=0, cond_dim=0, dual_stream=0, dtype=F32):
+                height=1, width=1, patch=1, cond_tokens=0, cond_dim=0, dual_stream=0, dtype=F32, max_batch=1):
     return DitConfig(layers, hidden, heads, head_dim, mlp, temb_dim, freq_dim, in_ch, frames, height, width, patch,
-                     cond_tokens, cond_dim, dual_stream, dtype)
+                     cond_tokens, cond_dim, dual_stream, dtype, max_batch)
 
 
 def _ptr(t):
@@ -280,6 +284,17 @@ class Context:
         self._check(LIB.wdc_dit_forward(self._h, _ptr(z_t), float(t), _ptr(cond_tokens), _ptr(v), _stream(stream)),
                     "dit_forward")
 
+    def dit_forward_batch(self, z_list, t, cond_list, v_list, cfg=False, guidance=1.0, stream=None):
+        """wdc_dit_forward_batch: one batched (optionally guided) forward of
+        len(z_list) latents at timestep t; cond_list may be None when the
+        model has no condition tokens."""
+        B = len(z_list)
+        zs = (ctypes.c_void_p * B)(*[t_.data_ptr() for t_ in z_list])
+        vs = (ctypes.c_void_p * B)(*[t_.data_ptr() for t_ in v_list])
+        cs = None if cond_list is None else (ctypes.c_void_p * B)(*[t_.data_ptr() for t_ in cond_list])
+        self._check(LIB.wdc_dit_forward_batch(self._h, B, zs, float(t), cs, int(bool(cfg)), float(guidance), vs,
+                                              _stream(stream)), "dit_forward_batch")
+
     def dit_block_forward(self, layer, x, mod6, stream=None):
         self._check(LIB.wdc_dit_block_forward(self._h, layer, _ptr(x), _ptr(mod6), _stream(stream)),
                     "dit_block_forward")
@@ -353,6 +368,32 @@ class Context:
         H, L, d = q.shape
         self._check(LIB.wdc_op_attention(self._h, _ptr(q), _ptr(k), _ptr(vt), _ptr(o), H, L, d, _stream(stream)),
                     "op_attention")
+
+
+def rollout_batch(ctxs, z_T_list, conds, z_out_list, cfg=False, guidance=1.0, trace=True, stream=None):
+    """wdc_rollout_batch: len(ctxs) cached rollouts in lockstep; ctxs[0] owns
+    the denoiser, ctxs[b] holds sample b's cache state.  conds: one wdc_cond
+    per sample (used for every step) or a list of T per sample.  Returns
+    (decisions per sample, traces per sample or None)."""
+    B = len(ctxs)
+    T = ctxs[0].sched.T
+    per = [c if isinstance(c, (list, tuple)) else [c] for c in conds]
+    n_cond = len(per[0])
+    flat = [c for p in per for c in p]
+    carr = (Cond * len(flat))(*flat)
+    hs = (ctypes.c_void_p * B)(*[c._h.value for c in ctxs])
+    zs = (ctypes.c_void_p * B)(*[t.data_ptr() for t in z_T_list])
+    outs = (ctypes.c_void_p * B)(*[t.data_ptr() for t in z_out_list])
+    dec = (ctypes.c_int * (B * T))()
+    tr = (StepInfo * (B * T))() if trace else None
+    st = LIB.wdc_rollout_batch(hs, B, zs, carr, n_cond, int(bool(cfg)), float(guidance), outs, dec, tr,
+                               _stream(stream))
+    if st != 0:
+        msgs = [LIB.wdc_last_error(c._h).decode() for c in ctxs]
+        raise WdcError(st, "rollout_batch: " + " | ".join(f"sample {b}: {m}" for b, m in enumerate(msgs) if m))
+    decs = [list(dec[b * T:(b + 1) * T]) for b in range(B)]
+    traces = [[tr[b * T + k].as_dict() for k in range(T)] for b in range(B)] if trace else None
+    return decs, traces
 
 
 def observe_noalloc(z_out, kappa, z_a, z_hat, stats, sketch_seed=0x2545F491, stream=None):

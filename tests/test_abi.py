@@ -4,6 +4,8 @@ import ctypes
 import os
 import re
 
+import pytest
+
 from paper_2608_01845_gb300 import wdc
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -53,22 +55,30 @@ def test_ablation_flags_and_defaults_match_the_header():
     assert p.period == 8 and p.ridge == 1e-6
 
 
-def test_cache_params_layout_matches_a_c_compiler(tmp_path):
+@pytest.mark.parametrize("cname,pystruct", [("wdc_cache_params", "CacheParams"), ("wdc_dit_config", "DitConfig"),
+                                             ("wdc_schedule", "Schedule"), ("wdc_cond", "Cond"),
+                                             ("wdc_step_info", "StepInfo")])
+def test_struct_layout_matches_a_c_compiler(tmp_path, cname, pystruct):
     import shutil
     import subprocess
     cc = shutil.which("gcc") or shutil.which("cc")
     if cc is None:
-        import pytest
         pytest.skip("no C compiler")
-    fields = [f for f, _ in wdc.CacheParams._fields_]
+    st = getattr(wdc, pystruct)
+    fields = [f for f, _ in st._fields_]
     prog = tmp_path / "layout.c"
     prog.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "wdc.h"\nint main(void) {\n'
-                    '  printf("%zu\\n", sizeof(wdc_cache_params));\n'
-                    + "".join(f'  printf("%zu\\n", offsetof(wdc_cache_params, {f}));\n' for f in fields)
+                    f'  printf("%zu\\n", sizeof({cname}));\n'
+                    + "".join(f'  printf("%zu\\n", offsetof({cname}, {f}));\n' for f in fields)
                     + "  return 0;\n}\n")
     exe = tmp_path / "layout"
     subprocess.run([cc, "-I", os.path.join(ROOT, "include"), "-I", "/usr/local/cuda/include", str(prog), "-o", str(exe)],
                    check=True)
     out = [int(x) for x in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()]
-    assert out[0] == ctypes.sizeof(wdc.CacheParams)
-    assert out[1:] == [getattr(wdc.CacheParams, f).offset for f in fields]
+    assert out[0] == ctypes.sizeof(st)
+    assert out[1:] == [getattr(st, f).offset for f in fields]
+
+
+def test_batch_limit_matches_the_header():
+    src = open(os.path.join(ROOT, "include", "wdc.h")).read()
+    assert int(re.search(r"#define WDC_MAX_BATCH\s+(\d+)", src).group(1)) == wdc.MAX_BATCH
