@@ -342,6 +342,24 @@ ABLATIONS = {
 }
 
 
+def max_over_ranks(x, world, device):
+    """The slowest rank's figure: every rank contributes its own time, the
+    job's time is the maximum (one all-reduce; nothing else crosses ranks)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_steps_per_s(world, T, rollouts, seconds):
+    """Whole-job throughput of replicas: each of `world` ranks rolls out
+    `rollouts` independent T-step rollouts in `seconds` (the max over ranks)."""
+    return world * T * rollouts / seconds
+
+
 def run_gpu(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -386,12 +404,8 @@ def run_gpu(args, rank, world, local_rank):
     prof = ctx.profile_read()
     ctx.profile_enable(False)
     launches = ctx.launches - launches0
-    ms = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * T * args.steps / (ms * 1e-3)
+    ms = max_over_ranks(e0.elapsed_time(e1), world, "cuda")
+    value = job_steps_per_s(world, T, args.steps, ms * 1e-3)
     exact = [T - sum(d) for d in all_dec]
 
     # ---- dominant kernel of the timed region and its roofline
@@ -437,12 +451,8 @@ def run_gpu(args, rank, world, local_rank):
     for _ in range(args.steps):
         ctx.rollout(zT_h, cond_h, out_h, trace=False)
     torch.cuda.synchronize()
-    et = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([et], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        et = float(t.item())
-    line["e2e"] = {"value": world * T * args.steps / et, "unit": UNIT,
+    et = max_over_ranks(time.perf_counter() - t0, world, "cuda")
+    line["e2e"] = {"value": job_steps_per_s(world, T, args.steps, et), "unit": UNIT,
                    "h2d_bytes_per_step": zT.nbytes + ct.nbytes, "d2h_bytes_per_step": zT.nbytes}
 
     # device-side control flow on the same workload (graph built by a first call)
