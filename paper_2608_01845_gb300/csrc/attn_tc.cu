@@ -139,7 +139,9 @@ __device__ __forceinline__ float half2_sum(uint32_t v) {
 }
 
 
-template <int D>
+// BATCH: heads of several samples, output rows through the batch's
+// stream-major token layout; otherwise row = token, head = h (one sample).
+template <int D, bool BATCH>
 __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
                    const __grid_constant__ CUtensorMap tv, const __grid_constant__ AttnArgs g) {
@@ -454,8 +456,13 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                 if (tok < g.L) {
                     // head h = (sample, head within the sample); O row of
                     // (sample, token) in the batch's stream-major token rows
-                    const int b = h / g.Hs, hs = h - b * g.Hs;
-                    const size_t orow = (size_t)batch_row(b, tok, g.nb, g.Lc, g.L);
+                    size_t orow = (size_t)tok;
+                    int hs = h;
+                    if constexpr (BATCH) {
+                        const int b = h / g.Hs;
+                        hs = h - b * g.Hs;
+                        orow = (size_t)batch_row(b, tok, g.nb, g.Lc, g.L);
+                    }
                     uint4* dst = reinterpret_cast<uint4*>(g.o + orow * g.Hs * D + (size_t)hs * D + c);
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
@@ -478,18 +485,18 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     }
 }
 
-template <int D>
+template <int D, bool BATCH>
 wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int Hs, int Lc,
                   cudaStream_t s) {
     using Cf = AttnCfg<D>;
     static bool attr = false;
     static bool regs_ok = false;
     if (!attr) {
-        cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cf::SMEM);
+        cudaFuncSetAttribute(attn_tc_kernel<D, BATCH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cf::SMEM);
         // the warpgroups' register requests must fit the launch allocation,
         // or setmaxnreg.inc would wait forever: refuse to launch otherwise
         cudaFuncAttributes fa;
-        regs_ok = cudaFuncGetAttributes(&fa, attn_tc_kernel<D>) == cudaSuccess &&
+        regs_ok = cudaFuncGetAttributes(&fa, attn_tc_kernel<D, BATCH>) == cudaSuccess &&
                   fa.maxThreadsPerBlock >= Cf::THREADS &&
                   (uint32_t)fa.numRegs * Cf::THREADS >= 128 * Cf::REGS_CONTROL + 256 * Cf::REGS_SOFTMAX;
         cudaGetLastError();
@@ -514,7 +521,7 @@ wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o,
     g.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
     g.o = reinterpret_cast<__nv_bfloat16*>(o);
     g.err = c->err;
-    attn_tc_kernel<D><<<H * g.q_blocks, Cf::THREADS, Cf::SMEM, s>>>(tq, tk, tv, g);
+    attn_tc_kernel<D, BATCH><<<H * g.q_blocks, Cf::THREADS, Cf::SMEM, s>>>(tq, tk, tv, g);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 attention launch: ") + cudaGetErrorString(e));
     return WDC_OK;
@@ -529,7 +536,10 @@ wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, vo
     if (((uintptr_t)q | (uintptr_t)k | (uintptr_t)vt | (uintptr_t)o) & 15)
         return fail(c, WDC_ERR_INVALID_ARG, "attention operands must be 16-byte aligned");
     if (Hs <= 0 || H % Hs || Lc < 0 || Lc >= L) return fail(c, WDC_ERR_INVALID_ARG, "bad attention batch layout");
-    return d == 64 ? launch<64>(c, q, k, vt, o, H, L, Hs, Lc, s) : launch<128>(c, q, k, vt, o, H, L, Hs, Lc, s);
+    if (Hs == H)
+        return d == 64 ? launch<64, false>(c, q, k, vt, o, H, L, Hs, Lc, s)
+                       : launch<128, false>(c, q, k, vt, o, H, L, Hs, Lc, s);
+    return d == 64 ? launch<64, true>(c, q, k, vt, o, H, L, Hs, Lc, s) : launch<128, true>(c, q, k, vt, o, H, L, Hs, Lc, s);
 }
 
 }  // namespace wdc
