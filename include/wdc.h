@@ -255,6 +255,12 @@ wdc_status wdc_selftest_wait_timeout(wdc_ctx* ctx, unsigned long long limit_ns, 
  * round-to-nearest-even).  layer/stream are ignored for global tensors. */
 wdc_status wdc_set_tensor(wdc_ctx* ctx, int tensor_id, int layer, int stream,
                           const float* host, size_t count);
+/* Reads one parameter tensor back into `host` (fp32, `count` elements, the
+ * wdc_set_tensor layout); bf16 values are widened exactly.  Synchronous.  Lets
+ * a checker evaluate the model the device actually holds (e.g. after
+ * wdc_init_weights).  WDC_ERR_INVALID_ARG on a size mismatch or bad id. */
+wdc_status wdc_get_tensor(wdc_ctx* ctx, int tensor_id, int layer, int stream,
+                          float* host, size_t count);
 /* Initialises every matrix N(0, std^2) and every bias to 0 on the device from
  * a counter-based Philox4x32-10 stream (Salmon et al., SC'11) keyed by seed. */
 wdc_status wdc_init_weights(wdc_ctx* ctx, unsigned long long seed, float std);

@@ -462,6 +462,13 @@ wdc_status wdc_set_tensor(wdc_ctx* h, int tensor_id, int layer, int stream, cons
     return dit_set_tensor(c, tensor_id, layer, stream, host, count);
 }
 
+wdc_status wdc_get_tensor(wdc_ctx* h, int tensor_id, int layer, int stream, float* host, size_t count) {
+    Ctx* c = reinterpret_cast<Ctx*>(h);
+    if (!c) return WDC_ERR_INVALID_ARG;
+    cudaSetDevice(c->device);
+    return dit_get_tensor(c, tensor_id, layer, stream, host, count);
+}
+
 wdc_status wdc_init_weights(wdc_ctx* h, unsigned long long seed, float std) {
     Ctx* c = reinterpret_cast<Ctx*>(h);
     if (!c) return WDC_ERR_INVALID_ARG;

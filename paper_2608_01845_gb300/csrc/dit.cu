@@ -584,16 +584,23 @@ static wdc_status upload(Ctx* c, void* dst, const float* host, size_t count, boo
     return WDC_OK;
 }
 
-wdc_status dit_set_tensor(Ctx* c, int id, int layer, int stream, const float* host, size_t count) {
+// Device location of parameter tensor `id`: pointer, element count and
+// whether it is stored in the model dtype (matrices) or fp32 (biases).
+struct TensorLoc {
+    void* p = nullptr;
+    size_t count = 0;
+    bool model_dtype = false;
+};
+
+static wdc_status locate_tensor(Ctx* c, int id, int layer, int stream, TensorLoc& loc) {
     DiT* t = c->dit;
     if (!t) return fail(c, WDC_ERR_UNSUPPORTED, "context has no denoiser (layers == 0)");
-    if (!host) return fail(c, WDC_ERR_INVALID_ARG, "null host pointer");
     const bool per_layer = id >= WDC_T_MOD_W;
     if (per_layer && (layer < 0 || layer >= t->layers || stream < 0 || stream >= t->S))
         return fail(c, WDC_ERR_INVALID_ARG, "layer/stream out of range");
     const int li = layer * t->S + stream;
     Lin* lin = nullptr;
-    bool bias = (id % 2) == 1;
+    const bool bias = (id % 2) == 1;
     switch (id) {
         case WDC_T_PATCH_W: case WDC_T_PATCH_B: lin = &t->patch; break;
         case WDC_T_COND_W: case WDC_T_COND_B: lin = &t->cond; break;
@@ -605,24 +612,59 @@ wdc_status dit_set_tensor(Ctx* c, int id, int layer, int stream, const float* ho
         case WDC_T_FC1_W: case WDC_T_FC1_B: lin = &t->fc1[li]; break;
         case WDC_T_FC2_W: case WDC_T_FC2_B: lin = &t->fc2[li]; break;
         case WDC_T_MOD_W: case WDC_T_MOD_B: case WDC_T_FMOD_W: case WDC_T_FMOD_B: {
-            const size_t row0 = (id == WDC_T_MOD_W || id == WDC_T_MOD_B) ? (size_t)li * 6 * t->D
-                                                                         : (size_t)t->layers * t->S * 6 * t->D;
-            const size_t rows = (id == WDC_T_MOD_W || id == WDC_T_MOD_B) ? 6 * (size_t)t->D : 2 * (size_t)t->D;
+            const bool blk = id == WDC_T_MOD_W || id == WDC_T_MOD_B;
+            const size_t row0 = blk ? (size_t)li * 6 * t->D : (size_t)t->layers * t->S * 6 * t->D;
+            const size_t rows = blk ? 6 * (size_t)t->D : 2 * (size_t)t->D;
             if (bias) {
-                if (count != rows) return fail(c, WDC_ERR_INVALID_ARG, "modulation bias size mismatch");
-                return upload(c, t->modB + row0, host, count, false);
+                loc.p = t->modB + row0;
+                loc.count = rows;
+            } else {
+                loc.p = (char*)t->modW + row0 * t->E * t->esz;
+                loc.count = rows * t->E;
+                loc.model_dtype = true;
             }
-            if (count != rows * t->E) return fail(c, WDC_ERR_INVALID_ARG, "modulation weight size mismatch");
-            return upload(c, (char*)t->modW + row0 * t->E * t->esz, host, count, true);
+            return WDC_OK;
         }
         default: return fail(c, WDC_ERR_INVALID_ARG, "unknown tensor id");
     }
     if (bias) {
-        if (count != (size_t)lin->out) return fail(c, WDC_ERR_INVALID_ARG, "bias size mismatch");
-        return upload(c, lin->b, host, count, false);
+        loc.p = lin->b;
+        loc.count = (size_t)lin->out;
+    } else {
+        loc.p = lin->w;
+        loc.count = (size_t)lin->out * lin->in;
+        loc.model_dtype = true;
     }
-    if (count != (size_t)lin->out * lin->in) return fail(c, WDC_ERR_INVALID_ARG, "weight size mismatch");
-    return upload(c, lin->w, host, count, true);
+    return WDC_OK;
+}
+
+wdc_status dit_set_tensor(Ctx* c, int id, int layer, int stream, const float* host, size_t count) {
+    if (c->dit && !host) return fail(c, WDC_ERR_INVALID_ARG, "null host pointer");
+    TensorLoc loc;
+    wdc_status st = locate_tensor(c, id, layer, stream, loc);
+    if (st) return st;
+    if (count != loc.count) return fail(c, WDC_ERR_INVALID_ARG, "tensor size mismatch");
+    return upload(c, loc.p, host, count, loc.model_dtype);
+}
+
+// Reads a parameter back to host fp32 (bf16 values widen exactly).
+wdc_status dit_get_tensor(Ctx* c, int id, int layer, int stream, float* host, size_t count) {
+    if (c->dit && !host) return fail(c, WDC_ERR_INVALID_ARG, "null host pointer");
+    TensorLoc loc;
+    wdc_status st = locate_tensor(c, id, layer, stream, loc);
+    if (st) return st;
+    if (count != loc.count) return fail(c, WDC_ERR_INVALID_ARG, "tensor size mismatch");
+    if (!loc.model_dtype || c->dit->dtype == WDC_F32) {
+        WDC_CUDA_TRY(c, cudaMemcpy(host, loc.p, count * sizeof(float), cudaMemcpyDeviceToHost));
+        return WDC_OK;
+    }
+    std::vector<uint16_t> tmp(count);
+    WDC_CUDA_TRY(c, cudaMemcpy(tmp.data(), loc.p, count * 2, cudaMemcpyDeviceToHost));
+    for (size_t i = 0; i < count; ++i) {
+        const uint32_t u = (uint32_t)tmp[i] << 16;
+        std::memcpy(&host[i], &u, 4);
+    }
+    return WDC_OK;
 }
 
 static void init_normal(Ctx* c, void* dst, size_t n, unsigned long long seed, uint32_t sid, float std) {

@@ -190,6 +190,7 @@ ParamsDev to_dev_params(const wdc_cache_params& p);
 wdc_status dit_create(Ctx* c);
 void dit_destroy(Ctx* c);
 wdc_status dit_set_tensor(Ctx* c, int id, int layer, int stream, const float* host, size_t count);
+wdc_status dit_get_tensor(Ctx* c, int id, int layer, int stream, float* host, size_t count);
 wdc_status dit_init_weights(Ctx* c, unsigned long long seed, float std);
 wdc_status dit_forward(Ctx* c, const float* z, float t, const float* cond, float* v, cudaStream_t s);
 // B latents at one timestep through one batched forward; cfg doubles the

@@ -126,6 +126,7 @@ def _load():
         "wdc_latent_numel": (S, [P]),
         "wdc_launch_count": (ctypes.c_ulonglong, [P]),
         "wdc_set_tensor": (I, [P, I, I, I, P, S]),
+        "wdc_get_tensor": (I, [P, I, I, I, P, S]),
         "wdc_init_weights": (I, [P, ctypes.c_ulonglong, F]),
         "wdc_dit_forward": (I, [P, P, F, P, P, P]),
         "wdc_dit_forward_batch": (I, [P, I, ctypes.POINTER(P), F, ctypes.POINTER(P), I, F, ctypes.POINTER(P), P]),
@@ -267,6 +268,24 @@ class Context:
         import numpy as np
         a = np.ascontiguousarray(array, dtype=np.float32)
         self._check(LIB.wdc_set_tensor(self._h, tensor_id, layer, stream, a.ctypes.data, a.size), "set_tensor")
+
+    def get_tensor(self, tensor_id, shape, layer=0, stream=0):
+        """wdc_get_tensor: one parameter tensor back as a float32 array."""
+        import numpy as np
+        a = np.empty(shape, dtype=np.float32)
+        self._check(LIB.wdc_get_tensor(self._h, tensor_id, layer, stream, a.ctypes.data, a.size), "get_tensor")
+        return a
+
+    def get_weights(self, shapes):
+        """{name: shape} (names as in set_weights) -> {name: float32 array} read from the device."""
+        out = {}
+        for name, shape in shapes.items():
+            if name in GLOBAL_TENSORS:
+                out[name] = self.get_tensor(GLOBAL_TENSORS[name], shape)
+            else:
+                lay, strm, rest = name.split(".", 2)
+                out[name] = self.get_tensor(LAYER_TENSORS[rest], shape, layer=int(lay[1:]), stream=int(strm[1:]))
+        return out
 
     def set_weights(self, weights):
         """Uploads a {name: array} dict (names as produced by the seeded generators)."""

@@ -15,7 +15,10 @@ guidance).
 * wdc_rollout_batch on the bf16 model equals each sample's wdc_rollout alone,
   bitwise.
 * Argument errors: batch above max_batch, a context shared by two samples,
-  contexts of different latent size."""
+  contexts of different latent size.
+* The largest batch (16 forwards, and 8 guided pairs) on the bf16 model.
+* Per-step conditions (n_cond = T) and pinned host latents in a batched
+  rollout, against each sample's single rollout."""
 import numpy as np
 import pytest
 import torch
@@ -197,3 +200,60 @@ def test_batch_argument_errors(parity):
     ctx.dit_forward_batch(z[:2], 500.0, c[:2], v[:2])
     torch.cuda.synchronize()
     assert torch.equal(v[0], v[1])
+
+
+def test_batched_forward_at_max_batch_bf16():
+    W = synth.dit_weights(PARITY_MODEL, 9, std=0.02, bias_std=0.02, bf16=True)
+    ctx = _ctx(PARITY_MODEL, wdc.BF16, wdc.MAX_BATCH, W)
+    B = wdc.MAX_BATCH
+    zs = [_dev(synth.latent(100 + b, SHAPE)) for b in range(B)]
+    cts = [_dev(synth.cond_tokens(200 + b, 16, 256, bf16=True)) for b in range(B)]
+    vs = [torch.empty(N, device="cuda") for _ in range(B)]
+    ctx.dit_forward_batch(zs, 420.0, cts, vs)
+    for b in (0, 7, B - 1):
+        ref = torch.empty(N, device="cuda")
+        ctx.dit_forward(zs[b], 420.0, cts[b], ref)
+        torch.cuda.synchronize()
+        assert torch.equal(vs[b], ref), b
+    # a guided batch of 8 pairs fills the same 16 slots
+    gv = [torch.empty(N, device="cuda") for _ in range(B // 2)]
+    ctx.dit_forward_batch(zs[:B // 2], 420.0, cts[:B // 2], gv, cfg=True, guidance=3.0)
+    torch.cuda.synchronize()
+    zero = torch.zeros(16, 256, device="cuda")
+    for b in (0, B // 2 - 1):
+        vc, vu = torch.empty(N, device="cuda"), torch.empty(N, device="cuda")
+        ctx.dit_forward(zs[b], 420.0, cts[b], vc)
+        ctx.dit_forward(zs[b], 420.0, zero, vu)
+        torch.cuda.synchronize()
+        assert torch.allclose(gv[b], vu + 3.0 * (vc - vu), rtol=1e-6, atol=1e-6), b
+    assert ctx.device_errors() == 0
+
+
+def test_rollout_batch_per_step_conditions_and_host_latents(parity):
+    W, cfg, zs, cts, _ = parity
+    B = 2
+    descs = [synth.cond_descriptors(300 + b, T, static=False) for b in range(B)]
+    ct_d = [_dev(c) for c in cts[:B]]
+    conds = [[wdc.make_cond(ct_d[b], d["cam"], d["depth"]) for d in descs[b]] for b in range(B)]
+    taus = [0.5, 0.3]
+    ctxs = [_ctx(PARITY_MODEL, wdc.F32, B, W, params=wdc.make_params(tau_risk=taus[0]))]
+    ctxs.append(wdc.Context(wdc.make_config(in_ch=16, frames=4, height=16, width=16), T,
+                            params=wdc.make_params(tau_risk=taus[1])))
+    outs = [torch.empty(N, device="cuda") for _ in range(B)]
+    decs, tr = wdc.rollout_batch(ctxs, [_dev(z) for z in zs[:B]], conds, outs)
+    # host (pinned) latents in and out give the same result
+    zh = [torch.from_numpy(np.ascontiguousarray(z, dtype=np.float32).ravel()).pin_memory() for z in zs[:B]]
+    oh = [torch.empty(N).pin_memory() for _ in range(B)]
+    decs_h, _ = wdc.rollout_batch(ctxs, zh, conds, oh)
+    assert decs_h == decs
+    for b in range(B):
+        assert torch.equal(oh[b], outs[b].cpu())
+    # each sample alone, with its per-step conditions
+    single = _ctx(PARITY_MODEL, wdc.F32, 1, W)
+    for b in range(B):
+        single.set_cache_params(wdc.make_params(tau_risk=taus[b]))
+        out = torch.empty(N, device="cuda")
+        dec, trs = single.rollout(_dev(zs[b]), conds[b], out)
+        assert dec == decs[b]
+        assert torch.equal(out, outs[b])
+        assert [t["d_hat"] for t in trs] == [t["d_hat"] for t in tr[b]]

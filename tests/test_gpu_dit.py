@@ -154,6 +154,46 @@ def test_bf16_block_5b_scale_sampled_rows():
     assert rel_l2(got, want) <= BF16_TOL
 
 
+def test_bench_model_forward_5b_sampled_tokens():
+    """The bench's 5B-shape model as the device builds it -- wdc_init_weights
+    with the bench's seed (the global tensors and layer 0 draw the same
+    Philox streams in a 1-layer context as in the 42-layer one) -- run through
+    one full forward (modulation, embeddings, one block in the bench's launch
+    configuration, final layer, unpatchify) on the bench's synthetic inputs at
+    the first step's timestep, and checked on 64 sampled video tokens (64
+    latent entries each) against the oracle evaluated on the weights read back
+    from the device."""
+    import bench
+    w = dict(bench.WORKLOADS["5b"], layers=1)
+    keys = ["layers", "hidden", "heads", "head_dim", "mlp", "temb_dim", "freq_dim", "in_ch", "frames", "height",
+            "width", "patch", "cond_tokens", "cond_dim", "dual_stream"]
+    cfgd = {k: w[k] for k in keys}
+    cfg = DiTConfig(**cfgd)
+    ctx = _ctx(cfgd, wdc.BF16, T=w["T"])
+    ctx.init_weights(w["weight_seed"], 0.02)
+    W = ctx.get_weights(dit.param_shapes(cfg))
+    for name in ["L0.s0.qkv.w", "L0.s0.fc2.w", "patch.w"]:          # N(0, 0.02^2), biases 0
+        a = W[name]
+        assert abs(a.std() - 0.02) < 5e-4 and abs(a.mean()) < 5e-4, name
+    assert not W["L0.s0.qkv.b"].any()
+    zT, ct, _ = bench.inputs(w, 0)
+    C, F, H, Wd, p = cfg.in_ch, cfg.frames, cfg.height, cfg.width, cfg.patch
+    t = 1000.0                                                       # sigma_0 = 1
+    v = torch.empty(zT.size, dtype=torch.float32, device="cuda")
+    ctx.dit_forward(_to_dev(zT), t, _to_dev(ct), v)
+    torch.cuda.synchronize()
+    assert ctx.device_errors() == 0
+    Lc = cfg.cond_tokens
+    toks = np.sort(np.random.default_rng(35).choice(cfg.video_tokens, 64, replace=False))
+    _, mods, fmod = dit.conditioning(W, cfg, t)
+    x0 = dit.embed(W, cfg, zT, ct)
+    xr = dit.block_rows(x0, W, cfg, 0, [mods[(0, 0)]], Lc + toks)
+    hr = dit.modulate(dit.layer_norm(xr), fmod[0], fmod[1])
+    want = dit.linear(hr, W["final.w"], W["final.b"])               # [64 tokens, C*p*p]
+    got = dit.patchify(v.cpu().numpy().reshape(C, F, H, Wd), p)[toks]
+    assert rel_l2(got, want) <= BF16_TOL
+
+
 BLOCK13B = dict(layers=1, hidden=3072, heads=24, head_dim=128, mlp=12288, temb_dim=512, freq_dim=256, in_ch=16,
                 frames=13, height=64, width=64, patch=2, cond_tokens=256, cond_dim=3072, dual_stream=1)
 
