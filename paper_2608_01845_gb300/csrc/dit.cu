@@ -131,11 +131,21 @@ __global__ void ln_mod_kernel(const T* __restrict__ x, T* __restrict__ h, int r0
 }
 
 // bf16 variant with 16-byte accesses: lane l owns the 8-element vectors
-// l, l+32, ..., so a warp moves 512 contiguous bytes per access (D % 256 == 0).
+// l, l+32, ..., so a warp moves 512 contiguous bytes per access (D = 256 NV).
+// The block stages (1 + scale) and shift in shared memory once for its rows
+// instead of every row reading them from L2.
 template <int NV>
 __global__ void ln_mod_vec_kernel(const __nv_bfloat16* __restrict__ x, __nv_bfloat16* __restrict__ h, int r0, int r1,
                                   int D, const float* __restrict__ shift, const float* __restrict__ scale,
                                   int h_row_off) {
+    __shared__ float4 s_sc[NV * 64], s_sh[NV * 64];        // 256 NV floats each
+    for (int i = threadIdx.x; i < NV * 64; i += blockDim.x) {
+        float4 a = __ldg(reinterpret_cast<const float4*>(scale) + i);
+        a.x += 1.0f; a.y += 1.0f; a.z += 1.0f; a.w += 1.0f;
+        s_sc[i] = a;
+        s_sh[i] = __ldg(reinterpret_cast<const float4*>(shift) + i);
+    }
+    __syncthreads();
     const int row = r0 + ((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
     if (row >= r1) return;
     const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)row * D);
@@ -170,18 +180,16 @@ __global__ void ln_mod_vec_kernel(const __nv_bfloat16* __restrict__ x, __nv_bflo
     uint4* hr = reinterpret_cast<uint4*>(h + (size_t)(row - h_row_off) * D);
 #pragma unroll
     for (int i = 0; i < NV; ++i) {
-        const int c0 = (i * 32 + lane) * 8;
-        const float4 sc0 = __ldg(reinterpret_cast<const float4*>(scale + c0));
-        const float4 sc1 = __ldg(reinterpret_cast<const float4*>(scale + c0 + 4));
-        const float4 sh0 = __ldg(reinterpret_cast<const float4*>(shift + c0));
-        const float4 sh1 = __ldg(reinterpret_cast<const float4*>(shift + c0 + 4));
+        const int c4 = (i * 32 + lane) * 2;                   // float4 index of column (i*32+lane)*8
+        const float4 sc0 = s_sc[c4], sc1 = s_sc[c4 + 1];
+        const float4 sh0 = s_sh[c4], sh1 = s_sh[c4 + 1];
         const float sc[8] = {sc0.x, sc0.y, sc0.z, sc0.w, sc1.x, sc1.y, sc1.z, sc1.w};
         const float sh[8] = {sh0.x, sh0.y, sh0.z, sh0.w, sh1.x, sh1.y, sh1.z, sh1.w};
         uint32_t w[4];
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-            const float a = fmaf((v[i][2 * q] - mean) * rstd, 1.0f + sc[2 * q], sh[2 * q]);
-            const float b = fmaf((v[i][2 * q + 1] - mean) * rstd, 1.0f + sc[2 * q + 1], sh[2 * q + 1]);
+            const float a = fmaf((v[i][2 * q] - mean) * rstd, sc[2 * q], sh[2 * q]);
+            const float b = fmaf((v[i][2 * q + 1] - mean) * rstd, sc[2 * q + 1], sh[2 * q + 1]);
             __nv_bfloat162 hb = __floats2bfloat162_rn(a, b);
             w[q] = *reinterpret_cast<uint32_t*>(&hb);
         }
