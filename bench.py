@@ -417,7 +417,7 @@ def run_gpu(args, rank, world, local_rank):
         avg_ms = prof["attention"][0] / prof["attention"][1]
         achieved = block_flops(w)[1] / (avg_ms * 1e-3) / 1e12
         kfile = os.path.join(ROOT, "paper_2608_01845_gb300", "csrc", "attn_tc.cu")
-        kname = f"attn_tc_kernel<{w['head_dim']}> ({w['heads']} heads x {tokens(w)} tokens x {w['head_dim']})"
+        kname = f"attn_tc_kernel<{w['head_dim']}, false> ({w['heads']} heads x {tokens(w)} tokens x {w['head_dim']})"
         traffic = traffic_for(kfile, args.workload)
     else:
         avg_ms = prof["gemm"][0] / prof["gemm"][1]
