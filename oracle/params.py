@@ -28,7 +28,7 @@ OBS_RESIDUAL = 0x100
 class CacheParams:
     # Memory and retrieval (Eq. 3-5, section "Local Lifted Evolution").
     bank_capacity: int = 4        # FIFO capacity K of the exact-transition bank
-    min_support: int = 1          # |N_t| needed for "adequate retrieval support"
+    min_support: int = 1          # |N_t| that counts as enough retrieval support (Eq. 10 text)
     sim_min: float = 0.0          # compatibility: sim(s(phi_t), s(phi_in)) >= sim_min
     q_gap_max: float = 0.25       # compatibility: |q_t - q_in| <= q_gap_max
     gamma_q: float = 10.0         # phase penalty in the retrieval score (Eq. 3)
@@ -55,7 +55,7 @@ class CacheParams:
     a_phase: float = 1.0
     lam: float = 0.9
     tau_risk: float = 0.5
-    max_age: int = 6              # "pre-decision age at most six" (Eq. 10 text)
+    max_age: int = 6              # largest pre-decision anchor age that allows a candidate (Eq. 10 text)
     n_init_exact: int = 1         # mandatory-exact initialisation steps
     n_final_exact: int = 0        # mandatory-exact refinement steps at the end
     # Ablation variants (Tables 3 and 4).
