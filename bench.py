@@ -254,13 +254,12 @@ def traffic_for(kernel_file, workload):
     return e.get("dram_bytes_per_launch")
 
 
-def skip_pass_gbps(torch, wdc, peaks, secant=False):
-    """Fused skip pass alone at 2^28 fp32 elements, bank of 4 (reads 4 N,
-    writes N), L2 flushed by a 512 MB write before every launch.  With
-    ``secant`` the native-latent-secant ablation's pass instead (reads z_t,
-    the stored displacement and z_a, writes N)."""
+def skip_pass_gbps(torch, wdc, peaks, secant=False, n=SKIP_SWEEP_N):
+    """Fused skip pass alone at n fp32 elements (2^28 by default), bank of 4
+    (reads 4 N, writes N), L2 flushed by a 512 MB write before every launch.
+    With ``secant`` the native-latent-secant ablation's pass instead (reads
+    z_t, the stored displacement and z_a, writes N)."""
     import numpy as np
-    n = SKIP_SWEEP_N
     flags = wdc.ABL_SECANT if secant else 0
     ctx = wdc.Context(wdc.make_config(layers=0, width=n), 50,
                       params=wdc.make_params(bank_capacity=4, sim_min=-1.0, flags=flags))
@@ -586,7 +585,7 @@ def run_op(args):
         print(json.dumps({"op": "gemms", "workload": args.workload, **out}))
         return
     else:
-        r = skip_pass_gbps(torch, wdc, peaks, secant=args.op == "secant")
+        r = skip_pass_gbps(torch, wdc, peaks, secant=args.op == "secant", n=args.n)
         print(json.dumps({"op": args.op, **r}))
         return
     for _ in range(2):
@@ -666,6 +665,7 @@ def main():
                     help="time one operator at its 5B-scale shape (profiler captures); batch: the batched "
                          "cached rollout against one-at-a-time rollouts")
     ap.add_argument("--batch", type=int, default=2, help="--op batch: samples per batch")
+    ap.add_argument("--n", type=int, default=SKIP_SWEEP_N, help="--op skip / secant: latent elements")
     ap.add_argument("--cfg", action="store_true", help="--op batch: classifier-free guidance on every exact step")
     ap.add_argument("--guidance", type=float, default=5.0, help="--op batch: guidance scale with --cfg")
     ap.add_argument("--reps", type=int, default=3)
