@@ -420,6 +420,12 @@ def run_gpu(args, rank, world, local_rank):
         traffic = traffic_for(kfile, args.workload)
     else:
         avg_ms = prof["gemm"][0] / prof["gemm"][1]
+        if w["dual_stream"]:
+            # the condition rows' block GEMMs run on the forked stream, untimed:
+            # the timed GEMM work is the video rows' blocks plus the embeddings
+            Lv = tokens(w) - w["cond_tokens"]
+            g_all, _ = block_flops(w)
+            fwd_gemm -= w["layers"] * g_all * (1.0 - Lv / tokens(w))
         achieved = n_fwd * fwd_gemm / (prof["gemm"][0] * 1e-3) / 1e12
         kfile = os.path.join(ROOT, "paper_2608_01845_gb300", "csrc", "gemm_tc.cu")
         kname = "gemm_tc2_kernel / gemm_tc_kernel (all denoiser GEMMs)"

@@ -545,6 +545,7 @@ wdc_status dit_create(Ctx* c) {
     if (t->S == 2) {
         if (cudaStreamCreateWithFlags(&t->aux, cudaStreamNonBlocking) != cudaSuccess)
             return fail(c, WDC_ERR_CUDA, "DiT init: auxiliary stream");
+        c->untimed_stream = t->aux;
         for (int i = 0; i < 2; ++i)
             if (cudaEventCreateWithFlags(&t->fork[i], cudaEventDisableTiming) != cudaSuccess ||
                 cudaEventCreateWithFlags(&t->join[i], cudaEventDisableTiming) != cudaSuccess)
@@ -569,6 +570,7 @@ void dit_destroy(Ctx* c) {
         if (c->dit->join[i]) cudaEventDestroy(c->dit->join[i]);
     }
     if (c->dit->aux) cudaStreamDestroy(c->dit->aux);
+    c->untimed_stream = nullptr;
     delete c->dit;
     c->dit = nullptr;
 }

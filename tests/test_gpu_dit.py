@@ -265,3 +265,29 @@ def test_bf16_gemm_sampled_full_size_and_no_device_errors(M, N, K):
     want = A[rows].astype(np.float64) @ W.astype(np.float64).T
     assert rel_l2(C.float().cpu().numpy()[rows], want) <= 1e-2
     assert ctx.device_errors() == 0
+
+
+def test_profiler_times_main_stream_launches_only():
+    """The event profiler times the main stream's launches; the condition
+    rows' kernels of a dual-stream model (forked stream, overlapping the timed
+    ones) count in the total launch number but are not timed."""
+    cfgd = dict(PARITY_MODEL, layers=1, dual_stream=1)
+    ctx = _ctx(cfgd, wdc.BF16)
+    ctx.init_weights(3, 0.02)
+    z = _to_dev(synth.latent(3, (16, 4, 16, 16)))
+    ct = _to_dev(synth.cond_tokens(4, 16, 256))
+    v = torch.empty(z.numel(), dtype=torch.float32, device="cuda")
+    ctx.dit_forward(z, 500.0, ct, v)
+    torch.cuda.synchronize()
+    n0 = ctx.launches
+    ctx.profile_enable(True)
+    ctx.dit_forward(z, 500.0, ct, v)
+    prof = ctx.profile_read()
+    ctx.profile_enable(False)
+    # main stream: condition and patch embeddings, the video rows' 4 block GEMMs, the final GEMM
+    assert prof["gemm"][1] == 7
+    assert prof["attention"][1] == 1
+    assert prof["norm"][1] == 3                    # the video rows' two LayerNorms + the final one
+    # the forked stream adds the condition rows' 4 GEMMs and 2 LayerNorms
+    assert ctx.launches - n0 == sum(n for _, n in prof.values()) + 6
+    assert all(ms > 0 for ms, n in prof.values() if n)
