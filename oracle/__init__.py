@@ -22,6 +22,12 @@ Modules (each function cites the passage it follows):
 * ``rollout``   -- the exact-transition bank and the cached / native rollouts
                    (section "Inference and Complexity").
 * ``dit``       -- the adaLN DiT denoiser F_theta used as the exact branch.
+* ``ablation``  -- the ablation variants of Tables 3 and 4 (section
+                   "Ablation Study"), as switches of the steps above.
+* ``diagnostics`` -- the synthetic transition diagnostics of Fig. 2 and
+                   Fig. 3a.
+* ``batch``     -- batched and guided rollouts (serving extensions: a batch of
+                   independent trajectories; classifier-free guidance).
 
 Parity status: the controller constants and the lift's normalisation details
 are not printed in the paper (it defers them to supplementary material that is
