@@ -422,15 +422,20 @@ wdc_status wdc_profile_read(wdc_ctx* ctx, double* ms, unsigned long long* launch
 /* C = epilogue(A W^T): A [M, K], W [N, K] (model dtype, device, row-major);
  * bias [N] fp32 or NULL; gelu != 0 applies GELU_tanh; when res != NULL
  * C = res + gate * (.) with gate [N] fp32 (NULL = 1) and res/C [M, N] in the
- * model dtype (res may equal C). */
+ * model dtype (res may equal C).  A bf16 model runs every GEMM on the tcgen05
+ * kernel, which needs N % 32 == 0 and K % 8 == 0: other shapes return
+ * WDC_ERR_UNSUPPORTED (the fp32 parity mode takes any shape). */
 wdc_status wdc_op_gemm(wdc_ctx* ctx, const void* A, const void* W, const float* bias, void* C,
                        int M, int N, int K, int gelu, const void* res, const float* gate,
                        wdc_stream stream);
 /* O = softmax(Q K^T / sqrt(d)) V per head, non-causal: q, k [heads, L, d],
- * vt [heads, d, L] (V transposed), o [L, heads*d]; device memory.  q, k and
- * o are in the model dtype; vt is fp32 for an fp32 model and fp16 for a bf16
- * model (the QKV projection stores V that way so that the PV product takes
- * the probabilities in fp16). */
+ * vt [heads, d, ldv] (V transposed, row stride ldv), o [L, heads*d]; device
+ * memory, 16-byte aligned.  q, k and o are in the model dtype; vt is fp32
+ * for an fp32 model (ldv = L) and fp16 for a bf16 model (the QKV projection
+ * stores V that way so that the PV product takes the probabilities in fp16),
+ * with ldv = L rounded up to a multiple of 8 so that every V^T row starts on
+ * a 16-byte boundary; the padding columns are never read.  Any L >= 1; d 64
+ * or 128. */
 wdc_status wdc_op_attention(wdc_ctx* ctx, const void* q, const void* k, const void* vt, void* o,
                             int heads, int L, int d, wdc_stream stream);
 
@@ -447,8 +452,12 @@ wdc_status wdc_op_attention(wdc_ctx* ctx, const void* q, const void* k, const vo
  * file-scope __device__ array that every GPU loading libwdc.so holds until the
  * process exits.  The first call on a device, with that device current, looks
  * up the array's device address (cudaGetSymbolAddress) and caches it; make that
- * first call before any stream capture.  Each call clears the counter on
- * `stream` before its kernel.  All calls on a device share the scratch, so
+ * first call before any stream capture.  The cached address belongs to the
+ * device's primary context as it was at that first call: after a
+ * cudaDeviceReset (or anything else that destroys and re-creates the primary
+ * context) restart the process before calling this entry point again.  Each
+ * call clears the counter on `stream` before its kernel.  All calls on a
+ * device share the scratch, so
  * calls that overlap on the GPU (different streams, no ordering) race; order
  * them on one stream.
  *

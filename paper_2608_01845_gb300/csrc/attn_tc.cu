@@ -486,8 +486,8 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
 }
 
 template <int D, bool BATCH>
-wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int Hs, int Lc,
-                  cudaStream_t s) {
+wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, int ldv, void* o, int H, int L, int Hs,
+                  int Lc, cudaStream_t s) {
     using Cf = AttnCfg<D>;
     static bool attr = false;
     static bool regs_ok = false;
@@ -508,7 +508,7 @@ wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o,
     const uint64_t row = (uint64_t)D * 2, head = (uint64_t)L * D * 2;
     if (!encode_tmap_3d(&tq, q, D, L, H, row, head, 64, BQ, 1, &why) ||
         !encode_tmap_3d(&tk, k, D, L, H, row, head, 64, BKV, 1, &why) ||
-        !encode_tmap_3d(&tv, vt, L, D, H, (uint64_t)L * 2, (uint64_t)L * D * 2, 64, D, 1, &why, true))
+        !encode_tmap_3d(&tv, vt, L, D, H, (uint64_t)ldv * 2, (uint64_t)ldv * D * 2, 64, D, 1, &why, true))
         return fail(c, WDC_ERR_CUDA, why);
     AttnArgs g;
     g.H = H;
@@ -529,17 +529,21 @@ wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, void* o,
 
 }  // namespace
 
-bool tc_attention_supported(int L, int d) { return L > 0 && L % 8 == 0 && (d == 64 || d == 128); }
+// Any L: V^T rows are padded to ldv (a multiple of 8 tokens, so every TMA row
+// starts on a 16-byte boundary); keys past L are zero-filled by TMA and masked.
+bool tc_attention_supported(int L, int d) { return L > 0 && (d == 64 || d == 128); }
 
-wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
+wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, int ldv, void* o, int H, int L, int d,
                         int Hs, int Lc, cudaStream_t s) {
     if (((uintptr_t)q | (uintptr_t)k | (uintptr_t)vt | (uintptr_t)o) & 15)
         return fail(c, WDC_ERR_INVALID_ARG, "attention operands must be 16-byte aligned");
+    if (ldv < L || ldv % 8) return fail(c, WDC_ERR_INVALID_ARG, "V^T row stride must be >= L and a multiple of 8");
     if (Hs <= 0 || H % Hs || Lc < 0 || Lc >= L) return fail(c, WDC_ERR_INVALID_ARG, "bad attention batch layout");
     if (Hs == H)
-        return d == 64 ? launch<64, false>(c, q, k, vt, o, H, L, Hs, Lc, s)
-                       : launch<128, false>(c, q, k, vt, o, H, L, Hs, Lc, s);
-    return d == 64 ? launch<64, true>(c, q, k, vt, o, H, L, Hs, Lc, s) : launch<128, true>(c, q, k, vt, o, H, L, Hs, Lc, s);
+        return d == 64 ? launch<64, false>(c, q, k, vt, ldv, o, H, L, Hs, Lc, s)
+                       : launch<128, false>(c, q, k, vt, ldv, o, H, L, Hs, Lc, s);
+    return d == 64 ? launch<64, true>(c, q, k, vt, ldv, o, H, L, Hs, Lc, s)
+                   : launch<128, true>(c, q, k, vt, ldv, o, H, L, Hs, Lc, s);
 }
 
 }  // namespace wdc

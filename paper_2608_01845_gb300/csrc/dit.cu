@@ -26,7 +26,7 @@ namespace wdc {
 bool tc_gemm_supported(int M, int N, int K);
 wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, const Epi& e, cudaStream_t s);
 bool tc_attention_supported(int L, int d);
-wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
+wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, int ldv, void* o, int H, int L, int d,
                         int Hs, int Lc, cudaStream_t s);
 
 struct Lin {
@@ -40,6 +40,7 @@ struct DiT {
     size_t esz = 4;
     int S = 1;                            // weight streams (2 with dual_stream)
     int D = 0, H = 0, d = 0, M = 0, E = 0, Fd = 0, P = 0, Lc = 0, Lv = 0, L = 0, Dc = 0, layers = 0;
+    int ldv = 0;                          // V^T row stride: L, rounded up to 8 tokens in bf16 (16-byte TMA rows)
     int B = 1;                            // most samples one forward holds (activation buffers sized for it)
     Lin patch, cond, t1, t2, fin;
     void* modW = nullptr;                 // [(layers*S*6 + 2) * D, E]
@@ -340,8 +341,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
 // One thread per query row, online softmax over key tiles staged in shared memory.
 template <typename T, typename TV, int HD>
 __global__ void __launch_bounds__(128) attn_simt_kernel(const T* __restrict__ q, const T* __restrict__ k,
-                                                         const TV* __restrict__ vt, T* __restrict__ o, int Hs, int nb,
-                                                         int Lc, int L, float scale) {
+                                                         const TV* __restrict__ vt, int ldv, T* __restrict__ o, int Hs,
+                                                         int nb, int Lc, int L, float scale) {
     constexpr int KT = HD <= 64 ? 64 : 32;
     __shared__ float Ks[KT][HD + 1];
     __shared__ float Vs[KT][HD + 1];
@@ -359,7 +360,7 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const T* __restrict__ q,
             const int jj = i / HD, dd = i % HD;
             Ks[jj][dd] = (j0 + jj < L) ? ld_act<T>(k + ((size_t)h * L + j0 + jj) * HD + dd) : 0.f;
             const int dv = i / KT, jv = i % KT;
-            Vs[jv][dv] = (j0 + jv < L) ? ld_act<TV>(vt + ((size_t)h * HD + dv) * L + j0 + jv) : 0.f;
+            Vs[jv][dv] = (j0 + jv < L) ? ld_act<TV>(vt + ((size_t)h * HD + dv) * ldv + j0 + jv) : 0.f;
         }
         __syncthreads();
         const int nk = min(KT, L - j0);
@@ -417,44 +418,45 @@ void launch_ln_mod(const void* x, void* h, int r0, int r1, int D, const float* s
 }  // namespace
 
 // ---------------------------------------------------------------- dispatch
+// bf16 runs on the tcgen05 kernels only: a shape outside their limits is an
+// error, not a silent SIMT run.  The SIMT kernels serve the fp32 parity mode.
 static wdc_status gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, const Epi& e, cudaStream_t s) {
     if (M <= 0 || N <= 0) return WDC_OK;
+    if (c->cfg.dtype == WDC_BF16) {
+        if (!tc_gemm_supported(M, N, K))
+            return fail(c, WDC_ERR_UNSUPPORTED, "bf16 GEMM " + std::to_string(M) + "x" + std::to_string(N) + "x" +
+                                                    std::to_string(K) + ": the tcgen05 GEMM needs N % 32 == 0 and K % 8 == 0");
+        LaunchScope ls(c, WDC_K_GEMM, s);
+        return tc_gemm(c, A, W, M, N, K, e, s);
+    }
     LaunchScope ls(c, WDC_K_GEMM, s);
-    if (c->cfg.dtype == WDC_BF16 && tc_gemm_supported(M, N, K)) return tc_gemm(c, A, W, M, N, K, e, s);
     dim3 grid(blocks_for(N, 64), blocks_for(M, 64));
-    if (c->cfg.dtype == WDC_BF16)
-        gemm_simt_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(reinterpret_cast<const __nv_bfloat16*>(A),
-                                                             reinterpret_cast<const __nv_bfloat16*>(W), M, N, K, e);
-    else
-        gemm_simt_kernel<float><<<grid, 256, 0, s>>>(reinterpret_cast<const float*>(A),
-                                                     reinterpret_cast<const float*>(W), M, N, K, e);
+    gemm_simt_kernel<float><<<grid, 256, 0, s>>>(reinterpret_cast<const float*>(A),
+                                                 reinterpret_cast<const float*>(W), M, N, K, e);
     return WDC_OK;
 }
 
 // H heads in all = nb samples x Hs heads; sample b's output rows follow the
 // batch's stream-major token layout (Lc condition tokens per sample).
-static wdc_status attention(Ctx* c, const void* q, const void* k, const void* vt, void* o, int H, int L, int d,
-                            int Hs, int Lc, cudaStream_t s) {
+// V^T rows have stride ldv (>= L).  bf16 runs on the tcgen05 kernel only;
+// the SIMT kernel serves the fp32 parity mode.
+static wdc_status attention(Ctx* c, const void* q, const void* k, const void* vt, int ldv, void* o, int H, int L,
+                            int d, int Hs, int Lc, cudaStream_t s) {
+    if (c->cfg.dtype == WDC_BF16) {
+        if (!tc_attention_supported(L, d))
+            return fail(c, WDC_ERR_UNSUPPORTED, "bf16 attention needs head_dim 64 or 128 and L > 0");
+        LaunchScope ls(c, WDC_K_ATTN, s);
+        return tc_attention(c, q, k, vt, ldv, o, H, L, d, Hs, Lc, s);
+    }
     LaunchScope ls(c, WDC_K_ATTN, s);
-    if (c->cfg.dtype == WDC_BF16 && tc_attention_supported(L, d))
-        return tc_attention(c, q, k, vt, o, H, L, d, Hs, Lc, s);
     dim3 grid(blocks_for(L, 128), H);
     const float scale = 1.0f / sqrtf((float)d);
     const int nb = H / Hs;
-    if (c->cfg.dtype == WDC_BF16) {
-        using T = __nv_bfloat16;
-        using TV = __half;          // V^T is fp16 in the bf16 model (the PV product takes P in fp16)
-        if (d == 64)
-            attn_simt_kernel<T, TV, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const TV*)vt, (T*)o, Hs, nb, Lc, L, scale);
-        else
-            attn_simt_kernel<T, TV, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const TV*)vt, (T*)o, Hs, nb, Lc, L, scale);
-    } else {
-        using T = float;
-        if (d == 64)
-            attn_simt_kernel<T, T, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, Hs, nb, Lc, L, scale);
-        else
-            attn_simt_kernel<T, T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, (T*)o, Hs, nb, Lc, L, scale);
-    }
+    using T = float;
+    if (d == 64)
+        attn_simt_kernel<T, T, 64><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, ldv, (T*)o, Hs, nb, Lc, L, scale);
+    else
+        attn_simt_kernel<T, T, 128><<<grid, 128, 0, s>>>((const T*)q, (const T*)k, (const T*)vt, ldv, (T*)o, Hs, nb, Lc, L, scale);
     return WDC_OK;
 }
 
@@ -503,6 +505,7 @@ wdc_status dit_create(Ctx* c) {
     t->Lc = g.cond_tokens;
     t->Lv = g.frames * (g.height / g.patch) * (g.width / g.patch);
     t->L = t->Lc + t->Lv;
+    t->ldv = t->dtype == WDC_BF16 ? (t->L + 7) / 8 * 8 : t->L;
     t->Dc = g.cond_dim;
     t->layers = g.layers;
     t->B = g.max_batch > 1 ? g.max_batch : 1;
@@ -531,7 +534,7 @@ wdc_status dit_create(Ctx* c) {
     if ((s = dalloc(c, &t->h, LD))) return s;
     if ((s = dalloc(c, &t->q, LD))) return s;
     if ((s = dalloc(c, &t->k, LD))) return s;
-    if ((s = dalloc(c, &t->vt, LD))) return s;
+    if ((s = dalloc(c, &t->vt, (size_t)t->B * t->ldv * t->D * t->esz))) return s;
     if ((s = dalloc(c, &t->ao, LD))) return s;
     if ((s = dalloc(c, &t->m, (size_t)t->B * t->L * t->M * t->esz))) return s;
     if ((s = dalloc(c, &t->tok, (size_t)t->B * t->Lv * t->P * t->esz))) return s;
@@ -764,11 +767,11 @@ static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, int nb
         const Lin& w = t->qkv[layer * t->S + sidx];
         Epi e{};
         e.mode = kEpiQKV; e.bias = w.b; e.q = t->q; e.k = t->k; e.vt = t->vt;
-        e.L = t->L; e.H = t->H; e.d = t->d; e.D = D; e.row_off = r0[sidx]; e.nb = nb; e.Lc = t->Lc;
+        e.L = t->L; e.H = t->H; e.d = t->d; e.D = D; e.row_off = r0[sidx]; e.nb = nb; e.Lc = t->Lc; e.ldv = t->ldv;
         if ((st = gemm(c, (char*)t->h + (size_t)r0[sidx] * D * es, w.w, r1[sidx] - r0[sidx], 3 * D, D, e, s))) return st;
     }
     if ((st = join(0))) return st;
-    if ((st = attention(c, t->q, t->k, t->vt, t->ao, nb * t->H, t->L, t->d, t->H, t->Lc, s))) return st;
+    if ((st = attention(c, t->q, t->k, t->vt, t->ldv, t->ao, nb * t->H, t->L, t->d, t->H, t->Lc, s))) return st;
     if ((st = fork(1))) return st;
     for (int sidx = 0; sidx < t->S; ++sidx) {
         const float* m6 = mod + (size_t)sidx * 6 * D;
@@ -935,7 +938,8 @@ wdc_status op_attention(Ctx* c, const void* q, const void* k, const void* vt, vo
                         cudaStream_t s) {
     if (!q || !k || !vt || !o || H <= 0 || L <= 0 || (d != 64 && d != 128))
         return fail(c, WDC_ERR_INVALID_ARG, "bad attention arguments");
-    wdc_status st = attention(c, q, k, vt, o, H, L, d, H, 0, s);
+    const int ldv = c->cfg.dtype == WDC_BF16 ? (L + 7) / 8 * 8 : L;
+    wdc_status st = attention(c, q, k, vt, ldv, o, H, L, d, H, 0, s);
     if (st) return st;
     cudaError_t ce = cudaGetLastError();
     if (ce != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("attention: ") + cudaGetErrorString(ce));

@@ -71,10 +71,11 @@ struct Epi {
     const void* res;          // kEpiResid: [M, ldo] (may equal out)
     const float* gate;        // kEpiResid: [N] or null (= 1)
     int res_rows;             // kEpiResid: > 0 reads residual row m % res_rows
-    // kEpiQKV: q, k [nb*H, L, d], vt [nb*H, d, L]; (sample, token) of batch
-    // row row_off + m (batch_token); head of sample b = b*H + h
+    // kEpiQKV: q, k [nb*H, L, d], vt [nb*H, d, ldv] (ldv >= L: the V^T row
+    // stride); (sample, token) of batch row row_off + m (batch_token); head
+    // of sample b = b*H + h
     void* q; void* k; void* vt;
-    int L, H, d, D, row_off, nb, Lc;
+    int L, H, d, D, row_off, nb, Lc, ldv;
     // kEpiUnpatch: v fp32 [nb][C, F, Hh, Ww]; row m = (sample, f, h', w'),
     // column = (c, ph, pw)
     float* v;
@@ -107,9 +108,9 @@ __device__ __forceinline__ void epi_apply(const Epi& e, int m, int n, float acc)
             else if (which == 1)
                 reinterpret_cast<T*>(e.k)[(h * e.L + tok) * e.d + dd] = to_act<T>(x);
             else if constexpr (sizeof(T) == 2)
-                reinterpret_cast<__half*>(e.vt)[(h * e.d + dd) * e.L + tok] = to_vt_half(x);
+                reinterpret_cast<__half*>(e.vt)[(h * e.d + dd) * e.ldv + tok] = to_vt_half(x);
             else
-                reinterpret_cast<T*>(e.vt)[(h * e.d + dd) * e.L + tok] = to_act<T>(x);
+                reinterpret_cast<T*>(e.vt)[(h * e.d + dd) * e.ldv + tok] = to_act<T>(x);
             break;
         }
         case kEpiUnpatch: {

@@ -139,9 +139,9 @@ __device__ __forceinline__ void epilogue_chunk(const Epi& e, int m, int col0, co
                 o4[q] = w;
             }
         } else {
-            __half* base = reinterpret_cast<__half*>(e.vt) + (h * e.d + dd0) * e.L + tok;
+            __half* base = reinterpret_cast<__half*>(e.vt) + (h * e.d + dd0) * e.ldv + tok;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) base[(size_t)j * e.L] = to_vt_half(v[j]);
+            for (int j = 0; j < 32; ++j) base[(size_t)j * e.ldv] = to_vt_half(v[j]);
         }
         return;
     }

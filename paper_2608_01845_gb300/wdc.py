@@ -418,8 +418,29 @@ def rollout_batch(ctxs, z_T_list, conds, z_out_list, cfg=False, guidance=1.0, tr
 def observe_noalloc(z_out, kappa, z_a, z_hat, stats, sketch_seed=0x2545F491, stream=None):
     """wdc_observe_noalloc: z_hat = sum_i kappa_i z_out_i plus the next lift's
     statistics (stats: device float64 tensor of 123 values), with no device
-    allocation inside the call (see include/wdc.h)."""
+    allocation inside the call (see include/wdc.h).
+
+    The entry point has no context that knows the latent size, so the sizes of
+    the tensors given here are its only guard: each is checked (dtype, element
+    count, contiguity, device) before the call, and a mismatch raises
+    ValueError."""
+    import torch
     K = len(z_out)
+    if len(kappa) != K:
+        raise ValueError(f"observe_noalloc: {len(kappa)} weights for {K} latents")
+    if not (1 <= K <= MAX_BANK):
+        raise ValueError(f"observe_noalloc: K = {K} outside 1..{MAX_BANK}")
+    if stats.dtype != torch.float64 or stats.numel() < SKETCH + 3 or not stats.is_contiguous():
+        raise ValueError(f"observe_noalloc: stats must be a contiguous float64 tensor of >= {SKETCH + 3} values")
+    n = z_hat.numel()
+    lat = [("z_hat", z_hat), ("z_a", z_a)] + [(f"z_out[{i}]", t) for i, t in enumerate(z_out)]
+    for name, t in lat:
+        if t.dtype != torch.float32 or t.numel() != n or not t.is_contiguous():
+            raise ValueError(f"observe_noalloc: {name} must be a contiguous float32 tensor of {n} elements")
+    dev = torch.device("cuda", torch.cuda.current_device()) if torch.cuda.is_available() else None
+    for name, t in lat + [("stats", stats)]:
+        if dev is None or t.device != dev:
+            raise ValueError(f"observe_noalloc: {name} must be on the current CUDA device")
     ptrs = (ctypes.c_void_p * K)(*[t.data_ptr() for t in z_out])
     kap = (ctypes.c_double * K)(*[float(x) for x in kappa])
     st = LIB.wdc_observe_noalloc(ptrs, K, kap, _ptr(z_a), _ptr(z_hat), _ptr(stats), z_hat.numel(), sketch_seed,

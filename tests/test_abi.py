@@ -82,3 +82,20 @@ def test_struct_layout_matches_a_c_compiler(tmp_path, cname, pystruct):
 def test_batch_limit_matches_the_header():
     src = open(os.path.join(ROOT, "include", "wdc.h")).read()
     assert int(re.search(r"#define WDC_MAX_BATCH\s+(\d+)", src).group(1)) == wdc.MAX_BATCH
+
+
+def test_observe_noalloc_binding_checks_sizes_before_the_call():
+    """wdc_observe_noalloc has no context that knows the latent size, so the
+    binding checks every tensor before calling in: a short statistics buffer
+    (120 of the 123 values) or a weight count that differs from the latent
+    count raises ValueError without reaching the library."""
+    import torch
+    z = torch.zeros(256, dtype=torch.float32)
+    with pytest.raises(ValueError, match="stats"):
+        wdc.observe_noalloc([z], [1.0], z, torch.zeros_like(z), torch.zeros(120, dtype=torch.float64))
+    with pytest.raises(ValueError, match="weights"):
+        wdc.observe_noalloc([z, z], [1.0], z, torch.zeros_like(z), torch.zeros(123, dtype=torch.float64))
+    with pytest.raises(ValueError, match="z_out"):
+        wdc.observe_noalloc([z[:128]], [1.0], z, torch.zeros_like(z), torch.zeros(123, dtype=torch.float64))
+    with pytest.raises(ValueError, match="device"):
+        wdc.observe_noalloc([z], [1.0], z, torch.zeros_like(z), torch.zeros(123, dtype=torch.float64))

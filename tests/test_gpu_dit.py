@@ -97,21 +97,39 @@ def test_bf16_gemm_matches_oracle(M, N, K, mode):
 @pytest.mark.parametrize("H,L,d", [(2, 1000, 64), (1, 1000, 128), (3, 264, 64), (1, 64, 128), (2, 4104, 64),
                                    (1, 2056, 128), (2, 300, 64), (1, 129, 128)])
 def test_bf16_attention_matches_oracle(H, L, d):
-    """L % 8 == 0 runs the tcgen05 kernel (ragged against its 128-key and
-    256-query tiles); other L the SIMT kernel."""
+    """Every L runs the tcgen05 kernel (ragged against its 128-key and
+    256-query tiles); V^T rows are padded to a multiple of 8 tokens, and the
+    padding holds NaN to show it is never read."""
     ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.BF16)
     q = _bf(synth.normal(11, (H, L, d)))
     k = _bf(synth.normal(12, (H, L, d)))
     v = _h(synth.normal(13, (H, L, d)))
     o = torch.empty(L, H * d, dtype=torch.bfloat16, device="cuda")
-    ctx.op_attention(_to_dev(q, torch.bfloat16), _to_dev(k, torch.bfloat16),
-                     _to_dev(np.ascontiguousarray(v.transpose(0, 2, 1)), torch.float16), o)
+    ldv = (L + 7) // 8 * 8
+    vt = np.full((H, d, ldv), np.nan, dtype=np.float32)
+    vt[:, :, :L] = v.transpose(0, 2, 1)
+    ctx.op_attention(_to_dev(q, torch.bfloat16), _to_dev(k, torch.bfloat16), _to_dev(vt, torch.float16), o)
     torch.cuda.synchronize()
     qf = q.transpose(1, 0, 2).reshape(L, H * d).astype(np.float64)
     kf = k.transpose(1, 0, 2).reshape(L, H * d).astype(np.float64)
     vf = v.transpose(1, 0, 2).reshape(L, H * d).astype(np.float64)
     want = dit.attention(qf, kf, vf, H)
     assert rel_l2(o.float().cpu().numpy(), want) <= 1e-2
+
+
+def test_bf16_shapes_outside_the_tensor_core_limits_are_errors():
+    """A bf16 model runs on the tcgen05 kernels only: a GEMM shape they do not
+    take is reported (WDC_ERR_UNSUPPORTED), never run on a slower path."""
+    ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.BF16)
+    launches = ctx.launches
+    for M, N, K in [(64, 48, 64), (64, 64, 12)]:
+        A = torch.zeros(M, K, dtype=torch.bfloat16, device="cuda")
+        W = torch.zeros(N, K, dtype=torch.bfloat16, device="cuda")
+        C = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+        with pytest.raises(wdc.WdcError) as e:
+            ctx.op_gemm(A, W, C)
+        assert e.value.status == 3 and "tcgen05" in str(e.value)
+    assert ctx.launches == launches
 
 
 @pytest.mark.parametrize("H,L,d", [(2, 300, 64), (2, 257, 128)])

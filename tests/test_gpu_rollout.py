@@ -1,7 +1,8 @@
 """Cached rollout on the GPU against the CPU oracle (2-layer D=256 model,
 latent 16x4x16x16, fp32 parity mode): the anchor/skip decision sequence must
-be identical and the final latent within 1e-4 relative L2 (fp32 kernels vs
-fp64).  Plus the invariants: all-exact == native bitwise, host-pointer API ==
+be identical and the final latent within 1e-5 relative L2 (fp32 kernels vs
+fp64), for the host-driven rollout and for the device-side control flow.
+Plus the invariants: all-exact == native bitwise, host-pointer API ==
 device-pointer API, and the printed 7-of-50 exact-call budget."""
 import json
 import os
@@ -52,12 +53,42 @@ def test_cfg0_decisions_and_latent_match_oracle():
     out = torch.empty(z0.size, dtype=torch.float32, device="cuda")
     dec, tr = ctx.rollout(torch.from_numpy(z0.ravel().copy()).cuda(), c, out)
     assert dec == dec_o
-    assert rel_l2(out.cpu().numpy(), zf_o) <= 1e-4
+    assert rel_l2(out.cpu().numpy(), zf_o) <= TOL
+    _check_trace(tr, tr_o)
+
+
+TOL = 1e-5
+
+
+def _check_trace(tr, tr_o, d_cf=True):
     for a, b in zip(tr, tr_o):
+        assert a["decision"] == b["decision"]
         for key in ["p", "d_hat", "w", "R_cand", "R", "eta"]:
-            assert abs(a[key] - b[key]) <= 1e-4 * max(1.0, abs(b[key])), (a["k"], key)
-        if not np.isnan(b["d_cf"]):
-            assert abs(a["d_cf"] - b["d_cf"]) <= 1e-4 * max(1.0, b["d_cf"])
+            assert abs(a[key] - b[key]) <= TOL * max(1.0, abs(b[key])), (a["k"], key)
+        if d_cf and not np.isnan(b["d_cf"]):
+            assert abs(a["d_cf"] - b["d_cf"]) <= TOL * max(1.0, b["d_cf"])
+
+
+@pytest.mark.parametrize("flags", [0, wdc.ABL_SECANT])
+def test_graph_rollout_matches_oracle(flags):
+    """wdc_rollout_graph (device-side control flow) against the CPU oracle's
+    cached rollout directly: the same decision sequence, the final latent
+    within 1e-5 relative L2 and the controller scalars of every step within
+    1e-5 relative."""
+    T = 10
+    op, cp, W, ctx, z0, ct, desc = _setup(T, tau_risk=0.5, flags=flags)
+    zf_o, dec_o, tr_o = _oracle(op, W, z0, ct, desc, T)
+    assert 0 < sum(dec_o) < T
+    for info in tr_o:
+        if info["margins"]:
+            assert min(info["margins"]) > 1e-4
+    c = wdc.make_cond(torch.from_numpy(ct).cuda(), desc["cam"], desc["depth"])
+    out = torch.empty(z0.size, dtype=torch.float32, device="cuda")
+    dec, tr = ctx.rollout_graph(torch.from_numpy(z0.ravel().copy()).cuda(), c, out)
+    assert dec == dec_o
+    assert rel_l2(out.cpu().numpy(), zf_o) <= TOL
+    _check_trace(tr, tr_o)
+    assert ctx.device_errors() == 0
 
 
 def test_all_exact_equals_native_bitwise():

@@ -49,12 +49,46 @@ def test_observe_noalloc_matches_skip_pass(n, K):
         assert s[122] == 0.0, call
 
 
+def _raw_call(z_out, kappa, z_a, z_hat, stats, n):
+    """The C entry point itself, without the binding's argument checks."""
+    import ctypes
+    ptrs = (ctypes.c_void_p * len(z_out))(*[t.data_ptr() for t in z_out])
+    kap = (ctypes.c_double * len(kappa))(*kappa)
+    return wdc.LIB.wdc_observe_noalloc(ptrs, len(z_out), kap, ctypes.c_void_p(z_a.data_ptr()),
+                                       ctypes.c_void_p(z_hat.data_ptr()), ctypes.c_void_p(stats.data_ptr()), n,
+                                       0x2545F491, ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+
+
 def test_observe_noalloc_rejects_sizes_beyond_its_limits():
     z = torch.zeros(1024, dtype=torch.float32, device="cuda")
+    zh = torch.empty_like(z)
     st = torch.zeros(123, dtype=torch.float64, device="cuda")
-    with pytest.raises(wdc.WdcError) as e:
-        wdc.observe_noalloc([z] * 9, [0.1] * 9, z, torch.empty_like(z), st)      # K > 8
-    assert e.value.status == 1
-    with pytest.raises(wdc.WdcError) as e:
-        wdc.observe_noalloc([z[1:]], [1.0], z, torch.empty_like(z), st)         # misaligned latent
-    assert e.value.status == 1
+    assert _raw_call([z] * 9, [0.1] * 9, z, zh, st, 1024) == 1              # K > 8
+    assert _raw_call([z[1:]], [1.0], z, zh, st, 1023) == 1                  # misaligned latent
+    assert _raw_call([z], [1.0], z, zh, st, 1 << 31) == 1                   # n beyond 32-bit indices
+    assert _raw_call([z], [1.0], z, zh, st, 0) == 1                         # empty
+    with pytest.raises(ValueError):
+        wdc.observe_noalloc([z] * 9, [0.1] * 9, z, zh, st)
+    with pytest.raises(ValueError):
+        wdc.observe_noalloc([z], [1.0], z, zh, st[:120])                    # short statistics buffer
+
+
+def test_observe_noalloc_allocates_no_device_memory():
+    """The property the entry point exists for: after a first call (which
+    looks up the scratch array's address), further calls leave the device's
+    free memory unchanged."""
+    n = 1 << 20
+    g = torch.Generator(device="cuda").manual_seed(3)
+    bank = [torch.randn(n, device="cuda", generator=g) for _ in range(4)]
+    zh = torch.empty(n, dtype=torch.float32, device="cuda")
+    stats = torch.empty(123, dtype=torch.float64, device="cuda")
+    kappa = [0.1, 0.2, 0.3, 0.4]
+    wdc.observe_noalloc(bank, kappa, bank[-1], zh, stats)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    first = zh.clone()
+    for _ in range(5):
+        wdc.observe_noalloc(bank, kappa, bank[-1], zh, stats)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert torch.equal(zh, first)
