@@ -254,51 +254,82 @@ def traffic_for(kernel_file, workload):
     return e.get("dram_bytes_per_launch")
 
 
-def skip_pass_gbps(torch, wdc, peaks, secant=False, n=SKIP_SWEEP_N):
-    """Fused skip pass alone at n fp32 elements (2^28 by default), bank of 4
-    (reads 4 N, writes N), L2 flushed by a 512 MB write before every launch.
-    With ``secant`` the native-latent-secant ablation's pass instead (reads
-    z_t, the stored displacement and z_a, writes N)."""
+def skip_pass_time(torch, wdc, n, K=4, secant=False, flush=True, reps=10, seed=0):
+    """The fused skip pass alone at n fp32 elements with a bank of K records
+    drawn by the sweep's recipe (z_out_i = z0 + 0.05 i sin(2 pi 8 idx/n +
+    phase_i), z0 ~ N(0,1)), every record compatible so the pass streams;
+    the average of `reps` launches timed with CUDA events on the launching
+    stream, L2 flushed by a 512 MB write before each launch (or not, for the
+    L2-resident figure).  With ``secant`` the native-latent-secant pass
+    instead (reads z_t, the stored displacement and z_a, writes N).  Returns
+    (ms per launch, algorithmic bytes, info of the last launch)."""
     import numpy as np
+    from paper_2608_01845_gb300 import synth
     flags = wdc.ABL_SECANT if secant else 0
     ctx = wdc.Context(wdc.make_config(layers=0, width=n), 50,
-                      params=wdc.make_params(bank_capacity=4, sim_min=-1.0, flags=flags))
-    dev = torch.device("cuda")
-    bank = [torch.randn(n, device=dev) for _ in range(4)]
+                      params=wdc.make_params(bank_capacity=K, sim_min=-1.0, q_gap_max=1.0, flags=flags))
+    bank = synth.drift_bank_device(seed + n % 1000003 + K, n, K)
     st = wdc.StateHost()
-    st.n_bank, st.R, st.eta = 4, 0.1, 1.0
-    g = np.random.default_rng(0)
-    for i in range(4):
+    st.n_bank, st.R, st.eta = K, 0.1, 1.0
+    g = np.random.default_rng(seed)
+    for i in range(K):
         a = g.standard_normal(256)
         for j in range(256):
             st.rec[i].s_in[j] = a[j]
             st.rec[i].s_out[j] = a[j] + 0.1
             st.rec[i].s_dphi[j] = 0.1
-        st.rec[i].q_in = 0.6 + 0.02 * (4 - i)
+        st.rec[i].q_in = 0.6 + 0.02 * (K - i)
         st.rec[i].q_out = st.rec[i].q_in - 0.02
-    st.q_a_in, st.q_a_out = st.rec[3].q_in, st.rec[3].q_out
-    zc = torch.randn(n, device=dev)
+    st.q_a_in, st.q_a_out = st.rec[K - 1].q_in, st.rec[K - 1].q_out
+    zc = bank[-1] + 0.01
     ctx.state_set(st, bank, zc)
-    zh = torch.empty(n, device=dev)
-    flush = torch.empty(128 * 1024 * 1024, device=dev)
+    zh = torch.empty(n, device="cuda")
+    buf = torch.empty(128 * 1024 * 1024, device="cuda") if flush else None
     cond = wdc.make_cond()
     for _ in range(3):
-        flush.zero_()
+        if flush:
+            buf.zero_()
         ctx.surrogate_step(20, cond, zh)
     ctx.profile_enable(True)
-    reps = 10
     for _ in range(reps):
-        flush.zero_()
+        if flush:
+            buf.zero_()
         info = ctx.surrogate_step(20, cond, zh)
     prof = ctx.profile_read()
+    ctx.profile_enable(False)
     ms = prof["skip"][0] / prof["skip"][1]
-    streams = 4 if secant else 5
-    gbs = streams * 4 * n / (ms * 1e-3) / 1e9
+    streams = 4 if secant else K + 1
     ctx.close()
-    del bank, zc, zh, flush
+    del bank, zc, zh, buf
     torch.cuda.empty_cache()
-    return {"gbps": gbs, "ms": ms, "n": n, "bank": 4, "supported": bool(info.supported),
-            "bytes": streams * 4 * n, "frac_of_measured_copy": gbs / peaks["hbm_gbs"]}
+    return ms, streams * 4 * n, info
+
+
+def skip_pass_gbps(torch, wdc, peaks, secant=False, n=SKIP_SWEEP_N, K=4, flush=True):
+    ms, nbytes, info = skip_pass_time(torch, wdc, n, K, secant=secant, flush=flush)
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    return {"gbps": gbs, "ms": ms, "n": n, "bank": K, "supported": bool(info.supported), "bytes": nbytes,
+            "frac_of_measured_copy": gbs / peaks["hbm_gbs"], "l2": "flushed" if flush else "resident"}
+
+
+def skip_sweep(torch, wdc, peaks, workload_n):
+    """The skipped-step kernel sweep: N in {2^20, 2^24, 2^26, 2^28} fp32
+    elements x K in {2, 3, 4} bank records, L2 flushed before every launch;
+    plus 2^20 L2-resident and the workload's own latent size."""
+    rows = []
+    for e in (20, 24, 26, 28):
+        for K in (2, 3, 4):
+            r = skip_pass_gbps(torch, wdc, peaks, n=1 << e, K=K)
+            rows.append({"n": f"2^{e}", "K": K, "gbps": round(r["gbps"], 1), "ms": round(r["ms"], 5),
+                         "frac_of_measured_copy": round(r["frac_of_measured_copy"], 4)})
+    r = skip_pass_gbps(torch, wdc, peaks, n=1 << 20, K=4, flush=False)
+    rows.append({"n": "2^20", "K": 4, "l2": "resident", "gbps": round(r["gbps"], 1), "ms": round(r["ms"], 5),
+                 "frac_of_measured_copy": round(r["frac_of_measured_copy"], 4)})
+    r = skip_pass_gbps(torch, wdc, peaks, n=workload_n, K=4)
+    rows.append({"n": workload_n, "K": 4, "note": "the rollout's own latent", "gbps": round(r["gbps"], 1),
+                 "ms": round(r["ms"], 5), "frac_of_measured_copy": round(r["frac_of_measured_copy"], 4)})
+    return {"bytes_per_launch": "(K+1)*4*N", "timing": "CUDA events on the launching stream, mean of 10",
+            "rows": rows}
 
 
 def block_tflops(torch, ctx, w, peaks):
@@ -320,6 +351,125 @@ def block_tflops(torch, ctx, w, peaks):
     g, a = block_flops(w)
     tf = (g + a) / (ms * 1e-3) / 1e12
     return {"tflops": tf, "ms": ms, "frac_of_measured_burst": tf / peaks["bf16_tflops"]}
+
+
+# The 2-layer parity model (the oracle-checked configuration): fp32, D = 256,
+# 4 x 64 heads, MLP 1024, latent 16x4x16x16 + 16 condition tokens, T = 10.
+WORKLOAD_CFG0 = dict(
+    name="cached rollout, 2-layer fp32 DiT 256/4x64/1024, latent 16x4x16x16 + 16 cond tokens, T=10",
+    layers=2, hidden=256, heads=4, head_dim=64, mlp=1024, temb_dim=256, freq_dim=256, in_ch=16, frames=4,
+    height=16, width=16, patch=2, cond_tokens=16, cond_dim=256, dual_stream=0, T=10, tau_risk=0.5,
+)
+
+
+def surrogate_reading(flags):
+    """Which reading of Eq. 5's observation the run used."""
+    if flags & 0x02:
+        return "native latent secant (ablation)"
+    if flags & 0x100:
+        return "residual reading of Eq. 5: z_t + sum_i kappa_i (z_out_i - z_in_i)"
+    return "Eq. 5 as printed: sum_i kappa_i z_out_i"
+
+
+def rollout_component(torch, wdc, w, peaks, reps=2):
+    """One workload's cached rollout on its own context: steps/s over `reps`
+    timed rollouts after one warm-up, the exact-step count, and the dominant
+    kernel class against the measured sustained bf16 peak (live CUDA-event
+    durations)."""
+    T = w["T"]
+    ctx = wdc.Context(dit_config(w), T, params=wdc.make_params(tau_risk=w["tau_risk"]))
+    ctx.init_weights(w["weight_seed"], 0.02)
+    zT, ct, desc = inputs(w, 0)
+    zT_d = torch.from_numpy(zT).cuda()
+    ct_d = torch.from_numpy(ct).cuda()
+    cond = wdc.make_cond(ct_d, desc["cam"], desc["depth"])
+    out = torch.empty_like(zT_d)
+    ctx.rollout(zT_d, cond, out, trace=False)
+    torch.cuda.synchronize()
+    ctx.profile_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    exact = []
+    for _ in range(reps):
+        dec, _ = ctx.rollout(zT_d, cond, out, trace=False)
+        exact.append(T - sum(dec))
+    e1.record()
+    torch.cuda.synchronize()
+    prof = ctx.profile_read()
+    ctx.profile_enable(False)
+    ms = e0.elapsed_time(e1) / reps
+    cls = {k: v[0] for k, v in prof.items()}
+    dom = max(cls, key=cls.get)
+    if dom == "attention":
+        avg = prof["attention"][0] / prof["attention"][1]
+        achieved = block_flops(w)[1] / (avg * 1e-3) / 1e12
+    else:
+        avg = None
+        achieved = None
+    ctx.close()
+    del zT_d, ct_d, out
+    torch.cuda.empty_cache()
+    res = {"workload": w["name"], "steps_per_s": T / (ms * 1e-3), "ms_per_rollout": ms, "exact_steps": exact,
+           "tau_risk": w["tau_risk"], "dominant_kernel": dom,
+           "time_share": {k: v / sum(cls.values()) for k, v in cls.items()}}
+    if achieved is not None:
+        res.update({"attention_avg_launch_ms": avg, "attention_tflops": achieved,
+                    "attention_frac_of_measured_sustained": achieved / peaks["bf16_tflops_sustained"]})
+    return res
+
+
+def cfg0_component(torch, wdc, cpu=True, reps=20):
+    """The 2-layer fp32 parity model's cached rollout (T = 10): steps/s on the
+    GPU (host-driven and graph rollout, median of `reps`), and the CPU oracle's
+    own cached rollout of the same inputs timed on the host cores."""
+    import numpy as np
+    from paper_2608_01845_gb300 import synth
+    w = WORKLOAD_CFG0
+    keys = ["layers", "hidden", "heads", "head_dim", "mlp", "temb_dim", "freq_dim", "in_ch", "frames", "height",
+            "width", "patch", "cond_tokens", "cond_dim", "dual_stream"]
+    cfgd = {k: w[k] for k in keys}
+    T = w["T"]
+    W = synth.dit_weights(cfgd, 0, std=0.02)
+    ctx = wdc.Context(wdc.make_config(dtype=wdc.F32, **cfgd), T, params=wdc.make_params(tau_risk=w["tau_risk"]))
+    ctx.set_weights(W)
+    z0 = synth.latent(1, (16, 4, 16, 16))
+    ct = synth.cond_tokens(2, 16, 256)
+    desc = synth.cond_descriptors(3)
+    zT = torch.from_numpy(z0.ravel().copy()).cuda()
+    cond = wdc.make_cond(torch.from_numpy(ct).cuda(), desc["cam"], desc["depth"])
+    out = torch.empty_like(zT)
+    res = {"workload": w["name"]}
+    for mode, fn in [("host", lambda: ctx.rollout(zT, cond, out, trace=False)),
+                     ("graph", lambda: ctx.rollout_graph(zT, cond, out, trace=False))]:
+        for _ in range(3):
+            dec, _ = fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        ms = statistics.median(ts)
+        res[mode] = {"steps_per_s": T / (ms * 1e-3), "ms_per_rollout": ms, "exact_steps": T - sum(dec)}
+    res["decisions"] = dec
+    ctx.close()
+    if cpu:
+        from oracle import dit
+        from oracle import rollout as ro
+        from oracle import schedule as sch
+        from oracle.params import CacheParams, DiTConfig
+        cfg = DiTConfig(**cfgd)
+        F = lambda z, t, c, k: dit.forward(W, cfg, np.asarray(z).reshape(16, 4, 16, 16), t, ct)
+        t0 = time.perf_counter()
+        _, dec_o, _ = ro.cached_rollout(z0, F, desc, sch.sigmas(T), CacheParams(tau_risk=w["tau_risk"]))
+        sec = time.perf_counter() - t0
+        res["cpu_oracle"] = {"steps_per_s": T / sec, "s_per_rollout": sec, "cores": os.cpu_count(),
+                             "kind": "oracle", "decisions_equal": dec_o == dec,
+                             "sample": "the whole 10-step cached rollout (fp64 numpy)"}
+    return res
 
 
 # Ablation variants of Tables 3-4 (and the residual reading of Eq. 5) for
@@ -441,6 +591,7 @@ def run_gpu(args, rank, world, local_rank):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": w["name"] + (f", ablation {args.ablation}" if args.ablation else ""),
                        "T": T, "tau_risk": w["tau_risk"], "bank_capacity": 4,
+                       "surrogate_reading": surrogate_reading(params.flags),
                        "l2": f"inputs larger than L2 ({weight_gb(w):.1f} GB of weights per forward)",
                        "parallelism": f"replicas x{world}"},
             "exact_steps_per_rollout": exact, "gpu_launches": launches, "clocks": clk, "roofline": roofline}
@@ -487,8 +638,14 @@ def run_gpu(args, rank, world, local_rank):
         line["components"] = {"dit_block": block_tflops(torch, ctx, w, peaks)}
         ctx.close()
         torch.cuda.empty_cache()
+        if not args.ablation and not args.no_extra_rollouts:
+            other = "13b" if args.workload == "5b" else "5b"
+            line["components"][f"rollout_{other}"] = rollout_component(torch, wdc, WORKLOADS[other], peaks)
+            line["components"]["rollout_cfg0"] = cfg0_component(torch, wdc, cpu=world == 1)
         line["components"]["skip_pass"] = skip_pass_gbps(torch, wdc, peaks)
         line["components"]["secant_pass"] = skip_pass_gbps(torch, wdc, peaks, secant=True)
+        line["components"]["skip_sweep"] = skip_sweep(torch, wdc, peaks,
+                                                      w["in_ch"] * w["frames"] * w["height"] * w["width"])
         line["components"]["peaks"] = {"hbm_gbs": peaks["hbm_gbs"], "bf16_tflops": peaks["bf16_tflops"],
                                        "source": peak_src}
         if world == 1 and not args.no_cpu_baseline:
@@ -590,8 +747,11 @@ def run_op(args):
             del A, Wt, C
         print(json.dumps({"op": "gemms", "workload": args.workload, **out}))
         return
+    elif args.op == "skip_sweep":
+        print(json.dumps({"op": "skip_sweep", **skip_sweep(torch, wdc, peaks, 16 * 13 * 60 * 90)}))
+        return
     else:
-        r = skip_pass_gbps(torch, wdc, peaks, secant=args.op == "secant", n=args.n)
+        r = skip_pass_gbps(torch, wdc, peaks, secant=args.op == "secant", n=args.n, K=args.bank)
         print(json.dumps({"op": args.op, **r}))
         return
     for _ in range(2):
@@ -664,14 +824,18 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="wdc", choices=["wdc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra-rollouts", action="store_true",
+                    help="skip the other full-size workload's and the 2-layer model's rollouts")
     ap.add_argument("--ablation", choices=sorted(ABLATIONS),
                     help="run the timed rollout under one ablation variant (Tables 3-4) and report its "
                          "final latent against the uncached rollout")
-    ap.add_argument("--op", choices=["attention", "gemm", "gemms", "block", "skip", "secant", "control", "batch"],
+    ap.add_argument("--op", choices=["attention", "gemm", "gemms", "block", "skip", "secant", "skip_sweep", "control",
+                                     "batch"],
                     help="time one operator at its 5B-scale shape (profiler captures); batch: the batched "
                          "cached rollout against one-at-a-time rollouts")
     ap.add_argument("--batch", type=int, default=2, help="--op batch: samples per batch")
     ap.add_argument("--n", type=int, default=SKIP_SWEEP_N, help="--op skip / secant: latent elements")
+    ap.add_argument("--bank", type=int, default=4, help="--op skip: bank records K")
     ap.add_argument("--cfg", action="store_true", help="--op batch: classifier-free guidance on every exact step")
     ap.add_argument("--guidance", type=float, default=5.0, help="--op batch: guidance scale with --cfg")
     ap.add_argument("--reps", type=int, default=3)

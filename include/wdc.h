@@ -300,6 +300,31 @@ wdc_status wdc_dit_block_forward(wdc_ctx* ctx, int layer, void* x, const float* 
  * followed by the final layer's [2][hidden] into mod_out (device fp32). */
 wdc_status wdc_dit_modulation(wdc_ctx* ctx, float t, float* mod_out, wdc_stream stream);
 
+/* The schedule's T + 1 noise levels sigma_0..sigma_T (fp64, as the context
+ * computes them: sigma_k = 1 - k/T, time-shifted when shift != 1) into the
+ * host array out[T + 1].  Step k runs the denoiser at model timestep
+ * (float)(1000 sigma_k) and its phase is q_k = sigma_k (section
+ * "Condition-Aware Lifted State": the normalised timestep stands in for the
+ * scheduler phase). */
+wdc_status wdc_schedule_sigmas(const wdc_ctx* ctx, double* out);
+
+/* ------------------------------------------------------------------ diagnostics
+ * Device reductions for the synthetic diagnostics of section "Motivation and
+ * Observations" (Fig. 2) and section "Transition Risk Controller" (Fig. 3a):
+ * for latents a, b and c (device fp32, N elements each, 16-byte aligned; c may
+ * be NULL, read as zero) writes to the host array out[5]
+ *   out[0] = sum (a - c)^2,  out[1] = sum (b - c)^2,  out[2] = sum (a - c)(b - c),
+ *   out[3] = sum (a - b)^2,  out[4] = sum b^2
+ * (fp32 arithmetic, deterministic fixed-order reductions), from which the
+ * downstream impact ||a - b|| / ||b|| and the direction error between the
+ * increments a - c and b - c follow.  Synchronises the stream. */
+wdc_status wdc_latent_pair_stats(wdc_ctx* ctx, const float* a, const float* b, const float* c, double* out,
+                                 wdc_stream stream);
+/* Pearson and Spearman (average ranks) correlations of two host samples x, y
+ * of n >= 2 values (Fig. 3a: predicted versus counterfactual defect); NaN
+ * when a sample is constant.  Host code, no context or device needed. */
+wdc_status wdc_correlations(const double* x, const double* y, int n, double* pearson, double* spearman);
+
 /* ------------------------------------------------------------------ Psi_t */
 /* z_next = Psi_k(z_t, v) = z_t + (sigma_{k+1} - sigma_k) v (Eq. 1, flow-matching
  * Euler), elementwise fp32 (one fused multiply-add).  z_next may equal z_t. */
@@ -448,7 +473,7 @@ wdc_status wdc_op_attention(wdc_ctx* ctx, const void* q, const void* k, const vo
  * The paper has no counterpart: it is a deployment variant of the same kernel.
  *
  * It allocates nothing and needs no wdc_ctx.  Its scratch (per-CTA partial sums
- * and a completion counter, 256 CTAs x 248 doubles + 256 bytes = 508 KB) is a
+ * and a completion counter, 256 CTAs x 248 floats + 256 bytes = 254 KB) is a
  * file-scope __device__ array that every GPU loading libwdc.so holds until the
  * process exits.  The first call on a device, with that device current, looks
  * up the array's device address (cudaGetSymbolAddress) and caches it; make that

@@ -10,6 +10,7 @@
 #include "wdc_internal.h"
 #include "ptx.cuh"
 
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <new>
@@ -336,9 +337,10 @@ wdc_status wdc_create(const wdc_dit_config* cfg, const wdc_schedule* sched, cons
         return true;
     };
     if (!dm((void**)&c->st, sizeof(DevState))) return bail(WDC_ERR_OOM);
-    if (!dm((void**)&c->partials, (size_t)c->num_sms * 2 * kPartials * sizeof(double))) return bail(WDC_ERR_OOM);
+    if (!dm((void**)&c->partials, (size_t)c->num_sms * kPartials * sizeof(float))) return bail(WDC_ERR_OOM);
     if (!dm((void**)&c->counter, 64)) return bail(WDC_ERR_OOM);
     if (!dm((void**)&c->err, 64)) return bail(WDC_ERR_OOM);
+    if (!dm((void**)&c->pstat, 64)) return bail(WDC_ERR_OOM);
     for (int i = 0; i < c->prm.bank_capacity; ++i)
         if (!dm((void**)&c->bank[i], lat)) return bail(WDC_ERR_OOM);
     if (!dm((void**)&c->z_init, lat)) return bail(WDC_ERR_OOM);
@@ -364,6 +366,7 @@ void wdc_destroy(wdc_ctx* h) {
     cudaFree(c->partials);
     cudaFree(c->counter);
     cudaFree(c->err);
+    cudaFree(c->pstat);
     for (int i = 0; i < kMaxBank; ++i) cudaFree(c->bank[i]);
     cudaFree(c->z_init);
     cudaFree(c->cand[0]);
@@ -510,6 +513,69 @@ wdc_status wdc_dit_modulation(wdc_ctx* h, float t, float* mod_out, wdc_stream st
     return dit_modulation(c, t, mod_out, (cudaStream_t)stream);
 }
 
+wdc_status wdc_schedule_sigmas(const wdc_ctx* h, double* out) {
+    const Ctx* c = reinterpret_cast<const Ctx*>(h);
+    if (!c || !out) return WDC_ERR_INVALID_ARG;
+    for (size_t k = 0; k < c->sigma.size(); ++k) out[k] = c->sigma[k];
+    return WDC_OK;
+}
+
+wdc_status wdc_latent_pair_stats(wdc_ctx* h, const float* a, const float* b, const float* cz, double* out,
+                                 wdc_stream stream) {
+    Ctx* c = reinterpret_cast<Ctx*>(h);
+    if (!c) return WDC_ERR_INVALID_ARG;
+    if (!a || !b || !out) return fail(c, WDC_ERR_INVALID_ARG, "null pointer");
+    if (!aligned16(a) || !aligned16(b) || (cz && !aligned16(cz)))
+        return fail(c, WDC_ERR_INVALID_ARG, "latents must be 16-byte aligned device pointers");
+    cudaSetDevice(c->device);
+    cudaStream_t s = (cudaStream_t)stream;
+    wdc_status st = launch_pair_stats(c, a, b, cz, c->pstat, s);
+    if (st) return st;
+    WDC_CUDA_TRY(c, cudaMemcpyAsync(out, c->pstat, 5 * sizeof(double), cudaMemcpyDeviceToHost, s));
+    WDC_CUDA_TRY(c, cudaStreamSynchronize(s));
+    return WDC_OK;
+}
+
+// Average ranks (ties share the mean of their positions), 0-based.
+static void average_ranks(const double* x, int n, std::vector<double>& r) {
+    std::vector<int> idx(n);
+    for (int i = 0; i < n; ++i) idx[i] = i;
+    std::stable_sort(idx.begin(), idx.end(), [&](int p, int q) { return x[p] < x[q]; });
+    r.assign(n, 0.0);
+    for (int i = 0; i < n;) {
+        int j = i;
+        while (j + 1 < n && x[idx[j + 1]] == x[idx[i]]) ++j;
+        const double avg = 0.5 * (i + j);
+        for (int m = i; m <= j; ++m) r[idx[m]] = avg;
+        i = j + 1;
+    }
+}
+
+static double pearson(const double* x, const double* y, int n) {
+    double mx = 0, my = 0;
+    for (int i = 0; i < n; ++i) { mx += x[i]; my += y[i]; }
+    mx /= n;
+    my /= n;
+    double sxy = 0, sxx = 0, syy = 0;
+    for (int i = 0; i < n; ++i) {
+        const double dx = x[i] - mx, dy = y[i] - my;
+        sxy += dx * dy;
+        sxx += dx * dx;
+        syy += dy * dy;
+    }
+    return (sxx > 0 && syy > 0) ? sxy / std::sqrt(sxx * syy) : NAN;
+}
+
+wdc_status wdc_correlations(const double* x, const double* y, int n, double* pearson_out, double* spearman_out) {
+    if (!x || !y || !pearson_out || !spearman_out || n < 2) return WDC_ERR_INVALID_ARG;
+    *pearson_out = pearson(x, y, n);
+    std::vector<double> rx, ry;
+    average_ranks(x, n, rx);
+    average_ranks(y, n, ry);
+    *spearman_out = pearson(rx.data(), ry.data(), n);
+    return WDC_OK;
+}
+
 wdc_status wdc_scheduler_step(wdc_ctx* h, int k, const float* z_t, const float* v, float* z_next, wdc_stream stream) {
     Ctx* c = reinterpret_cast<Ctx*>(h);
     if (!c) return WDC_ERR_INVALID_ARG;
@@ -576,18 +642,22 @@ wdc_status wdc_state_get(wdc_ctx* h, wdc_state_host* out, wdc_stream stream) {
     for (int i = 0; i < c->n_bank; ++i) {
         const DevRecord& r = hs->rec[slot_of(c, i)];
         wdc_record_host& o = out->rec[i];
-        std::memcpy(o.s_in, r.s_in, sizeof(o.s_in));
-        std::memcpy(o.s_out, r.s_out, sizeof(o.s_out));
-        std::memcpy(o.s_dphi, r.s_dphi, sizeof(o.s_dphi));
+        for (int j = 0; j < kSummary; ++j) {
+            o.s_in[j] = r.s_in[j];
+            o.s_out[j] = r.s_out[j];
+            o.s_dphi[j] = r.s_dphi[j];
+        }
         o.q_in = r.q_in; o.q_out = r.q_out; o.r = r.r;
         for (int j = 0; j < 4; ++j) { o.cam[j] = r.cam[j]; o.depth[j] = r.depth[j]; }
     }
-    std::memcpy(out->cur_sketch, hs->cur_S, sizeof(out->cur_sketch));
+    for (int j = 0; j < kSketch; ++j) {
+        out->cur_sketch[j] = hs->cur_S[j];
+        out->anchor_sketch[j] = hs->anchor_S[j];
+    }
     out->cur_sumsq = hs->cur_sumsq;
     out->cur_sumsq_anchor = hs->cur_sumsq_anchor;
-    std::memcpy(out->anchor_sketch, hs->anchor_S, sizeof(out->anchor_sketch));
     out->anchor_sumsq = hs->anchor_sumsq;
-    std::memcpy(out->s_phi, hs->s_phi, sizeof(out->s_phi));
+    for (int j = 0; j < kSummary; ++j) out->s_phi[j] = hs->s_phi[j];
     out->cand_supported = hs->cand_supported;
     out->cand_finite = hs->cand_finite;
     out->cand_p = hs->cand_p;
@@ -617,13 +687,16 @@ wdc_status wdc_state_set(wdc_ctx* h, const wdc_state_host* in, const float* cons
     for (int i = 0; i < in->n_bank; ++i) {
         DevRecord& r = hs->rec[i];
         const wdc_record_host& o = in->rec[i];
-        std::memcpy(r.s_in, o.s_in, sizeof(r.s_in));
-        std::memcpy(r.s_out, o.s_out, sizeof(r.s_out));
-        std::memcpy(r.s_dphi, o.s_dphi, sizeof(r.s_dphi));
         double a = 0, b = 0;
-        for (int j = 0; j < kSummary; ++j) { a += o.s_in[j] * o.s_in[j]; b += o.s_out[j] * o.s_out[j]; }
-        r.n_in = std::sqrt(a);
-        r.n_out = std::sqrt(b);
+        for (int j = 0; j < kSummary; ++j) {
+            r.s_in[j] = (float)o.s_in[j];
+            r.s_out[j] = (float)o.s_out[j];
+            r.s_dphi[j] = (float)o.s_dphi[j];
+            a += (double)r.s_in[j] * r.s_in[j];
+            b += (double)r.s_out[j] * r.s_out[j];
+        }
+        r.n_in = (float)std::sqrt(a);
+        r.n_out = (float)std::sqrt(b);
         r.q_in = o.q_in; r.q_out = o.q_out; r.r = o.r;
         for (int j = 0; j < 4; ++j) { r.cam[j] = o.cam[j]; r.depth[j] = o.depth[j]; }
     }

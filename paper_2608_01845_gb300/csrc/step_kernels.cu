@@ -56,45 +56,72 @@ __device__ __forceinline__ float signed_term(uint32_t idx, uint32_t seed, float 
     return __int_as_float(__float_as_int(x) ^ (int)h);
 }
 
+// Butterfly sum over the 32 lanes (a fixed-order tree: every lane ends with
+// the same value).
 __device__ __forceinline__ float warp_sum_f(float v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     return v;
 }
-__device__ __forceinline__ double warp_sum_d(double v) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
+
+// Compensated (Kahan) accumulation s += x, c = running compensation.
+__device__ __forceinline__ void kahan_add(float& s, float& c, float x) {
+    const float y = x - c;
+    const float t = s + y;
+    c = (t - s) - y;
+    s = t;
 }
 
 // Sum NV values over the first 256 threads (8 warps) in fixed order; result in
 // out[0..NV) (shared).  Every thread of the block must call it.
 template <int NV>
-__device__ __forceinline__ void reduce256(double (&v)[NV], double* scratch, double* out) {
+__device__ __forceinline__ void reduce256(float (&v)[NV], float* scratch, float* out) {
     const int t = threadIdx.x, lane = t & 31, w = t >> 5;
 #pragma unroll
-    for (int j = 0; j < NV; ++j) v[j] = warp_sum_d(v[j]);
+    for (int j = 0; j < NV; ++j) v[j] = warp_sum_f(v[j]);
     if (lane == 0 && w < 8) {
 #pragma unroll
         for (int j = 0; j < NV; ++j) scratch[w * NV + j] = v[j];
     }
     __syncthreads();
     if (t < NV) {
-        double s = 0.0;
-        for (int q = 0; q < 8; ++q) s += scratch[q * NV + t];
-        out[t] = s;
+        const float* s = scratch + t;
+        out[t] = ((s[0] + s[NV]) + (s[2 * NV] + s[3 * NV])) + ((s[4 * NV] + s[5 * NV]) + (s[6 * NV] + s[7 * NV]));
+    }
+    __syncthreads();
+}
+
+// fp64 variant of reduce256 (the linear observation's ill-conditioned ridge
+// system only).
+template <int NV>
+__device__ __forceinline__ void reduce256d(double (&v)[NV], double* scratch, double* out) {
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+#pragma unroll
+    for (int j = 0; j < NV; ++j)
+#pragma unroll
+        for (int o = 16; o; o >>= 1) v[j] += __shfl_xor_sync(0xffffffffu, v[j], o);
+    if (lane == 0 && w < 8) {
+#pragma unroll
+        for (int j = 0; j < NV; ++j) scratch[w * NV + j] = v[j];
+    }
+    __syncthreads();
+    if (t < NV) {
+        double acc = 0.0;
+        for (int q = 0; q < 8; ++q) acc += scratch[q * NV + t];
+        out[t] = acc;
     }
     __syncthreads();
 }
 
 struct HeadShared {
-    double phi[kSummary];
-    double hat[kSummary];
-    double scratch[8 * (kMaxBank + 1)];
-    double red[kMaxBank + 1];
-    double gram[kMaxBank][kMaxBank];       // linear observation: the records' Gram matrix
-    double sim_in[kMaxBank], sim_out[kMaxBank], pi[kMaxBank], kappa[kMaxBank];
-    double alpha;
+    float phi[kSummary];
+    float hat[kSummary];
+    float scratch[8 * (kMaxBank + 1)];
+    float red[kMaxBank + 1];
+    double dscratch[8 * kMaxBank];          // linear observation: fp64 reduction scratch
+    double gram[kMaxBank + 1][kMaxBank];    // linear observation: the records' Gram matrix, then S_out s_hat
+    float sim_in[kMaxBank], sim_out[kMaxBank], pi[kMaxBank], kappa[kMaxBank];
+    float alpha;
     int compat[kMaxBank];
     int n_compat, supported;
 };
@@ -103,24 +130,25 @@ struct HeadShared {
 // coefficients of s(phi_hat) on the records' output summaries,
 // (G + rho I) beta = S_out s_hat with G_ij = s_out_i . s_out_j and
 // rho = ridge * trace(G) / K, solved by Cholesky in fp64 (G + rho I is
-// positive definite for rho > 0).  hs.red[0..K) still holds S_out s_hat.
+// positive definite for rho > 0).  The system is ill-conditioned at a small
+// ridge, so G and S_out s_hat are reduced in fp64 here.
 template <int K>
 __device__ __noinline__ void linear_readout(const PassArgs& a, HeadShared& hs) {
     if constexpr (K > 0) {
         const int t = threadIdx.x;
         const DevState* st = a.st;
+        // one row of G per reduction (keeps K values per thread); row K = S_out s_hat
+        for (int i = 0; i <= K; ++i) {
+            double v[K];
+            const double si = (t < kSummary) ? (i < K ? (double)st->rec[a.slot[i]].s_out[t] : (double)hs.hat[t]) : 0.0;
+#pragma unroll
+            for (int j = 0; j < K; ++j) v[j] = (t < kSummary) ? si * (double)st->rec[a.slot[j]].s_out[t] : 0.0;
+            reduce256d<K>(v, hs.dscratch, hs.gram[i]);
+        }
         double b[K];
         if (t == 0) {
 #pragma unroll
-            for (int i = 0; i < K; ++i) b[i] = hs.red[i];
-        }
-        // one row of G per reduction (keeps K values per thread)
-        for (int i = 0; i < K; ++i) {
-            double v[K];
-            const double si = (t < kSummary) ? st->rec[a.slot[i]].s_out[t] : 0.0;
-#pragma unroll
-            for (int j = 0; j < K; ++j) v[j] = (t < kSummary) ? si * st->rec[a.slot[j]].s_out[t] : 0.0;
-            reduce256<K>(v, hs.scratch, hs.gram[i]);
+            for (int i = 0; i < K; ++i) b[i] = hs.gram[K][i];
         }
         if (t == 0) {
             double A[K][K];
@@ -131,7 +159,7 @@ __device__ __noinline__ void linear_readout(const PassArgs& a, HeadShared& hs) {
             }
             if (tr == 0.0) {
 #pragma unroll
-                for (int i = 0; i < K; ++i) hs.kappa[i] = 0.0;
+                for (int i = 0; i < K; ++i) hs.kappa[i] = 0.f;
             } else {
                 const double rho = a.prm.ridge * tr / K;
 #pragma unroll
@@ -148,7 +176,7 @@ __device__ __noinline__ void linear_readout(const PassArgs& a, HeadShared& hs) {
                         A[i][j] = x / d;
                     }
                 }
-                double y[K];
+                double y[K], beta[K];
                 for (int i = 0; i < K; ++i) {
                     double x = b[i];
                     for (int m = 0; m < i; ++m) x -= A[i][m] * y[m];
@@ -156,144 +184,169 @@ __device__ __noinline__ void linear_readout(const PassArgs& a, HeadShared& hs) {
                 }
                 for (int i = K - 1; i >= 0; --i) {
                     double x = y[i];
-                    for (int m = i + 1; m < K; ++m) x -= A[m][i] * hs.kappa[m];
-                    hs.kappa[i] = x / A[i][i];
+                    for (int m = i + 1; m < K; ++m) x -= A[m][i] * beta[m];
+                    beta[i] = x / A[i][i];
                 }
+                for (int i = 0; i < K; ++i) hs.kappa[i] = (float)beta[i];
             }
         }
         __syncthreads();
     }
 }
 
-// Skip-pass head (every CTA, redundantly): Eq. 2-5 scalar part.
+// Skip-pass head, Eq. 2-5 scalar part, in fp32 (every CTA computes it; it is
+// a few hundred cycles of latency, and no CTA has to wait for another).
 template <int K>
 __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
     const DevState* st = a.st;
     const int t = threadIdx.x;
-    const double N = (double)a.n;
-    const double sc = sqrt((double)kSketch / N);
+    const float N = (float)a.n;
+    const float sc = sqrtf((float)kSketch / N);
+    const float eps_nu = (float)a.prm.eps_nu;
+    const bool no_cond = a.prm.flags & WDC_ABL_NO_COND;
     // s(phi_k): current-state summary (Eq. 2 through the linear sketch)
     if (t < kSummary) {
-        double val;
+        float val;
         if (t < kSketch) {
-            val = sc * st->cur_S[t] / (sqrt(st->cur_sumsq / N) + a.prm.eps_nu);
+            val = sc * st->cur_S[t] / (sqrtf((float)st->cur_sumsq / N) + eps_nu);
         } else if (t < 2 * kSketch) {
             const int b = t - kSketch;
-            val = sc * (st->cur_S[b] - st->anchor_S[b]) / (sqrt(st->cur_sumsq_anchor / N) + a.prm.eps_nu);
+            val = sc * (st->cur_S[b] - st->anchor_S[b]) / (sqrtf((float)st->cur_sumsq_anchor / N) + eps_nu);
         } else if (t < kOffDepth) {
-            val = (a.prm.flags & WDC_ABL_NO_COND) ? 0.0 : a.cam[t - kOffCam];
+            val = no_cond ? 0.f : (float)a.cam[t - kOffCam];
         } else if (t < kOffQ) {
-            val = (a.prm.flags & WDC_ABL_NO_COND) ? 0.0 : a.depth[t - kOffDepth];
+            val = no_cond ? 0.f : (float)a.depth[t - kOffDepth];
         } else if (t == kOffQ) {
-            val = a.q_k;
+            val = (float)a.q_k;
         } else {
             // h(H): [r_1..3, T*(q_in - q_out)_1..3, n_bank/K], newest record first
             const int j = t - kOffH;
-            val = 0.0;
+            val = 0.f;
             if (j < 3) {
-                if (j < a.nsrc) val = st->rec[a.slot[a.nsrc - 1 - j]].r;
+                if (j < a.nsrc) val = (float)st->rec[a.slot[a.nsrc - 1 - j]].r;
             } else if (j < 6) {
                 if (j - 3 < a.nsrc) {
                     const DevRecord& r = st->rec[a.slot[a.nsrc - 1 - (j - 3)]];
-                    val = (double)a.T * (r.q_in - r.q_out);
+                    val = (float)((double)a.T * (r.q_in - r.q_out));
                 }
             } else {
-                val = (double)a.nsrc / (double)a.prm.K;
+                val = (float)a.nsrc / (float)a.prm.K;
             }
         }
         hs.phi[t] = val;
     }
     if (t == 0) {
         // Eq. 4: alpha = clip(|q_{t-1}-q_t| / (|q_{a-1}-q_a| + eps), alpha_min, alpha_max)
-        const double raw = fabs(a.q_next - a.q_k) / (fabs(st->q_a_out - st->q_a_in) + a.prm.eps);
-        hs.alpha = fmin(fmax(raw, a.prm.alpha_min), a.prm.alpha_max);
+        const float raw = (float)fabs(a.q_next - a.q_k) / ((float)fabs(st->q_a_out - st->q_a_in) + (float)a.prm.eps);
+        hs.alpha = fminf(fmaxf(raw, (float)a.prm.alpha_min), (float)a.prm.alpha_max);
     }
     __syncthreads();
     if (K == 0) return;
 
     // Eq. 3: similarities with the records' lifted inputs
     {
-        double v[K + 1];
-        const double ph = (t < kSummary) ? hs.phi[t] : 0.0;
+        float v[K + 1];
+        const float ph = (t < kSummary) ? hs.phi[t] : 0.f;
 #pragma unroll
-        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? ph * st->rec[a.slot[i]].s_in[t] : 0.0;
+        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? ph * st->rec[a.slot[i]].s_in[t] : 0.f;
         v[K] = ph * ph;
         reduce256<K + 1>(v, hs.scratch, hs.red);
     }
     if (t == 0) {
-        const double nphi = sqrt(hs.red[K]);
+        const float nphi = sqrtf(hs.red[K]);
         const bool filter = !(a.prm.flags & WDC_ABL_NO_SUPPORT);   // w/o support: N_t = whole bank
+        const float gq = (float)a.prm.gamma_q, inv_tin = 1.0f / (float)a.prm.tau_in;
         int nc = 0;
-        double mx = -INFINITY;
-        double ell[K > 0 ? K : 1];
+        float mx = -INFINITY;
+        float ell[K > 0 ? K : 1];
 #pragma unroll
         for (int i = 0; i < K; ++i) {
             const DevRecord& r = st->rec[a.slot[i]];
-            const double s = (nphi == 0.0 || r.n_in == 0.0) ? 0.0 : hs.red[i] / (nphi * r.n_in);
+            const float s = (nphi == 0.f || r.n_in == 0.f) ? 0.f : hs.red[i] / (nphi * r.n_in);
             const double dq = a.q_k - r.q_in;
             hs.sim_in[i] = s;
-            const int c = !filter || ((s >= a.prm.sim_min) && (fabs(dq) <= a.prm.q_gap_max));
+            const int c = !filter || ((s >= (float)a.prm.sim_min) && (fabs(dq) <= a.prm.q_gap_max));
             hs.compat[i] = c;
-            ell[i] = (s - a.prm.gamma_q * dq * dq) / a.prm.tau_in;
-            if (c) { ++nc; mx = fmax(mx, ell[i]); }
+            const float dqf = (float)dq;
+            ell[i] = (s - gq * dqf * dqf) * inv_tin;
+            if (c) { ++nc; mx = fmaxf(mx, ell[i]); }
         }
-        double tot = 0.0;
+        float tot = 0.f;
 #pragma unroll
         for (int i = 0; i < K; ++i) {
-            hs.pi[i] = hs.compat[i] ? exp(ell[i] - mx) : 0.0;
+            hs.pi[i] = hs.compat[i] ? expf(ell[i] - mx) : 0.f;
             tot += hs.pi[i];
         }
 #pragma unroll
-        for (int i = 0; i < K; ++i) hs.pi[i] = (nc > 0) ? hs.pi[i] / tot : 0.0;
+        for (int i = 0; i < K; ++i) hs.pi[i] = (nc > 0) ? hs.pi[i] / tot : 0.f;
         hs.n_compat = nc;
         hs.supported = filter ? (nc >= a.prm.min_support) : 1;
     }
     __syncthreads();
     // Eq. 4 in summary space, then Eq. 5 similarities with the lifted outputs
     {
-        double v[K + 1];
-        double hv = 0.0;
+        float v[K + 1];
+        float hv = 0.f;
         if (t < kSummary) {
-            double acc = 0.0;
+            float acc = 0.f;
 #pragma unroll
             for (int i = 0; i < K; ++i)
-                if (hs.pi[i] != 0.0) acc += hs.pi[i] * st->rec[a.slot[i]].s_dphi[t];
-            hv = hs.phi[t] + hs.alpha * acc;
+                if (hs.pi[i] != 0.f) acc = fmaf(hs.pi[i], st->rec[a.slot[i]].s_dphi[t], acc);
+            hv = fmaf(hs.alpha, acc, hs.phi[t]);
             hs.hat[t] = hv;
         }
 #pragma unroll
-        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? hv * st->rec[a.slot[i]].s_out[t] : 0.0;
+        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? hv * st->rec[a.slot[i]].s_out[t] : 0.f;
         v[K] = hv * hv;
         reduce256<K + 1>(v, hs.scratch, hs.red);
     }
     if (t == 0) {
-        const double nh = sqrt(hs.red[K]);
-        double mx = -INFINITY;
-        double e[K > 0 ? K : 1];
+        const float nh = sqrtf(hs.red[K]);
+        const float inv_tau = 1.0f / (float)a.prm.tau_obs;
+        float mx = -INFINITY;
+        float e[K > 0 ? K : 1];
 #pragma unroll
         for (int i = 0; i < K; ++i) {
             const DevRecord& r = st->rec[a.slot[i]];
-            const double s = (nh == 0.0 || r.n_out == 0.0) ? 0.0 : hs.red[i] / (nh * r.n_out);
+            const float s = (nh == 0.f || r.n_out == 0.f) ? 0.f : hs.red[i] / (nh * r.n_out);
             hs.sim_out[i] = s;
-            e[i] = s / a.prm.tau_obs;
-            mx = fmax(mx, e[i]);
+            e[i] = s * inv_tau;
+            mx = fmaxf(mx, e[i]);
         }
-        double tot = 0.0;
+        float tot = 0.f;
 #pragma unroll
-        for (int i = 0; i < K; ++i) { e[i] = exp(e[i] - mx); tot += e[i]; }
+        for (int i = 0; i < K; ++i) { e[i] = expf(e[i] - mx); tot += e[i]; }
+        const float inv = 1.0f / tot;
 #pragma unroll
-        for (int i = 0; i < K; ++i) hs.kappa[i] = e[i] / tot;
+        for (int i = 0; i < K; ++i) hs.kappa[i] = e[i] * inv;
     }
     __syncthreads();
     if (a.prm.flags & WDC_ABL_LINEAR_OBS) linear_readout<K>(a, hs);
 }
 
+// Per-block scalar slots: the stream's five sums and the non-finite count.
+constexpr int kScalars = 6;
+// Most blocks one pass launch may have (the final reduction's register tile).
+constexpr int kMaxPassBlocks = 256;
+
 struct PassShared {
     float wb[2][kWarps][kSketch];     // per-warp bucket rows (2 sketches for the stats pass)
-    double blk[kWarps][8];
-    double fin[kPartials];
+    float blk[kWarps][kScalars];
+    float fin[kPartials];
     int last;
 };
+
+// Sum over the 32 warps' rows of one bucket, in a fixed pairwise order.
+__device__ __forceinline__ float sum_warp_rows(const float (&rows)[kWarps][kSketch], int b) {
+    float x[kWarps];
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) x[w] = rows[w][b];
+#pragma unroll
+    for (int h = kWarps / 2; h; h >>= 1)
+#pragma unroll
+        for (int w = 0; w < h; ++w) x[w] += x[w + h];
+    return x[0];
+}
 
 template <int MODE, int K>
 __device__ __forceinline__ void pass_body(const PassArgs& a) {
@@ -314,11 +367,11 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
         skip_head<K>(a, hs);
         do_stream = (K > 0) && hs.supported;
 #pragma unroll
-        for (int i = 0; i < K; ++i) kap[i] = (float)hs.kappa[i];
+        for (int i = 0; i < K; ++i) kap[i] = hs.kappa[i];
     } else if (MODE == kModeSecant) {
         skip_head<0>(a, hs);               // lift summary and alpha only: no retrieval
         do_stream = a.nsrc > 0;
-        alpha_f = (float)hs.alpha;
+        alpha_f = hs.alpha;
     } else if (MODE == kModeObserve) {
 #pragma unroll
         for (int i = 0; i < K; ++i) kap[i] = a.kappa[i];
@@ -327,8 +380,9 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
         __syncthreads();
     }
 
-    // per-thread accumulators: fp32 over up to 16 runs, flushed to fp64
-    double acc[5] = {0, 0, 0, 0, 0};
+    // per-thread accumulators: plain fp32 over up to 16 runs (64 terms), then
+    // a compensated fp32 outer sum
+    float acc[5] = {0, 0, 0, 0, 0}, cmp[5] = {0, 0, 0, 0, 0};
     float fac[5] = {0, 0, 0, 0, 0};
     int nonfinite = 0;
     int since = 0;
@@ -337,7 +391,64 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
     if (do_stream) {
         const long long gw = (long long)blockIdx.x * kWarps + warp;
         const long long stride = (long long)gridDim.x * kWarps;
-        for (long long r = gw; r < nruns; r += stride) {
+        long long r = gw;
+        if constexpr ((MODE == kModeSkip || MODE == kModeObserve) && K > 0) {
+            // two full runs per iteration: both runs' loads are in flight
+            // together (a bank of two records alone keeps too few bytes in
+            // flight per SM to cover the HBM latency)
+            auto stats = [&](const float4& zh, const float4& za, long long base, long long rr) {
+                const float ov[4] = {zh.x, zh.y, zh.z, zh.w};
+                const float av[4] = {za.x, za.y, za.z, za.w};
+                float sg = 0.f;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float d = ov[e] - av[e];
+                    sg += signed_term((uint32_t)(base + e), seed, ov[e]);
+                    fac[0] = fmaf(ov[e], ov[e], fac[0]);
+                    fac[1] = fmaf(d, d, fac[1]);
+                    nonfinite += isfinite(ov[e]) ? 0 : 1;
+                }
+                sg = warp_sum_f(sg);
+                if (lane == 0) ps.wb[0][warp][(int)(rr % kSketch)] += sg;
+            };
+            for (; r + stride < full; r += 2 * stride) {
+                const long long b0 = r * kRun + lane * 4, b1 = (r + stride) * kRun + lane * 4;
+                float4 x0[K], x1[K], za0, za1;
+#pragma unroll
+                for (int i = 0; i < K; ++i) {
+                    x0[i] = __ldg(reinterpret_cast<const float4*>(a.src[i] + b0));
+                    x1[i] = __ldg(reinterpret_cast<const float4*>(a.src[i] + b1));
+                }
+                if constexpr (MODE == kModeObserve) {
+                    za0 = __ldg(reinterpret_cast<const float4*>(a.anchor + b0));
+                    za1 = __ldg(reinterpret_cast<const float4*>(a.anchor + b1));
+                } else {
+                    za0 = x0[K - 1];             // the anchor is the newest record
+                    za1 = x1[K - 1];
+                }
+                float4 z0, z1;
+                z0.x = kap[0] * x0[0].x; z0.y = kap[0] * x0[0].y; z0.z = kap[0] * x0[0].z; z0.w = kap[0] * x0[0].w;
+                z1.x = kap[0] * x1[0].x; z1.y = kap[0] * x1[0].y; z1.z = kap[0] * x1[0].z; z1.w = kap[0] * x1[0].w;
+#pragma unroll
+                for (int i = 1; i < K; ++i) {
+                    z0.x = fmaf(kap[i], x0[i].x, z0.x); z0.y = fmaf(kap[i], x0[i].y, z0.y);
+                    z0.z = fmaf(kap[i], x0[i].z, z0.z); z0.w = fmaf(kap[i], x0[i].w, z0.w);
+                    z1.x = fmaf(kap[i], x1[i].x, z1.x); z1.y = fmaf(kap[i], x1[i].y, z1.y);
+                    z1.z = fmaf(kap[i], x1[i].z, z1.z); z1.w = fmaf(kap[i], x1[i].w, z1.w);
+                }
+                *reinterpret_cast<float4*>(a.out + b0) = z0;
+                *reinterpret_cast<float4*>(a.out + b1) = z1;
+                stats(z0, za0, b0, r);
+                stats(z1, za1, b1, r + stride);
+                since += 2;
+                if (since >= 16) {
+#pragma unroll
+                    for (int j = 0; j < 5; ++j) { kahan_add(acc[j], cmp[j], fac[j]); fac[j] = 0.f; }
+                    since = 0;
+                }
+            }
+        }
+        for (; r < nruns; r += stride) {
             const long long base = r * kRun + lane * 4;
             float o[4], sa[4], sb[4];   // o: primary value, sa/sb: stats-pass anchor
             bool valid[4];
@@ -417,7 +528,7 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
                     sb[0] = z.x; sb[1] = z.y; sb[2] = z.z; sb[3] = z.w;
                     if (a.zcf) {
                         const float4 c = *reinterpret_cast<const float4*>(a.zcf + base);
-                        fac[0] += fabsf(ze.x - c.x) + fabsf(ze.y - c.y) + fabsf(ze.z - c.z) + fabsf(ze.w - c.w);
+                        fac[0] += (fabsf(ze.x - c.x) + fabsf(ze.y - c.y)) + (fabsf(ze.z - c.z) + fabsf(ze.w - c.w));
                     }
                 } else if constexpr (MODE == kModeStats) {
                     const float4 z = __ldg(reinterpret_cast<const float4*>(a.src[0] + base));
@@ -487,19 +598,19 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
                 const uint32_t idx = (uint32_t)(base + e);
                 sg += signed_term(idx, seed, x);
                 if (MODE == kModeSkip || MODE == kModeObserve || MODE == kModeSecant || MODE == kModeResidual) {
-                    fac[0] += x * x;
-                    fac[1] += d * d;
+                    fac[0] = fmaf(x, x, fac[0]);
+                    fac[1] = fmaf(d, d, fac[1]);
                     nonfinite += isfinite(x) ? 0 : 1;
                 } else if (MODE == kModeAnchor) {
                     fac[1] += fabsf(x);
-                    fac[2] += x * x;
-                    fac[3] += d * d;
+                    fac[2] = fmaf(x, x, fac[2]);
+                    fac[3] = fmaf(d, d, fac[3]);
                     const float dz = x - sb[e];
-                    fac[4] += dz * dz;
+                    fac[4] = fmaf(dz, dz, fac[4]);
                 } else {
-                    fac[0] += x * x;
-                    fac[1] += d * d;
-                    fac[2] += sa[e] * sa[e];
+                    fac[0] = fmaf(x, x, fac[0]);
+                    fac[1] = fmaf(d, d, fac[1]);
+                    fac[2] = fmaf(sa[e], sa[e], fac[2]);
                     sg2 += signed_term(idx, seed, sa[e]);
                 }
             }
@@ -510,38 +621,43 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
                 sg2 = warp_sum_f(sg2);
                 if (lane == 0) ps.wb[1][warp][bucket] += sg2;
             }
-            if (++since == 16) {
+            if (++since >= 16) {
 #pragma unroll
-                for (int j = 0; j < 5; ++j) { acc[j] += (double)fac[j]; fac[j] = 0.f; }
+                for (int j = 0; j < 5; ++j) { kahan_add(acc[j], cmp[j], fac[j]); fac[j] = 0.f; }
                 since = 0;
             }
         }
     }
+    float sum[kScalars];
 #pragma unroll
-    for (int j = 0; j < 5; ++j) acc[j] += (double)fac[j];
-    double cnt = (double)nonfinite;
+    for (int j = 0; j < 5; ++j) {
+        kahan_add(acc[j], cmp[j], fac[j]);
+        sum[j] = acc[j] - cmp[j];
+    }
+    sum[5] = (float)nonfinite;
 
-    // block combination (fixed order)
+    // block combination (fixed order): warp trees, then a tree over the warps
 #pragma unroll
-    for (int j = 0; j < 5; ++j) acc[j] = warp_sum_d(acc[j]);
-    cnt = warp_sum_d(cnt);
+    for (int j = 0; j < kScalars; ++j) sum[j] = warp_sum_f(sum[j]);
     if (lane == 0) {
 #pragma unroll
-        for (int j = 0; j < 5; ++j) ps.blk[warp][j] = acc[j];
-        ps.blk[warp][5] = cnt;
+        for (int j = 0; j < kScalars; ++j) ps.blk[warp][j] = sum[j];
     }
     __syncthreads();
-    double* part = a.partials + (size_t)blockIdx.x * kPartials;
-    if (t < 2 * kSketch) {
-        const int s = t / kSketch, b = t % kSketch;
-        double v = 0.0;
-        for (int w = 0; w < kWarps; ++w) v += (double)ps.wb[s][w][b];
-        part[t] = v;
-    } else if (t < 2 * kSketch + 6) {
-        const int j = t - 2 * kSketch;
-        double v = 0.0;
-        for (int w = 0; w < kWarps; ++w) v += ps.blk[w][j];
-        part[t] = v;
+    // partials are value-major, [kPartials][gridDim.x], so the last block
+    // reads each value's per-block entries with coalesced loads
+    const int G = gridDim.x;
+    float* part = a.partials + blockIdx.x;
+    const int nsk = (MODE == kModeStats) ? 2 : 1;       // sketches reduced by this mode
+    if (t < nsk * kSketch) {
+        part[(size_t)t * G] = sum_warp_rows(ps.wb[t / kSketch], t % kSketch);
+    } else if (warp == kWarps - 1) {
+        // the last warp: one lane per warp row, a butterfly per scalar
+#pragma unroll
+        for (int j = 0; j < kScalars; ++j) {
+            const float v = warp_sum_f(ps.blk[lane][j]);
+            if (lane == 0) part[(size_t)(2 * kSketch + j) * G] = v;
+        }
     }
     __threadfence();
     __syncthreads();
@@ -553,18 +669,36 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
     if (!ps.last) return;
     __threadfence();
 
-    // final reduction over blocks, fixed order: 4 threads per value
+    // final reduction over the blocks, fixed order: each warp takes values
+    // w, w + 32, ...; lane l sums blocks l, l + 32, ... (G <= kMaxPassBlocks),
+    // then a butterfly.  All of a warp's loads for four values are issued
+    // before any is added (one L2 round trip per four values).
     {
-        // the per-warp bucket rows are no longer needed: reuse them as scratch
-        double (*tmp)[kPartials] = reinterpret_cast<double (*)[kPartials]>(&ps.wb[0][0][0]);
-        const int v = t % 256, g = t / 256;
-        if (v < 2 * kSketch + 6) {
-            double s = 0.0;
-            for (int b = g; b < (int)gridDim.x; b += 4) s += __ldcg(a.partials + (size_t)b * kPartials + v);
-            tmp[g][v] = s;
+        const int nv = nsk * kSketch;             // sketch values, then the scalars at 2 * kSketch
+        const int total = nv + kScalars;
+        for (int v0 = warp; v0 < total; v0 += 4 * kWarps) {
+            float x[4][kMaxPassBlocks / 32];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int vi = v0 + j * kWarps;
+                const int v = vi < nv ? vi : 2 * kSketch + (vi - nv);
+#pragma unroll
+                for (int i = 0; i < kMaxPassBlocks / 32; ++i) {
+                    const int b = lane + 32 * i;
+                    x[j][i] = (vi < total && b < G) ? __ldcg(a.partials + (size_t)v * G + b) : 0.f;
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int vi = v0 + j * kWarps;
+                const int v = vi < nv ? vi : 2 * kSketch + (vi - nv);
+                float s = 0.f;
+#pragma unroll
+                for (int i = 0; i < kMaxPassBlocks / 32; ++i) s += x[j][i];
+                s = warp_sum_f(s);
+                if (lane == 0 && vi < total) ps.fin[v] = s;
+            }
         }
-        __syncthreads();
-        if (t < 2 * kSketch + 6) ps.fin[t] = ((tmp[0][t] + tmp[1][t]) + tmp[2][t]) + tmp[3][t];
         __syncthreads();
     }
     if (t == 0) *a.counter = 0u;
@@ -581,8 +715,8 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
     }
 
     DevState* st = a.st;
-    const double N = (double)n;
-    const double* fin = ps.fin;
+    const float N = (float)n;
+    const float* fin = ps.fin;
     const int sc0 = 2 * kSketch;   // scalar sums start here
 
     if (MODE == kModeStats) {
@@ -602,28 +736,33 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
         if (t < kSummary) st->s_phi[t] = hs.phi[t];
         // the secant needs no retrieval: its support term holds with a non-empty bank
         const int supported = (MODE == kModeSecant) ? (a.nsrc > 0) : ((K > 0) && hs.supported);
-        const int finite = supported && (fin[sc0 + 5] == 0.0);
+        const int finite = supported && (fin[sc0 + 5] == 0.f);
         __shared__ int s_dec;
         if (t == 0) {
+            // controller tail in fp32; the stored risk R stays fp64
             const ParamsDev& p = a.prm;
-            const double d_z = sqrt(st->cur_sumsq_anchor / N) / (sqrt(st->anchor_sumsq / N) + p.eps);
-            const double d_age = (double)a.age;
-            const double d_phase = fabs(a.q_next - st->q_a_out);
-            double dc = 0.0, dd = 0.0, uc = 0.0, ud = 0.0;
+            const float eps = (float)p.eps;
+            const float d_z = sqrtf((float)st->cur_sumsq_anchor / N) / (sqrtf((float)st->anchor_sumsq / N) + eps);
+            const float d_age = (float)a.age;
+            const float d_phase = (float)fabs(a.q_next - st->q_a_out);
+            float dc = 0.f, dd = 0.f, uc = 0.f, ud = 0.f;
             for (int j = 0; j < 4; ++j) {
-                dc += (a.cam[j] - st->cam_a[j]) * (a.cam[j] - st->cam_a[j]);
-                dd += (a.depth[j] - st->depth_a[j]) * (a.depth[j] - st->depth_a[j]);
-                uc += a.cam[j] * a.cam[j];
-                ud += a.depth[j] * a.depth[j];
+                const float cj = (float)a.cam[j], dj = (float)a.depth[j];
+                const float ca = (float)st->cam_a[j], da = (float)st->depth_a[j];
+                dc = fmaf(cj - ca, cj - ca, dc);
+                dd = fmaf(dj - da, dj - da, dd);
+                uc = fmaf(cj, cj, uc);
+                ud = fmaf(dj, dj, ud);
             }
-            const double pt = p.w_z * d_z + p.w_age * d_age + p.w_phase * d_phase + p.w_cam * sqrt(dc) +
-                              p.w_depth * sqrt(dd);
-            const double d_hat = st->eta * pt;
-            const double w = (p.flags & WDC_ABL_NO_IMPACT)
-                                 ? 1.0
-                                 : fmin(2.0, 1.0 + p.a_cam * sqrt(uc) + p.a_depth * sqrt(ud) + p.a_phase * a.q_k);
-            const double delta = w * d_hat;
-            const double R_cand = p.lam * st->R + delta;
+            const float pt = (float)p.w_z * d_z + (float)p.w_age * d_age + (float)p.w_phase * d_phase +
+                             (float)p.w_cam * sqrtf(dc) + (float)p.w_depth * sqrtf(dd);
+            const float d_hat = (float)st->eta * pt;
+            const float w = (p.flags & WDC_ABL_NO_IMPACT)
+                                ? 1.f
+                                : fminf(2.f, 1.f + (float)p.a_cam * sqrtf(uc) + (float)p.a_depth * sqrtf(ud) +
+                                                 (float)p.a_phase * (float)a.q_k);
+            const float delta = w * d_hat;
+            const double R_cand = p.lam * st->R + (double)delta;
             const bool avail = (a.nsrc > 0) && (a.age <= p.max_age) &&
                                (fabs(a.q_k - st->q_a_out) <= p.q_gap_max) && finite && supported &&
                                (a.k >= p.n_init_exact) && (a.k < a.T - p.n_final_exact);
@@ -646,8 +785,8 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
             o.d_z = d_z;
             o.r = 0.0;
             for (int i = 0; i < kMaxBank; ++i) {
-                o.kappa[i] = (i < K) ? hs.kappa[i] : 0.0;
-                o.pi[i] = (i < K) ? hs.pi[i] : 0.0;
+                o.kappa[i] = (i < K) ? hs.kappa[i] : 0.f;
+                o.pi[i] = (i < K) ? hs.pi[i] : 0.f;
             }
             if (dec) st->R = R_cand;
             if (a.graph) {
@@ -677,44 +816,49 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
         return;
     }
 
-    // ---- anchor pass tail (MODE == kModeAnchor)
-    __shared__ double s_rms[2];
+    // ---- anchor pass tail (MODE == kModeAnchor): fp32 arithmetic, fp64 state
+    __shared__ float s_rms[2];
     if (t == 0) {
         const ParamsDev& p = a.prm;
+        const float eps = (float)p.eps;
         st->R = p.lam * st->R;
         double d_cf = nan("");
         if (a.zcf != nullptr && st->cand_k == a.k && st->cand_supported && st->cand_finite) {
-            d_cf = (fin[sc0 + 0] / N) / (fin[sc0 + 1] / N + p.eps);
+            const float dcf = (fin[sc0 + 0] / N) / (fin[sc0 + 1] / N + eps);
+            d_cf = dcf;
             if (!(p.flags & WDC_ABL_NO_CALIB)) {
-                const double v = p.beta_d * st->eta + (1.0 - p.beta_d) * d_cf / (st->cand_p + p.eps);
-                st->eta = fmin(fmax(v, p.eta_min), p.eta_max);
+                const float bd = (float)p.beta_d;
+                const float v = bd * (float)st->eta + (1.f - bd) * dcf / ((float)st->cand_p + eps);
+                st->eta = fminf(fmaxf(v, (float)p.eta_min), (float)p.eta_max);
             }
         }
         st->out.d_cf = d_cf;
         st->out.R = st->R;
         st->out.eta = st->eta;
-        const double r = sqrt(fin[sc0 + 4] / N) / (sqrt(st->cur_sumsq / N) + p.eps);
+        const float r = sqrtf(fin[sc0 + 4] / N) / (sqrtf((float)st->cur_sumsq / N) + eps);
         st->out.r = r;
         st->rec[a.ins_slot].r = r;
-        s_rms[0] = sqrt(fin[sc0 + 2] / N);
-        s_rms[1] = sqrt(fin[sc0 + 3] / N);
+        s_rms[0] = sqrtf(fin[sc0 + 2] / N);
+        s_rms[1] = sqrtf(fin[sc0 + 3] / N);
     }
     __syncthreads();
     DevRecord& rec = st->rec[a.ins_slot];
-    const double sc = sqrt((double)kSketch / N);
-    double so = 0.0, si = 0.0;
+    const float sc = sqrtf((float)kSketch / N);
+    const float eps_nu = (float)a.prm.eps_nu;
+    const bool no_cond = a.prm.flags & WDC_ABL_NO_COND;
+    float so = 0.f, si = 0.f;
     if (t < kSummary) {
         if (t < kSketch) {
-            so = sc * fin[t] / (s_rms[0] + a.prm.eps_nu);
+            so = sc * fin[t] / (s_rms[0] + eps_nu);
         } else if (t < 2 * kSketch) {
             const int b = t - kSketch;
-            so = sc * (fin[b] - st->anchor_S[b]) / (s_rms[1] + a.prm.eps_nu);
+            so = sc * (fin[b] - st->anchor_S[b]) / (s_rms[1] + eps_nu);
         } else if (t < kOffDepth) {
-            so = (a.prm.flags & WDC_ABL_NO_COND) ? 0.0 : a.cam[t - kOffCam];
+            so = no_cond ? 0.f : (float)a.cam[t - kOffCam];
         } else if (t < kOffQ) {
-            so = (a.prm.flags & WDC_ABL_NO_COND) ? 0.0 : a.depth[t - kOffDepth];
+            so = no_cond ? 0.f : (float)a.depth[t - kOffDepth];
         } else if (t == kOffQ) {
-            so = a.q_next;
+            so = (float)a.q_next;
         } else {
             so = st->s_phi[t];     // pre-insertion history h(H)
         }
@@ -727,7 +871,7 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
         rec.s_dphi[t] = so - si;
     }
     {
-        double v[2] = {si * si, so * so};
+        float v[2] = {si * si, so * so};
         reduce256<2>(v, hs.scratch, hs.red);
     }
     if (t < kSketch) {
@@ -735,8 +879,8 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
         st->cur_S[t] = fin[t];
     }
     if (t == 0) {
-        rec.n_in = sqrt(hs.red[0]);
-        rec.n_out = sqrt(hs.red[1]);
+        rec.n_in = sqrtf(hs.red[0]);
+        rec.n_out = sqrtf(hs.red[1]);
         rec.q_in = a.q_k;
         rec.q_out = a.q_next;
         for (int j = 0; j < 4; ++j) {
@@ -770,12 +914,113 @@ void launch_skip(const PassArgs& a, int grid, cudaStream_t s, bool residual) {
     else pass_kernel<kModeSkip, K><<<grid, kThreads, 0, s>>>(a);
 }
 
+// Reductions of three latents for the synthetic diagnostics
+// (wdc_latent_pair_stats): out[0] = sum (a-c)^2, out[1] = sum (b-c)^2,
+// out[2] = sum (a-c)(b-c), out[3] = sum (a-b)^2, out[4] = sum b^2, with c = 0
+// when null.  The same deterministic scheme as the fused passes: per-thread
+// fp32 chains with a compensated outer sum, warp and block trees, value-major
+// per-block partials and a last-block final tree.
+constexpr int kPairStats = 5;
+__global__ void __launch_bounds__(kThreads, 1)
+    pair_stats_kernel(const float* __restrict__ a, const float* __restrict__ b, const float* __restrict__ c,
+                      long long n, float* partials, unsigned* counter, double* out) {
+    __shared__ float blk[kWarps][kPairStats];
+    __shared__ int last;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    float acc[kPairStats] = {}, cmp[kPairStats] = {}, fac[kPairStats] = {};
+    int since = 0;
+    const long long n4 = n / 4;
+    const long long stride = (long long)gridDim.x * kThreads;
+    for (long long i = (long long)blockIdx.x * kThreads + t; i < n4 + (n % 4 ? 1 : 0); i += stride) {
+        float av[4] = {0, 0, 0, 0}, bv[4] = {0, 0, 0, 0}, cv[4] = {0, 0, 0, 0};
+        if (i < n4) {
+            const float4 x = __ldg(reinterpret_cast<const float4*>(a) + i);
+            const float4 y = __ldg(reinterpret_cast<const float4*>(b) + i);
+            av[0] = x.x; av[1] = x.y; av[2] = x.z; av[3] = x.w;
+            bv[0] = y.x; bv[1] = y.y; bv[2] = y.z; bv[3] = y.w;
+            if (c) {
+                const float4 z = __ldg(reinterpret_cast<const float4*>(c) + i);
+                cv[0] = z.x; cv[1] = z.y; cv[2] = z.z; cv[3] = z.w;
+            }
+        } else {
+            for (int e = 0; e < 4; ++e) {
+                const long long idx = 4 * i + e;
+                if (idx < n) {
+                    av[e] = a[idx];
+                    bv[e] = b[idx];
+                    cv[e] = c ? c[idx] : 0.f;
+                }
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float u = av[e] - cv[e], v = bv[e] - cv[e], d = av[e] - bv[e];
+            fac[0] = fmaf(u, u, fac[0]);
+            fac[1] = fmaf(v, v, fac[1]);
+            fac[2] = fmaf(u, v, fac[2]);
+            fac[3] = fmaf(d, d, fac[3]);
+            fac[4] = fmaf(bv[e], bv[e], fac[4]);
+        }
+        if (++since >= 16) {
+#pragma unroll
+            for (int j = 0; j < kPairStats; ++j) { kahan_add(acc[j], cmp[j], fac[j]); fac[j] = 0.f; }
+            since = 0;
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < kPairStats; ++j) {
+        kahan_add(acc[j], cmp[j], fac[j]);
+        const float v = warp_sum_f(acc[j] - cmp[j]);
+        if (lane == 0) blk[warp][j] = v;
+    }
+    __syncthreads();
+    const int G = gridDim.x;
+    if (warp == 0) {
+#pragma unroll
+        for (int j = 0; j < kPairStats; ++j) {
+            const float v = warp_sum_f(blk[lane][j]);
+            if (lane == 0) partials[(size_t)j * G + blockIdx.x] = v;
+        }
+    }
+    __threadfence();
+    __syncthreads();
+    if (t == 0) last = (atomicAdd(counter, 1u) == (unsigned)G - 1);
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    if (warp < kPairStats) {
+        float x[kMaxPassBlocks / 32];
+#pragma unroll
+        for (int i = 0; i < kMaxPassBlocks / 32; ++i) {
+            const int blkid = lane + 32 * i;
+            x[i] = blkid < G ? __ldcg(partials + (size_t)warp * G + blkid) : 0.f;
+        }
+        float v = 0.f;
+#pragma unroll
+        for (int i = 0; i < kMaxPassBlocks / 32; ++i) v += x[i];
+        v = warp_sum_f(v);
+        if (lane == 0) out[warp] = v;
+    }
+    if (t == 0) *counter = 0u;
+}
+
 }  // namespace
+
+wdc_status launch_pair_stats(Ctx* c, const float* a, const float* b, const float* cz, double* out_dev,
+                             cudaStream_t s) {
+    const int grid = pass_grid(c);
+    LaunchScope ls(c, WDC_K_OTHER, s);
+    pair_stats_kernel<<<grid, kThreads, 0, s>>>(a, b, cz, (long long)c->n, c->partials, c->counter, out_dev);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("pair statistics launch: ") + cudaGetErrorString(e));
+    return WDC_OK;
+}
 
 int pass_grid(const Ctx* c) {
     const long long nruns = ((long long)c->n + kRun - 1) / kRun;
     long long g = (nruns + kWarps - 1) / kWarps;
     if (g > c->num_sms) g = c->num_sms;
+    if (g > kMaxPassBlocks) g = kMaxPassBlocks;
     if (g < 1) g = 1;
     return (int)g;
 }
@@ -895,7 +1140,8 @@ namespace wdc {
 namespace {
 
 constexpr int kNoAllocMaxBlocks = 256;                       // CTAs the scratch can serve
-constexpr size_t kNoAllocPartialBytes = (size_t)kNoAllocMaxBlocks * kPartials * sizeof(double);
+constexpr size_t kNoAllocPartialBytes = (size_t)kNoAllocMaxBlocks * kPartials * sizeof(float);
+static_assert(kNoAllocMaxBlocks <= kMaxPassBlocks, "the final reduction covers at most kMaxPassBlocks blocks");
 constexpr size_t kNoAllocBytes = kNoAllocPartialBytes + 256;  // + the done counter
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
 
@@ -962,7 +1208,7 @@ extern "C" wdc_status wdc_observe_noalloc(const float* const* z_out, int K, cons
     a.anchor = z_a;
     a.out = z_hat;
     a.prm.seed = sketch_seed;
-    a.partials = reinterpret_cast<double*>(d.scratch);
+    a.partials = reinterpret_cast<float*>(d.scratch);
     a.counter = reinterpret_cast<unsigned*>(d.scratch + kNoAllocPartialBytes);
     a.stats_out = stats;
     const long long nruns = ((long long)n + kRun - 1) / kRun;

@@ -26,10 +26,13 @@ constexpr int kOffH = kOffQ + 1;
 enum : unsigned { kErrTimeout = 1u, kErrBounds = 2u, kErrTmem = 4u };
 
 // ---------------------------------------------------------------- device state
-// One bank record; summaries in fp64 (section "Local Lifted Evolution").
+// One bank record (section "Local Lifted Evolution").  The summaries are
+// fp32: the step kernels do their per-element and reduction arithmetic in
+// fp32 (GB300's fp64 rate is a small fraction of its fp32 rate); the scalar
+// fields stay fp64.
 struct DevRecord {
-    double s_in[kSummary], s_out[kSummary], s_dphi[kSummary];
-    double n_in, n_out;           // Euclidean norms of s_in and s_out
+    float s_in[kSummary], s_out[kSummary], s_dphi[kSummary];
+    float n_in, n_out;            // Euclidean norms of s_in and s_out
     double q_in, q_out, r;
     double cam[4], depth[4];
 };
@@ -48,12 +51,15 @@ struct DevState {
     double q_a_in, q_a_out;
     double cam_a[4], depth_a[4];
     DevRecord rec[kMaxBank];                       // indexed by ring slot
-    double cur_S[kSketch], cur_sumsq, cur_sumsq_anchor;   // raw sums over the current latent
-    double anchor_S[kSketch], anchor_sumsq;
-    double s_phi[kSummary];                        // summary of the current state (this step)
+    float cur_S[kSketch];                          // raw signed bucket sums over the current latent
+    double cur_sumsq, cur_sumsq_anchor;            // sum z^2, sum (z - z_a)^2
+    float anchor_S[kSketch];
+    double anchor_sumsq;
+    float s_phi[kSummary];                         // summary of the current state (this step)
     int cand_k, cand_supported, cand_finite;
     double cand_p;
-    double cand_S[kSketch], cand_sumsq, cand_sumsq_anchor;
+    float cand_S[kSketch];
+    double cand_sumsq, cand_sumsq_anchor;
     StepOut out;
     // discrete state of the graph rollout (device-resident mirror of the
     // host's ring head, bank size and age)
@@ -93,7 +99,7 @@ struct PassArgs {
     double cam[4], depth[4];
     ParamsDev prm;
     DevState* st;
-    double* partials;                  // [gridDim.x][kPartials]
+    float* partials;                   // [kPartials][gridDim.x] (value-major)
     unsigned* counter;
     unsigned* err;
     float kappa[kMaxBank];             // observe: caller-given weights
@@ -120,9 +126,10 @@ struct Ctx {
 
     // memory
     DevState* st = nullptr;
-    double* partials = nullptr;
+    float* partials = nullptr;
     unsigned* counter = nullptr;
     unsigned* err = nullptr;
+    double* pstat = nullptr;           // wdc_latent_pair_stats output (5 doubles)
     StepOut* out_host = nullptr;       // pinned
     DevState* st_host = nullptr;       // pinned staging of the device state (reset / get / set)
     float* bank[kMaxBank] = {};
@@ -186,6 +193,9 @@ int pass_grid(const Ctx* c);
 wdc_status launch_pass(Ctx* c, int mode, const PassArgs& a, cudaStream_t s);
 wdc_status launch_pass_ptr(Ctx* c, int mode, int K, const PassArgs* pa, cudaStream_t s);
 ParamsDev to_dev_params(const wdc_cache_params& p);
+// wdc_latent_pair_stats: five sums over three latents into out_dev (device, 5 doubles)
+wdc_status launch_pair_stats(Ctx* c, const float* a, const float* b, const float* cz, double* out_dev,
+                             cudaStream_t s);
 
 // dit.cu
 wdc_status dit_create(Ctx* c);

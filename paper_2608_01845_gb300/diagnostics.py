@@ -2,9 +2,12 @@
 and Observations", Fig. 2; section "Transition Risk Controller", Fig. 3).
 
 Every transition runs through the C ABI (the fused step passes and the
-denoiser); this module only sequences the calls and reduces the copied-back
-latents to the reported numbers.  Readings (the paper defers the details to
-supplementary material):
+denoiser), and so does every reduction: the latent sums behind the downstream
+impact and the direction error come from wdc_latent_pair_stats, the local
+defect d_t from the anchor pass (Eq. 7), the schedule from
+wdc_schedule_sigmas and the correlations from wdc_correlations.  This module
+only sequences the calls and combines a few reduced scalars.  Readings (the
+paper defers the details to supplementary material):
 
 * Single-injection downstream impact (Observation 1).  The all-exact
   trajectory is rolled out with the cache's bookkeeping active (tau_risk < 0:
@@ -33,32 +36,20 @@ import numpy as np
 from . import wdc
 
 
-def _rel_l2(a, b):
-    a = np.asarray(a, dtype=np.float64).reshape(-1)
-    b = np.asarray(b, dtype=np.float64).reshape(-1)
-    return float(np.linalg.norm(a - b) / np.linalg.norm(b))
+def downstream_rel(ctx, z_inj, z_ref):
+    """||z_inj - z_ref|| / ||z_ref|| from the device sums of wdc_latent_pair_stats."""
+    s = ctx.latent_pair_stats(z_inj, z_ref)
+    return float(np.sqrt(s[3] / s[4]))
 
 
-def _angle(u, v):
-    """Angle between two increments; a zero increment carries no direction
-    and counts as orthogonal (pi/2)."""
-    nu, nv = np.linalg.norm(u), np.linalg.norm(v)
-    if nu == 0.0 or nv == 0.0:
+def increment_angle(ctx, z_hat, z_ex, z):
+    """Angle between the increments z_hat - z and z_ex - z from the device
+    sums of wdc_latent_pair_stats; an increment of zero length has no
+    direction and is reported as pi/2."""
+    s = ctx.latent_pair_stats(z_hat, z_ex, z)
+    if s[0] == 0.0 or s[1] == 0.0:
         return float(np.pi / 2)
-    return float(np.arccos(min(1.0, max(-1.0, float(np.dot(u, v) / (nu * nv))))))
-
-
-def _ranks(x):
-    order = np.argsort(np.asarray(x, dtype=np.float64), kind="stable")
-    r = np.empty(len(x))
-    r[order] = np.arange(len(x), dtype=np.float64)
-    return r
-
-
-def correlations(a, b):
-    a = np.asarray(a, dtype=np.float64)
-    b = np.asarray(b, dtype=np.float64)
-    return float(np.corrcoef(a, b)[0, 1]), float(np.corrcoef(_ranks(a), _ranks(b))[0, 1])
+    return float(np.arccos(np.clip(s[2] / np.sqrt(s[0] * s[1]), -1.0, 1.0)))
 
 
 class _Stepper:
@@ -89,14 +80,15 @@ class _Stepper:
         self.ctx.dit_forward(z, 1000.0 * self.sigmas[k], self.tok(k), self.v)
 
     def native_from(self, z0, k0):
-        """Exact inference from z0 (device) at step k0 to the end; returns host float32."""
+        """Exact inference from z0 (device) at step k0 to the end; returns the
+        device buffer holding the final latent."""
         T = len(self.sigmas) - 1
         cur = self.zbuf[0]
         cur.copy_(z0)
         for k in range(k0, T):
             self.velocity(k, cur)
             self.ctx.scheduler_step(k, cur, self.v, cur)
-        return cur.cpu().numpy()
+        return cur
 
 
 def _view(ptr, n):
@@ -109,13 +101,6 @@ def _view(ptr, n):
     return torch.as_tensor(_A(), device="cuda")
 
 
-def _sigmas(T, shift=1.0):
-    s = 1.0 - np.arange(T + 1, dtype=np.float64) / T
-    if shift != 1.0:
-        s = shift * s / (1.0 + (shift - 1.0) * s)
-    return s
-
-
 def downstream_impact(ctx, z_T, conds, cond_tokens, steps=None, tau_d=0.025, tau_D=0.06):
     """Single-injection diagnostics on the GPU (module docstring).  The
     context's tau_risk must be negative.  Returns the same dict layout as the
@@ -124,7 +109,7 @@ def downstream_impact(ctx, z_T, conds, cond_tokens, steps=None, tau_d=0.025, tau
     torch = __import__("torch")
     T = ctx.sched.T
     st = _Stepper(ctx, conds, cond_tokens)
-    st.sigmas = _sigmas(T, ctx.sched.shift)
+    st.sigmas = ctx.sigmas()
     n = ctx.numel
     ctx.state_reset(z_T)
     cur = z_T
@@ -141,14 +126,14 @@ def downstream_impact(ctx, z_T, conds, cond_tokens, steps=None, tau_d=0.025, tau
         d["d_cf"] = full.d_cf
         infos.append(d)
         cur = _view(nxt, n).clone()
-    z_final = cur.cpu().numpy()
+    z_final = cur.clone()
     rows = []
     for t, zh in enumerate(cands):
         if zh is None or (steps is not None and t not in steps):
             continue
         z_inj = st.native_from(zh, t + 1)
         i = infos[t]
-        rows.append({"t": t, "d": float(i["d_cf"]), "D_down": _rel_l2(z_inj, z_final),
+        rows.append({"t": t, "d": float(i["d_cf"]), "D_down": downstream_rel(ctx, z_inj, z_final),
                      "d_hat": float(i["d_hat"]), "w": float(i["w"]), "delta": float(i["delta"])})
         torch.cuda.synchronize()
     m = max(1, len(rows))
@@ -170,7 +155,7 @@ def direction_errors(ctx, z_T, conds, cond_tokens):
     context's parameters should select periodic placement."""
     T = ctx.sched.T
     st = _Stepper(ctx, conds, cond_tokens)
-    st.sigmas = _sigmas(T, ctx.sched.shift)
+    st.sigmas = ctx.sigmas()
     n = ctx.numel
     ctx.state_reset(z_T)
     cur = z_T.clone()
@@ -184,10 +169,8 @@ def direction_errors(ctx, z_T, conds, cond_tokens):
         st.velocity(k, cur)
         ctx.scheduler_step(k, cur, st.v, st.zex)
         if info.supported and info.finite:
-            z = cur.cpu().numpy().astype(np.float64)
             rows.append({"k": k, "streak": age, "decision": info.decision,
-                         "angle": _angle(zh.cpu().numpy().astype(np.float64) - z,
-                                         st.zex.cpu().numpy().astype(np.float64) - z)})
+                         "angle": increment_angle(ctx, zh, st.zex, cur)})
         if info.decision == 1:
             cur = zh.clone()
             ci ^= 1
@@ -231,7 +214,7 @@ def main():
     t1 = time.perf_counter()
     ctx.set_cache_params(wdc.make_params(tau_risk=0.1))
     pairs = proxy_vs_counterfactual(ctx, zT, cond)
-    pe, sp = correlations(*zip(*pairs)) if len(pairs) > 2 else (None, None)
+    pe, sp = wdc.correlations(*zip(*pairs)) if len(pairs) > 2 else (None, None)
     out["proxy_vs_cf"] = {"pairs": len(pairs), "pearson": pe, "spearman": sp, "seconds": time.perf_counter() - t1}
     strategies = {"native secant": wdc.ABL_SECANT, "lifted, no condition": wdc.ABL_NO_COND,
                   "lifted (Eq. 5 as printed)": 0, "lifted, residual reading": wdc.OBS_RESIDUAL}

@@ -119,3 +119,20 @@ def random_summaries(seed, K, dim=256):
     s_in = g.standard_normal(size=(K, dim), dtype=np.float32)
     s_out = s_in + np.float32(0.3) * g.standard_normal(size=(K, dim), dtype=np.float32)
     return s_in, s_out
+
+
+def drift_bank_device(seed, n, K, delta=0.05):
+    """drift_bank's recipe drawn on the current CUDA device with torch (for
+    the bandwidth sweep's large latents): z0 ~ N(0,1) from a seeded torch
+    generator, z_out_i = z0 + i * delta * sin(2 pi * 8 idx / n + phase_i);
+    returns a list of K float32 tensors of n elements."""
+    import torch
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    z0 = torch.randn(n, device="cuda", generator=g)
+    ph = torch.rand(K, device="cuda", generator=g, dtype=torch.float64) * (2.0 * np.pi)
+    idx = torch.arange(n, device="cuda", dtype=torch.float64) * (2.0 * np.pi * 8.0 / n)
+    out = []
+    for i in range(K):
+        out.append(z0 + (i * delta) * torch.sin(idx + ph[i]).float())
+    del idx
+    return out

@@ -133,6 +133,9 @@ def _load():
         "wdc_dit_block_forward": (I, [P, I, P, P, P]),
         "wdc_dit_modulation": (I, [P, F, P, P]),
         "wdc_scheduler_step": (I, [P, I, P, P, P, P]),
+        "wdc_schedule_sigmas": (I, [P, ctypes.POINTER(D)]),
+        "wdc_latent_pair_stats": (I, [P, P, P, P, ctypes.POINTER(D), P]),
+        "wdc_correlations": (I, [ctypes.POINTER(D), ctypes.POINTER(D), I, ctypes.POINTER(D), ctypes.POINTER(D)]),
         "wdc_state_reset": (I, [P, P, P]),
         "wdc_state_get": (I, [P, ctypes.POINTER(StateHost), P]),
         "wdc_state_set": (I, [P, ctypes.POINTER(StateHost), P, P, P]),
@@ -321,6 +324,21 @@ class Context:
     def dit_modulation(self, t, mod_out, stream=None):
         self._check(LIB.wdc_dit_modulation(self._h, float(t), _ptr(mod_out), _stream(stream)), "dit_modulation")
 
+    def sigmas(self):
+        """wdc_schedule_sigmas: the context's noise levels sigma_0..sigma_T."""
+        T = self.sched.T
+        out = (ctypes.c_double * (T + 1))()
+        self._check(LIB.wdc_schedule_sigmas(self._h, out), "schedule_sigmas")
+        return list(out)
+
+    def latent_pair_stats(self, a, b, c=None, stream=None):
+        """wdc_latent_pair_stats: [sum (a-c)^2, sum (b-c)^2, sum (a-c)(b-c),
+        sum (a-b)^2, sum b^2] over three device latents (c may be None)."""
+        out = (ctypes.c_double * 5)()
+        self._check(LIB.wdc_latent_pair_stats(self._h, _ptr(a), _ptr(b), _ptr(c), out, _stream(stream)),
+                    "latent_pair_stats")
+        return list(out)
+
     def scheduler_step(self, k, z_t, v, z_next, stream=None):
         self._check(LIB.wdc_scheduler_step(self._h, k, _ptr(z_t), _ptr(v), _ptr(z_next), _stream(stream)),
                     "scheduler_step")
@@ -387,6 +405,20 @@ class Context:
         H, L, d = q.shape
         self._check(LIB.wdc_op_attention(self._h, _ptr(q), _ptr(k), _ptr(vt), _ptr(o), H, L, d, _stream(stream)),
                     "op_attention")
+
+
+def correlations(x, y):
+    """wdc_correlations: (Pearson, Spearman) of two equal-length samples."""
+    n = len(x)
+    if len(y) != n:
+        raise ValueError("correlations: samples of different lengths")
+    xs = (ctypes.c_double * n)(*[float(v) for v in x])
+    ys = (ctypes.c_double * n)(*[float(v) for v in y])
+    pe, sp = ctypes.c_double(), ctypes.c_double()
+    st = LIB.wdc_correlations(xs, ys, n, ctypes.byref(pe), ctypes.byref(sp))
+    if st != 0:
+        raise WdcError(st, "wdc_correlations: needs n >= 2")
+    return pe.value, sp.value
 
 
 def rollout_batch(ctxs, z_T_list, conds, z_out_list, cfg=False, guidance=1.0, trace=True, stream=None):

@@ -80,3 +80,22 @@ def test_direction_errors_match_oracle(model, flags):
     assert sorted(got["mean_by_streak"]) == [0, 1, 2, 3]
     for a, b in zip(got["rows"], ref["rows"]):
         assert abs(a["angle"] - b["angle"]) <= 1e-4, (a["k"], a["angle"], b["angle"])
+
+
+@pytest.mark.parametrize("n,with_c", [(16 * 4 * 16 * 16, True), (16 * 4 * 16 * 16, False)])
+def test_latent_pair_stats_match_fp64_sums(n, with_c):
+    """The device reductions behind the diagnostics (wdc_latent_pair_stats)
+    against fp64 sums of the same fp32 latents, 1e-6 relative."""
+    W = synth.dit_weights(PARITY_MODEL, 0, std=0.02)
+    op, cp = params_for_both()
+    ctx = _ctx(W, cp)
+    g = np.random.default_rng(5)
+    a, b, c = (g.standard_normal(n).astype(np.float32) for _ in range(3))
+    dev = [torch.from_numpy(x.copy()).cuda() for x in (a, b, c)]
+    got = ctx.latent_pair_stats(dev[0], dev[1], dev[2] if with_c else None)
+    a64, b64 = a.astype(np.float64), b.astype(np.float64)
+    c64 = c.astype(np.float64) if with_c else np.zeros(n)
+    want = [np.sum((a64 - c64) ** 2), np.sum((b64 - c64) ** 2), np.sum((a64 - c64) * (b64 - c64)),
+            np.sum((a64 - b64) ** 2), np.sum(b64 ** 2)]
+    for k in range(5):
+        assert abs(got[k] - want[k]) <= 1e-6 * max(abs(want[k]), 1e-3 * want[0]), (k, got[k], want[k])
