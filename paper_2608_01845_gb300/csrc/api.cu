@@ -164,8 +164,7 @@ PassArgs base_args(Ctx* c, int k) {
     a.k = k;
     a.T = c->sched.T;
     a.age = c->age;
-    a.q_k = c->sigma[k];
-    a.q_next = c->sigma[k + 1];
+    a.sk = c->stepf[k];
     a.prm = to_dev_params(c->prm);
     a.st = c->st;
     a.partials = c->partials;
@@ -176,8 +175,8 @@ PassArgs base_args(Ctx* c, int k) {
 
 void set_cond(PassArgs& a, const wdc_cond* cd) {
     for (int j = 0; j < 4; ++j) {
-        a.cam[j] = cd ? cd->cam[j] : 0.0;
-        a.depth[j] = cd ? cd->depth[j] : 0.0;
+        a.cam[j] = cd ? (float)cd->cam[j] : 0.f;
+        a.depth[j] = cd ? (float)cd->depth[j] : 0.f;
     }
 }
 
@@ -226,7 +225,6 @@ wdc_status enqueue_anchor(Ctx* c, int k, const wdc_cond* cd, const float* z_t, c
     a.out = c->bank[ins];
     a.out2 = needs_disp(c) ? c->disp[ins] : nullptr;
     a.ins_slot = ins;
-    a.dsig = (float)(c->sigma[k + 1] - c->sigma[k]);
     wdc_status st = launch_pass(c, kModeAnchor, a, s);
     if (st) return st;
     if (dst) WDC_CUDA_TRY(c, cudaMemcpyAsync(dst, &c->st->out, sizeof(StepOut), cudaMemcpyDeviceToHost, s));
@@ -329,6 +327,14 @@ wdc_status wdc_create(const wdc_dit_config* cfg, const wdc_schedule* sched, cons
         double s = 1.0 - (double)k / (double)sched->T;
         if (sched->shift != 1.0) s = sched->shift * s / (1.0 + (sched->shift - 1.0) * s);
         c->sigma[k] = s;
+    }
+    c->stepf.resize(sched->T);
+    for (int k = 0; k < sched->T; ++k) {
+        StepScalars& f = c->stepf[k];
+        f.q_k = (float)c->sigma[k];
+        f.q_next = (float)c->sigma[k + 1];
+        f.dq = (float)(c->sigma[k + 1] - c->sigma[k]);
+        f.t_model = (float)(1000.0 * c->sigma[k]);
     }
     const size_t lat = c->n * sizeof(float);
     auto dm = [&](void** p, size_t b) -> bool {
@@ -587,7 +593,7 @@ wdc_status wdc_scheduler_step(wdc_ctx* h, int k, const float* z_t, const float* 
     const unsigned grid = (unsigned)(((n + 3) / 4 + 255) / 256);
     {
         LaunchScope ls(c, WDC_K_OTHER, (cudaStream_t)stream);
-        psi_kernel<<<grid, 256, 0, (cudaStream_t)stream>>>(z_t, v, z_next, n, (float)(c->sigma[k + 1] - c->sigma[k]));
+        psi_kernel<<<grid, 256, 0, (cudaStream_t)stream>>>(z_t, v, z_next, n, c->stepf[k].dq);
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("scheduler_step: ") + cudaGetErrorString(e));
@@ -611,9 +617,10 @@ wdc_status wdc_state_reset(wdc_ctx* h, const float* z_T, wdc_stream stream) {
     if (cs) return cs;
     DevState* hs = c->st_host;           // pinned staging owned by the context
     std::memset(hs, 0, sizeof(DevState));
-    hs->R = 0.0;
-    hs->eta = c->prm.eta_init;
-    hs->q_a_in = hs->q_a_out = c->sigma[0];
+    hs->R = 0.f;
+    hs->eta = (float)c->prm.eta_init;
+    hs->q_a_in = hs->q_a_out = (float)c->sigma[0];
+    hs->q_a_dq = 0.f;
     hs->cand_k = -1;
     cudaError_t e = cudaMemcpyAsync(c->st, hs, sizeof(DevState), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
@@ -678,11 +685,12 @@ wdc_status wdc_state_set(wdc_ctx* h, const wdc_state_host* in, const float* cons
     cudaStream_t s = (cudaStream_t)stream;
     DevState* hs = c->st_host;           // pinned staging owned by the context
     std::memset(hs, 0, sizeof(DevState));
-    hs->R = in->R;
-    hs->eta = in->eta;
-    hs->q_a_in = in->q_a_in;
-    hs->q_a_out = in->q_a_out;
-    for (int j = 0; j < 4; ++j) { hs->cam_a[j] = in->cam_a[j]; hs->depth_a[j] = in->depth_a[j]; }
+    hs->R = (float)in->R;
+    hs->eta = (float)in->eta;
+    hs->q_a_in = (float)in->q_a_in;
+    hs->q_a_out = (float)in->q_a_out;
+    hs->q_a_dq = (float)(in->q_a_out - in->q_a_in);
+    for (int j = 0; j < 4; ++j) { hs->cam_a[j] = (float)in->cam_a[j]; hs->depth_a[j] = (float)in->depth_a[j]; }
     hs->cand_k = -1;
     for (int i = 0; i < in->n_bank; ++i) {
         DevRecord& r = hs->rec[i];
@@ -697,8 +705,11 @@ wdc_status wdc_state_set(wdc_ctx* h, const wdc_state_host* in, const float* cons
         }
         r.n_in = (float)std::sqrt(a);
         r.n_out = (float)std::sqrt(b);
-        r.q_in = o.q_in; r.q_out = o.q_out; r.r = o.r;
-        for (int j = 0; j < 4; ++j) { r.cam[j] = o.cam[j]; r.depth[j] = o.depth[j]; }
+        r.q_in = (float)o.q_in;
+        r.q_out = (float)o.q_out;
+        r.dq = (float)(o.q_out - o.q_in);
+        r.r = (float)o.r;
+        for (int j = 0; j < 4; ++j) { r.cam[j] = (float)o.cam[j]; r.depth[j] = (float)o.depth[j]; }
     }
     cudaError_t e = cudaMemcpyAsync(c->st, hs, sizeof(DevState), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);

@@ -37,7 +37,7 @@ struct PlanArgs {
     float* cand;
     float* zcur;
     float* vbuf;
-    const double* sigma;             // [T + 1]
+    const StepScalars* stepf;        // [T]
     int K, mode, needs_disp;
     PassArgs* skip;                  // outputs
     PassArgs* anchor;
@@ -64,8 +64,7 @@ __global__ void plan_kernel(const PlanArgs* __restrict__ pp) {
     PassArgs a = p.tmpl;
     a.k = k;
     a.age = age;
-    a.q_k = p.sigma[k];
-    a.q_next = p.sigma[k + 1];
+    a.sk = p.stepf[k];
     a.nsrc = nb;
     for (int i = 0; i < nb; ++i) a.slot[i] = slot_of(i);
     if (p.mode == kModeSecant) {
@@ -85,8 +84,7 @@ __global__ void plan_kernel(const PlanArgs* __restrict__ pp) {
     b.graph = 0;
     b.k = k;
     b.age = age;
-    b.q_k = p.sigma[k];
-    b.q_next = p.sigma[k + 1];
+    b.sk = p.stepf[k];
     b.nsrc = 0;
     const int ins = nb < K ? slot_of(nb) : head;
     b.src[0] = p.zcur;
@@ -97,10 +95,9 @@ __global__ void plan_kernel(const PlanArgs* __restrict__ pp) {
     b.out2 = p.needs_disp ? p.disp[ins] : nullptr;
     b.out3 = p.zcur;
     b.ins_slot = ins;
-    b.dsig = (float)(p.sigma[k + 1] - p.sigma[k]);
     *p.anchor = b;
 
-    st->g_t_model = (float)(1000.0 * p.sigma[k]);
+    st->g_t_model = p.stepf[k].t_model;
     p.pre[2 * k] = nb;
     p.pre[2 * k + 1] = age;
     cudaGraphSetConditional((cudaGraphConditionalHandle)p.h_switch,
@@ -169,7 +166,7 @@ struct GraphRollout {
     cudaStream_t cap = nullptr;
     float* zcur = nullptr;
     float* cond = nullptr;           // [cond_tokens, cond_dim] fp32 copy of this rollout's tokens
-    double* sigma = nullptr;
+    StepScalars* stepf = nullptr;
     PassArgs* args = nullptr;        // [2]: skip, anchor
     PlanArgs* plan = nullptr;
     StepOut* trace = nullptr;
@@ -182,7 +179,7 @@ struct GraphRollout {
         if (cap) cudaStreamDestroy(cap);
         cudaFree(zcur);
         cudaFree(cond);
-        cudaFree(sigma);
+        cudaFree(stepf);
         cudaFree(args);
         cudaFree(plan);
         cudaFree(trace);
@@ -310,8 +307,8 @@ wdc_status graph_rollout(Ctx* c, const float* z_T, bool z_dev, const wdc_cond* c
         WDC_G(cudaMalloc((void**)&G->zcur, bytes));
         const size_t ce = (size_t)c->cfg.cond_tokens * c->cfg.cond_dim;
         WDC_G(cudaMalloc((void**)&G->cond, (ce ? ce : 1) * sizeof(float)));
-        WDC_G(cudaMalloc((void**)&G->sigma, (T + 1) * sizeof(double)));
-        WDC_G(cudaMemcpy(G->sigma, c->sigma.data(), (T + 1) * sizeof(double), cudaMemcpyHostToDevice));
+        WDC_G(cudaMalloc((void**)&G->stepf, T * sizeof(StepScalars)));
+        WDC_G(cudaMemcpy(G->stepf, c->stepf.data(), T * sizeof(StepScalars), cudaMemcpyHostToDevice));
         WDC_G(cudaMalloc((void**)&G->args, 2 * sizeof(PassArgs)));
         WDC_G(cudaMalloc((void**)&G->plan, sizeof(PlanArgs)));
         WDC_G(cudaMalloc((void**)&G->trace, T * sizeof(StepOut)));
@@ -354,7 +351,7 @@ wdc_status graph_rollout(Ctx* c, const float* z_T, bool z_dev, const wdc_cond* c
     p.cand = c->cand[0];
     p.zcur = G->zcur;
     p.vbuf = c->vbuf;
-    p.sigma = G->sigma;
+    p.stepf = G->stepf;
     p.K = K;
     p.mode = G->mode;
     p.needs_disp = (c->prm.flags & (WDC_ABL_SECANT | WDC_OBS_RESIDUAL)) ? 1 : 0;

@@ -31,6 +31,7 @@
 #include "wdc_internal.h"
 
 #include <cmath>
+#include <cstddef>
 #include <cstring>
 #include <mutex>
 
@@ -113,6 +114,26 @@ __device__ __forceinline__ void reduce256d(double (&v)[NV], double* scratch, dou
     __syncthreads();
 }
 
+// The part of the device state a pass reads, copied into shared memory by all
+// threads at the start in one batch of independent loads; the head and the
+// tails then work from shared memory.  (Read in place, the head and the
+// controller tail were chains of dependent L2 round trips -- the state may sit
+// in the other die's half of L2 -- that cost about 10 us per launch.)
+struct alignas(16) StateIn {
+    float cur_S[kSketch], anchor_S[kSketch];
+    float s_phi[kSummary];                 // anchor pass: the pre-insertion summary
+    float n_in[kMaxBank], n_out[kMaxBank]; // records by age (oldest first)
+    float q_in[kMaxBank], dq[kMaxBank], r[kMaxBank];
+    float cur_sumsq, cur_sumsq_anchor, anchor_sumsq, R, eta, q_a_out, q_a_dq, cand_p;
+    float cam_a[4], depth_a[4];
+    int cand_k, cand_supported, cand_finite;
+};
+// The records' summaries by age; shares storage with the stream's bucket
+// rows, which are used only after the head.
+struct alignas(16) RecSummaries {
+    float s_in[kMaxBank][kSummary], s_out[kMaxBank][kSummary], s_dphi[kMaxBank][kSummary];
+};
+
 struct HeadShared {
     float phi[kSummary];
     float hat[kSummary];
@@ -133,16 +154,15 @@ struct HeadShared {
 // positive definite for rho > 0).  The system is ill-conditioned at a small
 // ridge, so G and S_out s_hat are reduced in fp64 here.
 template <int K>
-__device__ __noinline__ void linear_readout(const PassArgs& a, HeadShared& hs) {
+__device__ __noinline__ void linear_readout(const PassArgs& a, const RecSummaries& rs, HeadShared& hs) {
     if constexpr (K > 0) {
         const int t = threadIdx.x;
-        const DevState* st = a.st;
         // one row of G per reduction (keeps K values per thread); row K = S_out s_hat
         for (int i = 0; i <= K; ++i) {
             double v[K];
-            const double si = (t < kSummary) ? (i < K ? (double)st->rec[a.slot[i]].s_out[t] : (double)hs.hat[t]) : 0.0;
+            const double si = (t < kSummary) ? (i < K ? (double)rs.s_out[i][t] : (double)hs.hat[t]) : 0.0;
 #pragma unroll
-            for (int j = 0; j < K; ++j) v[j] = (t < kSummary) ? si * (double)st->rec[a.slot[j]].s_out[t] : 0.0;
+            for (int j = 0; j < K; ++j) v[j] = (t < kSummary) ? si * (double)rs.s_out[j][t] : 0.0;
             reduce256d<K>(v, hs.dscratch, hs.gram[i]);
         }
         double b[K];
@@ -161,7 +181,7 @@ __device__ __noinline__ void linear_readout(const PassArgs& a, HeadShared& hs) {
 #pragma unroll
                 for (int i = 0; i < K; ++i) hs.kappa[i] = 0.f;
             } else {
-                const double rho = a.prm.ridge * tr / K;
+                const double rho = (double)a.prm.ridge * tr / K;
 #pragma unroll
                 for (int i = 0; i < K; ++i) A[i][i] += rho;
                 // Cholesky A = L L^T (L in the lower triangle of A)
@@ -197,38 +217,34 @@ __device__ __noinline__ void linear_readout(const PassArgs& a, HeadShared& hs) {
 // Skip-pass head, Eq. 2-5 scalar part, in fp32 (every CTA computes it; it is
 // a few hundred cycles of latency, and no CTA has to wait for another).
 template <int K>
-__device__ void skip_head(const PassArgs& a, HeadShared& hs) {
-    const DevState* st = a.st;
+__device__ void skip_head(const PassArgs& a, const StateIn& S, const RecSummaries& rs, HeadShared& hs) {
     const int t = threadIdx.x;
     const float N = (float)a.n;
     const float sc = sqrtf((float)kSketch / N);
-    const float eps_nu = (float)a.prm.eps_nu;
+    const float eps_nu = a.prm.eps_nu;
     const bool no_cond = a.prm.flags & WDC_ABL_NO_COND;
     // s(phi_k): current-state summary (Eq. 2 through the linear sketch)
     if (t < kSummary) {
         float val;
         if (t < kSketch) {
-            val = sc * st->cur_S[t] / (sqrtf((float)st->cur_sumsq / N) + eps_nu);
+            val = sc * S.cur_S[t] / (sqrtf(S.cur_sumsq / N) + eps_nu);
         } else if (t < 2 * kSketch) {
             const int b = t - kSketch;
-            val = sc * (st->cur_S[b] - st->anchor_S[b]) / (sqrtf((float)st->cur_sumsq_anchor / N) + eps_nu);
+            val = sc * (S.cur_S[b] - S.anchor_S[b]) / (sqrtf(S.cur_sumsq_anchor / N) + eps_nu);
         } else if (t < kOffDepth) {
-            val = no_cond ? 0.f : (float)a.cam[t - kOffCam];
+            val = no_cond ? 0.f : a.cam[t - kOffCam];
         } else if (t < kOffQ) {
-            val = no_cond ? 0.f : (float)a.depth[t - kOffDepth];
+            val = no_cond ? 0.f : a.depth[t - kOffDepth];
         } else if (t == kOffQ) {
-            val = (float)a.q_k;
+            val = a.sk.q_k;
         } else {
             // h(H): [r_1..3, T*(q_in - q_out)_1..3, n_bank/K], newest record first
             const int j = t - kOffH;
             val = 0.f;
             if (j < 3) {
-                if (j < a.nsrc) val = (float)st->rec[a.slot[a.nsrc - 1 - j]].r;
+                if (j < a.nsrc) val = S.r[a.nsrc - 1 - j];
             } else if (j < 6) {
-                if (j - 3 < a.nsrc) {
-                    const DevRecord& r = st->rec[a.slot[a.nsrc - 1 - (j - 3)]];
-                    val = (float)((double)a.T * (r.q_in - r.q_out));
-                }
+                if (j - 3 < a.nsrc) val = -(float)a.T * S.dq[a.nsrc - 1 - (j - 3)];
             } else {
                 val = (float)a.nsrc / (float)a.prm.K;
             }
@@ -237,8 +253,8 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
     }
     if (t == 0) {
         // Eq. 4: alpha = clip(|q_{t-1}-q_t| / (|q_{a-1}-q_a| + eps), alpha_min, alpha_max)
-        const float raw = (float)fabs(a.q_next - a.q_k) / ((float)fabs(st->q_a_out - st->q_a_in) + (float)a.prm.eps);
-        hs.alpha = fminf(fmaxf(raw, (float)a.prm.alpha_min), (float)a.prm.alpha_max);
+        const float raw = fabsf(a.sk.dq) / (fabsf(S.q_a_dq) + a.prm.eps);
+        hs.alpha = fminf(fmaxf(raw, a.prm.alpha_min), a.prm.alpha_max);
     }
     __syncthreads();
     if (K == 0) return;
@@ -248,27 +264,25 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
         float v[K + 1];
         const float ph = (t < kSummary) ? hs.phi[t] : 0.f;
 #pragma unroll
-        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? ph * st->rec[a.slot[i]].s_in[t] : 0.f;
+        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? ph * rs.s_in[i][t] : 0.f;
         v[K] = ph * ph;
         reduce256<K + 1>(v, hs.scratch, hs.red);
     }
     if (t == 0) {
         const float nphi = sqrtf(hs.red[K]);
         const bool filter = !(a.prm.flags & WDC_ABL_NO_SUPPORT);   // w/o support: N_t = whole bank
-        const float gq = (float)a.prm.gamma_q, inv_tin = 1.0f / (float)a.prm.tau_in;
+        const float gq = a.prm.gamma_q, inv_tin = 1.0f / a.prm.tau_in;
         int nc = 0;
         float mx = -INFINITY;
         float ell[K > 0 ? K : 1];
 #pragma unroll
         for (int i = 0; i < K; ++i) {
-            const DevRecord& r = st->rec[a.slot[i]];
-            const float s = (nphi == 0.f || r.n_in == 0.f) ? 0.f : hs.red[i] / (nphi * r.n_in);
-            const double dq = a.q_k - r.q_in;
+            const float s = (nphi == 0.f || S.n_in[i] == 0.f) ? 0.f : hs.red[i] / (nphi * S.n_in[i]);
+            const float dq = a.sk.q_k - S.q_in[i];
             hs.sim_in[i] = s;
-            const int c = !filter || ((s >= (float)a.prm.sim_min) && (fabs(dq) <= a.prm.q_gap_max));
+            const int c = !filter || ((s >= a.prm.sim_min) && (fabsf(dq) <= a.prm.q_gap_max));
             hs.compat[i] = c;
-            const float dqf = (float)dq;
-            ell[i] = (s - gq * dqf * dqf) * inv_tin;
+            ell[i] = (s - gq * dq * dq) * inv_tin;
             if (c) { ++nc; mx = fmaxf(mx, ell[i]); }
         }
         float tot = 0.f;
@@ -291,24 +305,23 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
             float acc = 0.f;
 #pragma unroll
             for (int i = 0; i < K; ++i)
-                if (hs.pi[i] != 0.f) acc = fmaf(hs.pi[i], st->rec[a.slot[i]].s_dphi[t], acc);
+                if (hs.pi[i] != 0.f) acc = fmaf(hs.pi[i], rs.s_dphi[i][t], acc);
             hv = fmaf(hs.alpha, acc, hs.phi[t]);
             hs.hat[t] = hv;
         }
 #pragma unroll
-        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? hv * st->rec[a.slot[i]].s_out[t] : 0.f;
+        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? hv * rs.s_out[i][t] : 0.f;
         v[K] = hv * hv;
         reduce256<K + 1>(v, hs.scratch, hs.red);
     }
     if (t == 0) {
         const float nh = sqrtf(hs.red[K]);
-        const float inv_tau = 1.0f / (float)a.prm.tau_obs;
+        const float inv_tau = 1.0f / a.prm.tau_obs;
         float mx = -INFINITY;
         float e[K > 0 ? K : 1];
 #pragma unroll
         for (int i = 0; i < K; ++i) {
-            const DevRecord& r = st->rec[a.slot[i]];
-            const float s = (nh == 0.f || r.n_out == 0.f) ? 0.f : hs.red[i] / (nh * r.n_out);
+            const float s = (nh == 0.f || S.n_out[i] == 0.f) ? 0.f : hs.red[i] / (nh * S.n_out[i]);
             hs.sim_out[i] = s;
             e[i] = s * inv_tau;
             mx = fmaxf(mx, e[i]);
@@ -321,7 +334,7 @@ __device__ void skip_head(const PassArgs& a, HeadShared& hs) {
         for (int i = 0; i < K; ++i) hs.kappa[i] = e[i] * inv;
     }
     __syncthreads();
-    if (a.prm.flags & WDC_ABL_LINEAR_OBS) linear_readout<K>(a, hs);
+    if (a.prm.flags & WDC_ABL_LINEAR_OBS) linear_readout<K>(a, rs, hs);
 }
 
 // Per-block scalar slots: the stream's five sums and the non-finite count.
@@ -329,12 +342,81 @@ constexpr int kScalars = 6;
 // Most blocks one pass launch may have (the final reduction's register tile).
 constexpr int kMaxPassBlocks = 256;
 
-struct PassShared {
-    float wb[2][kWarps][kSketch];     // per-warp bucket rows (2 sketches for the stats pass)
+// 16-byte aligned: load_state stores float4 values into the snapshot arrays.
+struct alignas(16) PassShared {
+    union {
+        float wb[2][kWarps][kSketch]; // per-warp bucket rows (2 sketches for the stats pass)
+        RecSummaries rs;              // the head's record summaries (before the stream)
+    };
     float blk[kWarps][kScalars];
     float fin[kPartials];
+    StateIn S;
     int last;
 };
+
+static_assert(alignof(PassShared) >= 16 && alignof(StateIn) >= 16 && alignof(RecSummaries) >= 16,
+              "float4 snapshot stores need 16-byte aligned shared arrays");
+static_assert(offsetof(PassShared, S) % 16 == 0 && offsetof(PassShared, rs) == 0, "snapshot offsets");
+static_assert(offsetof(StateIn, cur_S) % 16 == 0 && offsetof(StateIn, anchor_S) % 16 == 0 &&
+              offsetof(StateIn, s_phi) % 16 == 0, "snapshot vector offsets");
+static_assert((kSummary * sizeof(float)) % 16 == 0, "summary rows stay 16-byte aligned");
+static_assert(offsetof(DevRecord, s_in) % 16 == 0 && offsetof(DevRecord, s_out) % 16 == 0 &&
+              offsetof(DevRecord, s_dphi) % 16 == 0 && sizeof(DevRecord) % 16 == 0, "record layout");
+static_assert(offsetof(DevState, rec) % 16 == 0 && offsetof(DevState, cur_S) % 16 == 0 &&
+              offsetof(DevState, anchor_S) % 16 == 0 && offsetof(DevState, s_phi) % 16 == 0, "state layout");
+
+// Copies what this mode reads of the device state into shared memory (one
+// batch of independent loads spread over the block's threads).
+template <int MODE>
+__device__ __forceinline__ void load_state(const PassArgs& a, PassShared& ps) {
+    const DevState* st = a.st;
+    const int t = threadIdx.x;
+    StateIn& S = ps.S;
+    const bool head = MODE == kModeSkip || MODE == kModeResidual || MODE == kModeSecant;
+    if (MODE == kModeSkip || MODE == kModeResidual) {
+        // summaries of the nsrc records by age: 3 arrays x 64 float4 each
+        for (int idx = t; idx < a.nsrc * 192; idx += kThreads) {
+            const int i = idx / 192, rem = idx - i * 192, which = rem >> 6, c = rem & 63;
+            const DevRecord& R = st->rec[a.slot[i]];
+            const float* src = which == 0 ? R.s_in : (which == 1 ? R.s_out : R.s_dphi);
+            float* dst = which == 0 ? ps.rs.s_in[i] : (which == 1 ? ps.rs.s_out[i] : ps.rs.s_dphi[i]);
+            reinterpret_cast<float4*>(dst)[c] = __ldcg(reinterpret_cast<const float4*>(src) + c);
+        }
+    }
+    if (head || MODE == kModeAnchor) {
+        const int u = t - 384;                   // threads 384.. take the vectors and scalars
+        if (u >= 0 && u < 30) reinterpret_cast<float4*>(S.cur_S)[u] = __ldcg(reinterpret_cast<const float4*>(st->cur_S) + u);
+        else if (u >= 32 && u < 62)
+            reinterpret_cast<float4*>(S.anchor_S)[u - 32] = __ldcg(reinterpret_cast<const float4*>(st->anchor_S) + (u - 32));
+        else if (MODE == kModeAnchor && u >= 64 && u < 128)
+            reinterpret_cast<float4*>(S.s_phi)[u - 64] = __ldcg(reinterpret_cast<const float4*>(st->s_phi) + (u - 64));
+        else if (u >= 128 && u < 128 + kMaxBank) {
+            const int i = u - 128;
+            if (i < a.nsrc) {
+                const DevRecord& R = st->rec[a.slot[i]];
+                S.n_in[i] = __ldcg(&R.n_in);
+                S.n_out[i] = __ldcg(&R.n_out);
+                S.q_in[i] = __ldcg(&R.q_in);
+                S.dq[i] = __ldcg(&R.dq);
+                S.r[i] = __ldcg(&R.r);
+            }
+        } else if (u >= 160 && u < 168) {
+            const int j = u - 160;
+            if (j < 4) S.cam_a[j] = __ldcg(&st->cam_a[j]);
+            else S.depth_a[j - 4] = __ldcg(&st->depth_a[j - 4]);
+        } else if (u == 168) S.cur_sumsq = __ldcg(&st->cur_sumsq);
+        else if (u == 169) S.cur_sumsq_anchor = __ldcg(&st->cur_sumsq_anchor);
+        else if (u == 170) S.anchor_sumsq = __ldcg(&st->anchor_sumsq);
+        else if (u == 171) S.R = __ldcg(&st->R);
+        else if (u == 172) S.eta = __ldcg(&st->eta);
+        else if (u == 173) S.q_a_dq = __ldcg(&st->q_a_dq);
+        else if (u == 174) S.q_a_out = __ldcg(&st->q_a_out);
+        else if (u == 175) S.cand_p = __ldcg(&st->cand_p);
+        else if (u == 176) S.cand_k = __ldcg(&st->cand_k);
+        else if (u == 177) S.cand_supported = __ldcg(&st->cand_supported);
+        else if (u == 178) S.cand_finite = __ldcg(&st->cand_finite);
+    }
+}
 
 // Sum over the 32 warps' rows of one bucket, in a fixed pairwise order.
 __device__ __forceinline__ float sum_warp_rows(const float (&rows)[kWarps][kSketch], int b) {
@@ -358,27 +440,28 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
     const long long nruns = (n + kRun - 1) / kRun;
     const long long full = n / kRun;
 
-    for (int i = t; i < 2 * kWarps * kSketch; i += kThreads) (&ps.wb[0][0][0])[i] = 0.f;
+    load_state<MODE>(a, ps);
+    __syncthreads();
 
     bool do_stream = true;
     float kap[K > 0 ? K : 1];
     float alpha_f = 0.f;
     if (MODE == kModeSkip || MODE == kModeResidual) {
-        skip_head<K>(a, hs);
+        skip_head<K>(a, ps.S, ps.rs, hs);          // ends with a block barrier
         do_stream = (K > 0) && hs.supported;
 #pragma unroll
         for (int i = 0; i < K; ++i) kap[i] = hs.kappa[i];
     } else if (MODE == kModeSecant) {
-        skip_head<0>(a, hs);               // lift summary and alpha only: no retrieval
+        skip_head<0>(a, ps.S, ps.rs, hs);          // lift summary and alpha only: no retrieval
         do_stream = a.nsrc > 0;
         alpha_f = hs.alpha;
     } else if (MODE == kModeObserve) {
 #pragma unroll
         for (int i = 0; i < K; ++i) kap[i] = a.kappa[i];
-        __syncthreads();
-    } else {
-        __syncthreads();
     }
+    // the bucket rows share storage with the record summaries the head read
+    for (int i = t; i < 2 * kWarps * kSketch; i += kThreads) (&ps.wb[0][0][0])[i] = 0.f;
+    __syncthreads();
 
     // per-thread accumulators: plain fp32 over up to 16 runs (64 terms), then
     // a compensated fp32 outer sum
@@ -386,7 +469,7 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
     float fac[5] = {0, 0, 0, 0, 0};
     int nonfinite = 0;
     int since = 0;
-    const float dsig = a.dsig;
+    const float dsig = a.sk.dq;
 
     if (do_stream) {
         const long long gw = (long long)blockIdx.x * kWarps + warp;
@@ -741,30 +824,30 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
         if (t == 0) {
             // controller tail in fp32; the stored risk R stays fp64
             const ParamsDev& p = a.prm;
-            const float eps = (float)p.eps;
-            const float d_z = sqrtf((float)st->cur_sumsq_anchor / N) / (sqrtf((float)st->anchor_sumsq / N) + eps);
+            const float eps = p.eps;
+            const StateIn& S = ps.S;
+            const float d_z = sqrtf(S.cur_sumsq_anchor / N) / (sqrtf(S.anchor_sumsq / N) + eps);
             const float d_age = (float)a.age;
-            const float d_phase = (float)fabs(a.q_next - st->q_a_out);
+            const float d_phase = fabsf(a.sk.q_next - S.q_a_out);
             float dc = 0.f, dd = 0.f, uc = 0.f, ud = 0.f;
             for (int j = 0; j < 4; ++j) {
-                const float cj = (float)a.cam[j], dj = (float)a.depth[j];
-                const float ca = (float)st->cam_a[j], da = (float)st->depth_a[j];
+                const float cj = a.cam[j], dj = a.depth[j];
+                const float ca = S.cam_a[j], da = S.depth_a[j];
                 dc = fmaf(cj - ca, cj - ca, dc);
                 dd = fmaf(dj - da, dj - da, dd);
                 uc = fmaf(cj, cj, uc);
                 ud = fmaf(dj, dj, ud);
             }
-            const float pt = (float)p.w_z * d_z + (float)p.w_age * d_age + (float)p.w_phase * d_phase +
-                             (float)p.w_cam * sqrtf(dc) + (float)p.w_depth * sqrtf(dd);
-            const float d_hat = (float)st->eta * pt;
+            const float pt = p.w_z * d_z + p.w_age * d_age + p.w_phase * d_phase + p.w_cam * sqrtf(dc) +
+                             p.w_depth * sqrtf(dd);
+            const float d_hat = S.eta * pt;
             const float w = (p.flags & WDC_ABL_NO_IMPACT)
                                 ? 1.f
-                                : fminf(2.f, 1.f + (float)p.a_cam * sqrtf(uc) + (float)p.a_depth * sqrtf(ud) +
-                                                 (float)p.a_phase * (float)a.q_k);
+                                : fminf(2.f, 1.f + p.a_cam * sqrtf(uc) + p.a_depth * sqrtf(ud) + p.a_phase * a.sk.q_k);
             const float delta = w * d_hat;
-            const double R_cand = p.lam * st->R + (double)delta;
+            const float R_cand = fmaf(p.lam, S.R, delta);
             const bool avail = (a.nsrc > 0) && (a.age <= p.max_age) &&
-                               (fabs(a.q_k - st->q_a_out) <= p.q_gap_max) && finite && supported &&
+                               (fabsf(a.sk.q_k - S.q_a_out) <= p.q_gap_max) && finite && supported &&
                                (a.k >= p.n_init_exact) && (a.k < a.T - p.n_final_exact);
             // Eq. 10, or periodic placement (ablation): at most period - 1 surrogate steps in a row
             const bool accept = (p.flags & WDC_ABL_PERIODIC) ? (a.age + 1 < p.period) : (R_cand <= p.tau_risk);
@@ -774,28 +857,29 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
             o.finite = finite;
             o.supported = supported;
             o.n_compat = (MODE == kModeSecant) ? a.nsrc : ((K > 0) ? hs.n_compat : 0);
-            o.q = a.q_k;
-            o.alpha = (a.nsrc > 0) ? hs.alpha : 0.0;
+            o.q = a.sk.q_k;
+            o.alpha = (a.nsrc > 0) ? hs.alpha : 0.f;
             o.p = pt;
             o.d_hat = d_hat;
             o.w = w;
             o.delta = delta;
             o.R_cand = R_cand;
-            o.d_cf = nan("");
+            o.d_cf = __int_as_float(0x7fc00000);   // NaN: no exact step yet
             o.d_z = d_z;
-            o.r = 0.0;
+            o.r = 0.f;
             for (int i = 0; i < kMaxBank; ++i) {
                 o.kappa[i] = (i < K) ? hs.kappa[i] : 0.f;
                 o.pi[i] = (i < K) ? hs.pi[i] : 0.f;
             }
+            const float R_new = dec ? R_cand : S.R;
             if (dec) st->R = R_cand;
             if (a.graph) {
                 // device-side control flow: exactly one of the two branches runs
                 cudaGraphSetConditional((cudaGraphConditionalHandle)a.h_exact, dec ? 0u : 1u);
                 cudaGraphSetConditional((cudaGraphConditionalHandle)a.h_accept, dec ? 1u : 0u);
             }
-            o.R = st->R;
-            o.eta = st->eta;
+            o.R = R_new;
+            o.eta = S.eta;
             st->cand_k = a.k;
             st->cand_supported = supported;
             st->cand_finite = finite;
@@ -820,22 +904,25 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
     __shared__ float s_rms[2];
     if (t == 0) {
         const ParamsDev& p = a.prm;
-        const float eps = (float)p.eps;
-        st->R = p.lam * st->R;
-        double d_cf = nan("");
-        if (a.zcf != nullptr && st->cand_k == a.k && st->cand_supported && st->cand_finite) {
-            const float dcf = (fin[sc0 + 0] / N) / (fin[sc0 + 1] / N + eps);
-            d_cf = dcf;
+        const float eps = p.eps;
+        const StateIn& S = ps.S;
+        const float R = p.lam * S.R;
+        float eta = S.eta;
+        st->R = R;
+        float d_cf = __int_as_float(0x7fc00000);    // NaN: no calibration this step
+        if (a.zcf != nullptr && S.cand_k == a.k && S.cand_supported && S.cand_finite) {
+            d_cf = (fin[sc0 + 0] / N) / (fin[sc0 + 1] / N + eps);
             if (!(p.flags & WDC_ABL_NO_CALIB)) {
-                const float bd = (float)p.beta_d;
-                const float v = bd * (float)st->eta + (1.f - bd) * dcf / ((float)st->cand_p + eps);
-                st->eta = fminf(fmaxf(v, (float)p.eta_min), (float)p.eta_max);
+                const float bd = p.beta_d;
+                const float v = bd * S.eta + (1.f - bd) * d_cf / (S.cand_p + eps);
+                eta = fminf(fmaxf(v, p.eta_min), p.eta_max);
+                st->eta = eta;
             }
         }
         st->out.d_cf = d_cf;
-        st->out.R = st->R;
-        st->out.eta = st->eta;
-        const float r = sqrtf(fin[sc0 + 4] / N) / (sqrtf((float)st->cur_sumsq / N) + eps);
+        st->out.R = R;
+        st->out.eta = eta;
+        const float r = sqrtf(fin[sc0 + 4] / N) / (sqrtf(S.cur_sumsq / N) + eps);
         st->out.r = r;
         st->rec[a.ins_slot].r = r;
         s_rms[0] = sqrtf(fin[sc0 + 2] / N);
@@ -844,7 +931,7 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
     __syncthreads();
     DevRecord& rec = st->rec[a.ins_slot];
     const float sc = sqrtf((float)kSketch / N);
-    const float eps_nu = (float)a.prm.eps_nu;
+    const float eps_nu = a.prm.eps_nu;
     const bool no_cond = a.prm.flags & WDC_ABL_NO_COND;
     float so = 0.f, si = 0.f;
     if (t < kSummary) {
@@ -852,19 +939,18 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
             so = sc * fin[t] / (s_rms[0] + eps_nu);
         } else if (t < 2 * kSketch) {
             const int b = t - kSketch;
-            so = sc * (fin[b] - st->anchor_S[b]) / (s_rms[1] + eps_nu);
+            so = sc * (fin[b] - ps.S.anchor_S[b]) / (s_rms[1] + eps_nu);
         } else if (t < kOffDepth) {
-            so = no_cond ? 0.f : (float)a.cam[t - kOffCam];
+            so = no_cond ? 0.f : a.cam[t - kOffCam];
         } else if (t < kOffQ) {
-            so = no_cond ? 0.f : (float)a.depth[t - kOffDepth];
+            so = no_cond ? 0.f : a.depth[t - kOffDepth];
         } else if (t == kOffQ) {
-            so = (float)a.q_next;
+            so = a.sk.q_next;
         } else {
-            so = st->s_phi[t];     // pre-insertion history h(H)
+            so = ps.S.s_phi[t];    // pre-insertion history h(H)
         }
-        si = st->s_phi[t];
+        si = ps.S.s_phi[t];
     }
-    __syncthreads();               // everyone has read anchor_S and s_phi
     if (t < kSummary) {
         rec.s_in[t] = si;
         rec.s_out[t] = so;
@@ -881,8 +967,9 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
     if (t == 0) {
         rec.n_in = sqrtf(hs.red[0]);
         rec.n_out = sqrtf(hs.red[1]);
-        rec.q_in = a.q_k;
-        rec.q_out = a.q_next;
+        rec.q_in = a.sk.q_k;
+        rec.q_out = a.sk.q_next;
+        rec.dq = a.sk.dq;
         for (int j = 0; j < 4; ++j) {
             rec.cam[j] = a.cam[j];
             rec.depth[j] = a.depth[j];
@@ -891,9 +978,10 @@ __device__ __forceinline__ void pass_body(const PassArgs& a) {
         }
         st->anchor_sumsq = fin[sc0 + 2];
         st->cur_sumsq = fin[sc0 + 2];
-        st->cur_sumsq_anchor = 0.0;
-        st->q_a_in = a.q_k;
-        st->q_a_out = a.q_next;
+        st->cur_sumsq_anchor = 0.f;
+        st->q_a_in = a.sk.q_k;
+        st->q_a_out = a.sk.q_next;
+        st->q_a_dq = a.sk.dq;
     }
 }
 
@@ -1097,31 +1185,31 @@ ParamsDev to_dev_params(const wdc_cache_params& p) {
     d.n_init_exact = p.n_init_exact;
     d.n_final_exact = p.n_final_exact;
     d.seed = p.sketch_seed;
-    d.sim_min = p.sim_min;
-    d.q_gap_max = p.q_gap_max;
-    d.gamma_q = p.gamma_q;
-    d.tau_in = p.tau_in;
-    d.tau_obs = p.tau_obs;
-    d.alpha_min = p.alpha_min;
-    d.alpha_max = p.alpha_max;
-    d.eps = p.eps;
-    d.eps_nu = p.eps_nu;
-    d.w_z = p.w_z;
-    d.w_age = p.w_age;
-    d.w_phase = p.w_phase;
-    d.w_cam = p.w_cam;
-    d.w_depth = p.w_depth;
-    d.eta_min = p.eta_min;
-    d.eta_max = p.eta_max;
-    d.beta_d = p.beta_d;
-    d.a_cam = p.a_cam;
-    d.a_depth = p.a_depth;
-    d.a_phase = p.a_phase;
-    d.lam = (p.flags & WDC_ABL_INSTANT_RISK) ? 0.0 : p.lambda_;   // instantaneous risk: no accumulation
-    d.tau_risk = p.tau_risk;
+    d.sim_min = (float)p.sim_min;
+    d.q_gap_max = (float)p.q_gap_max;
+    d.gamma_q = (float)p.gamma_q;
+    d.tau_in = (float)p.tau_in;
+    d.tau_obs = (float)p.tau_obs;
+    d.alpha_min = (float)p.alpha_min;
+    d.alpha_max = (float)p.alpha_max;
+    d.eps = (float)p.eps;
+    d.eps_nu = (float)p.eps_nu;
+    d.w_z = (float)p.w_z;
+    d.w_age = (float)p.w_age;
+    d.w_phase = (float)p.w_phase;
+    d.w_cam = (float)p.w_cam;
+    d.w_depth = (float)p.w_depth;
+    d.eta_min = (float)p.eta_min;
+    d.eta_max = (float)p.eta_max;
+    d.beta_d = (float)p.beta_d;
+    d.a_cam = (float)p.a_cam;
+    d.a_depth = (float)p.a_depth;
+    d.a_phase = (float)p.a_phase;
+    d.lam = (p.flags & WDC_ABL_INSTANT_RISK) ? 0.f : (float)p.lambda_;   // instantaneous risk: no accumulation
+    d.tau_risk = (float)p.tau_risk;
     d.flags = p.flags;
     d.period = p.period;
-    d.ridge = p.ridge;
+    d.ridge = (float)p.ridge;
     return d;
 }
 

@@ -26,40 +26,53 @@ constexpr int kOffH = kOffQ + 1;
 enum : unsigned { kErrTimeout = 1u, kErrBounds = 2u, kErrTmem = 4u };
 
 // ---------------------------------------------------------------- device state
-// One bank record (section "Local Lifted Evolution").  The summaries are
-// fp32: the step kernels do their per-element and reduction arithmetic in
-// fp32 (GB300's fp64 rate is a small fraction of its fp32 rate); the scalar
-// fields stay fp64.
+// Device state is fp32 throughout.  On GB300 an fp64 operation has a
+// dependent latency of about 65 cycles (fp32: 5) and a conversion between the
+// two about as much, so the step kernels' scalar chains (lift, retrieval,
+// controller) run in fp32; the host converts at the API boundary, and
+// differences of schedule values (q_{k+1} - q_k, a record's interval) are
+// formed in fp64 on the host and rounded once.
+
+// One bank record (section "Local Lifted Evolution").
 struct DevRecord {
-    float s_in[kSummary], s_out[kSummary], s_dphi[kSummary];
+    alignas(16) float s_in[kSummary];
+    alignas(16) float s_out[kSummary];
+    alignas(16) float s_dphi[kSummary];
     float n_in, n_out;            // Euclidean norms of s_in and s_out
-    double q_in, q_out, r;
-    double cam[4], depth[4];
+    float q_in, q_out, dq, r;     // dq = q_out - q_in (rounded from fp64)
+    float cam[4], depth[4];
 };
 
-// Per-step output mirrored to the host.
+// Per-step output mirrored to the host (widened into wdc_step_info there).
 struct StepOut {
     int decision, finite, supported, n_compat;
-    double q, alpha, p, d_hat, w, delta, R_cand, R, eta, d_cf, d_z, r;
-    double kappa[kMaxBank], pi[kMaxBank];
+    float q, alpha, p, d_hat, w, delta, R_cand, R, eta, d_cf, d_z, r;
+    float kappa[kMaxBank], pi[kMaxBank];
+};
+
+// Schedule values of step k, from the fp64 schedule, rounded once.
+struct StepScalars {
+    float q_k, q_next;            // phases q_k = sigma_k, q_{k+1}
+    float dq;                     // sigma_{k+1} - sigma_k (also Psi's step)
+    float t_model;                // 1000 sigma_k
 };
 
 // Continuous controller/memory state (discrete state -- bank ring, age -- is
 // owned by the host and passed per launch).
 struct DevState {
-    double R, eta;
-    double q_a_in, q_a_out;
-    double cam_a[4], depth_a[4];
+    float R, eta;
+    float q_a_in, q_a_out, q_a_dq;  // latest exact interval and its length
+    float cam_a[4], depth_a[4];
     DevRecord rec[kMaxBank];                       // indexed by ring slot
-    float cur_S[kSketch];                          // raw signed bucket sums over the current latent
-    double cur_sumsq, cur_sumsq_anchor;            // sum z^2, sum (z - z_a)^2
-    float anchor_S[kSketch];
-    double anchor_sumsq;
-    float s_phi[kSummary];                         // summary of the current state (this step)
+    alignas(16) float cur_S[kSketch];              // raw signed bucket sums over the current latent
+    float cur_sumsq, cur_sumsq_anchor;             // sum z^2, sum (z - z_a)^2
+    alignas(16) float anchor_S[kSketch];
+    float anchor_sumsq;
+    alignas(16) float s_phi[kSummary];             // summary of the current state (this step)
     int cand_k, cand_supported, cand_finite;
-    double cand_p;
-    float cand_S[kSketch];
-    double cand_sumsq, cand_sumsq_anchor;
+    float cand_p;
+    alignas(16) float cand_S[kSketch];
+    float cand_sumsq, cand_sumsq_anchor;
     StepOut out;
     // discrete state of the graph rollout (device-resident mirror of the
     // host's ring head, bank size and age)
@@ -70,11 +83,11 @@ struct DevState {
 struct ParamsDev {
     int K, min_support, max_age, n_init_exact, n_final_exact;
     unsigned seed;
-    double sim_min, q_gap_max, gamma_q, tau_in, tau_obs, alpha_min, alpha_max, eps, eps_nu;
-    double w_z, w_age, w_phase, w_cam, w_depth, eta_min, eta_max, beta_d;
-    double a_cam, a_depth, a_phase, lam, tau_risk;   // lam = 0 under WDC_ABL_INSTANT_RISK
+    float sim_min, q_gap_max, gamma_q, tau_in, tau_obs, alpha_min, alpha_max, eps, eps_nu;
+    float w_z, w_age, w_phase, w_cam, w_depth, eta_min, eta_max, beta_d;
+    float a_cam, a_depth, a_phase, lam, tau_risk;    // lam = 0 under WDC_ABL_INSTANT_RISK
     int flags, period;                               // WDC_ABL_* bits; periodic placement
-    double ridge;                                    // linear observation
+    float ridge;                                     // linear observation
 };
 
 enum StreamMode { kModeStats = 0, kModeSkip = 1, kModeAnchor = 2, kModeObserve = 3, kModeSecant = 4, kModeResidual = 5 };
@@ -93,10 +106,9 @@ struct PassArgs {
     const float* zcf;                  // anchor: counterfactual candidate or nullptr
     float* out;                        // skip: z_hat; anchor: z_exact (bank slot)
     float* out2;                       // anchor: z_exact - z_k (the slot's displacement) or nullptr
-    float dsig;                        // anchor: sigma_{k+1} - sigma_k (fp32)
     int k, T, age, ins_slot;
-    double q_k, q_next;
-    double cam[4], depth[4];
+    StepScalars sk;                    // q_k, q_{k+1}, sigma_{k+1} - sigma_k, model timestep
+    float cam[4], depth[4];
     ParamsDev prm;
     DevState* st;
     float* partials;                   // [kPartials][gridDim.x] (value-major)
@@ -121,6 +133,7 @@ struct Ctx {
     int num_sms = 0;
     size_t n = 0;                      // latent numel
     std::vector<double> sigma;         // T+1 noise levels (host, fp64)
+    std::vector<StepScalars> stepf;    // [T] per-step fp32 schedule values
     std::string last_error;
     unsigned long long launches = 0;
 

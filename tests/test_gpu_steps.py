@@ -118,7 +118,8 @@ def test_anchor_pass_parity(n, K):
     assert s.n_bank == len(st_o.bank)
     for i, rec in enumerate(st_o.bank):
         h = s.rec[i]
-        assert h.q_in == pytest.approx(rec.q_in, abs=1e-12) and h.q_out == pytest.approx(rec.q_out, abs=1e-12)
+        # phases are held in fp32 on the device (2^-24 relative)
+        assert h.q_in == pytest.approx(rec.q_in, abs=1e-7) and h.q_out == pytest.approx(rec.q_out, abs=1e-7)
     new = s.rec[s.n_bank - 1]
     ref = st_o.bank[-1]
     assert rel_l2(np.array(new.s_in), ref.s_in) <= TOL
