@@ -357,6 +357,7 @@ struct alignas(16) PassShared {
 static_assert(alignof(PassShared) >= 16 && alignof(StateIn) >= 16 && alignof(RecSummaries) >= 16,
               "float4 snapshot stores need 16-byte aligned shared arrays");
 static_assert(offsetof(PassShared, S) % 16 == 0 && offsetof(PassShared, rs) == 0, "snapshot offsets");
+static_assert(sizeof(PassArgs) % 8 == 0 && alignof(PassArgs) <= 16, "the argument copy moves whole words");
 static_assert(offsetof(StateIn, cur_S) % 16 == 0 && offsetof(StateIn, anchor_S) % 16 == 0 &&
               offsetof(StateIn, s_phi) % 16 == 0, "snapshot vector offsets");
 static_assert((kSummary * sizeof(float)) % 16 == 0, "summary rows stay 16-byte aligned");
@@ -431,10 +432,20 @@ __device__ __forceinline__ float sum_warp_rows(const float (&rows)[kWarps][kSket
 }
 
 template <int MODE, int K>
-__device__ __forceinline__ void pass_body(const PassArgs& a) {
+__device__ __forceinline__ void pass_body(const PassArgs& a_in) {
     __shared__ HeadShared hs;
     __shared__ PassShared ps;
+    // The launch arguments, copied into shared memory by all threads at once:
+    // read in place, every newly touched line of the ~0.6 KB argument block
+    // is a miss of its own, and the head's and the controller tail's scalar
+    // chains walk many of them one after another (several microseconds per
+    // launch, measured).
+    __shared__ __align__(16) uint32_t s_args[(sizeof(PassArgs) + 3) / 4];
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    for (int i = t; i < (int)((sizeof(PassArgs) + 3) / 4); i += kThreads)
+        s_args[i] = reinterpret_cast<const uint32_t*>(&a_in)[i];
+    __syncthreads();
+    const PassArgs& a = *reinterpret_cast<const PassArgs*>(s_args);
     const uint32_t seed = a.prm.seed;
     const long long n = a.n;
     const long long nruns = (n + kRun - 1) / kRun;
