@@ -131,15 +131,47 @@ __global__ void ln_mod_kernel(const T* __restrict__ x, T* __restrict__ h, int r0
     }
 }
 
-// bf16 variant with 16-byte accesses: lane l owns the 8-element vectors
-// l, l+32, ..., so a warp moves 512 contiguous bytes per access (D = 256 NV).
-// The block stages (1 + scale) and shift in shared memory once for its rows
-// instead of every row reading them from L2.
+// bf16 variant for D = 256 NV, a persistent streaming kernel: one block of 8
+// warps per SM, each warp walks rows r0 + warp_id, r0 + warp_id + 8 * grid,
+// ...  Lane l owns the 8-element vectors l, l+32, ... of a row (a warp moves
+// 512 contiguous bytes per access).  Rows arrive through a per-warp ring of
+// kLnRing row buffers in shared memory filled by cp.async (16 bytes per lane
+// per vector): while a warp normalises row i, rows i+1 .. i+kLnRing-1 are in
+// flight, so an SM keeps 8 * kLnRing rows (144 KB at D = 3072) of loads
+// outstanding.  Each lane copies and reads only its own vectors, so its own
+// cp.async.wait_group is all the ordering it needs.  The block stages
+// (1 + scale) and shift in shared memory once.
+constexpr int kLnRing = 3;
+constexpr int kLnWarps = 8;
+
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
+                 "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
 template <int NV>
-__global__ void ln_mod_vec_kernel(const __nv_bfloat16* __restrict__ x, __nv_bfloat16* __restrict__ h, int r0, int r1,
-                                  int D, const float* __restrict__ shift, const float* __restrict__ scale,
-                                  int h_row_off) {
+__global__ void __launch_bounds__(kLnWarps * 32, 1)
+    ln_mod_stream_kernel(const __nv_bfloat16* __restrict__ x, __nv_bfloat16* __restrict__ h, int r0, int r1, int D,
+                         const float* __restrict__ shift, const float* __restrict__ scale, int h_row_off) {
     __shared__ float4 s_sc[NV * 64], s_sh[NV * 64];        // 256 NV floats each
+    extern __shared__ uint4 ring[];                        // [warp][kLnRing][NV * 32]
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int stride = gridDim.x * kLnWarps;
+    uint4* my = ring + (size_t)warp * kLnRing * NV * 32;
+    auto issue = [&](int slot, int row) {
+        if (row < r1) {
+            const uint4* src = reinterpret_cast<const uint4*>(x + (size_t)row * D);
+#pragma unroll
+            for (int i = 0; i < NV; ++i) cp_async16(my + (slot * NV + i) * 32 + lane, src + i * 32 + lane);
+        }
+        cp_async_commit();                                 // one group per row, empty past the end
+    };
+    const int row0 = r0 + blockIdx.x * kLnWarps + warp;
+#pragma unroll
+    for (int j = 0; j < kLnRing - 1; ++j) issue(j, row0 + j * stride);
     for (int i = threadIdx.x; i < NV * 64; i += blockDim.x) {
         float4 a = __ldg(reinterpret_cast<const float4*>(scale) + i);
         a.x += 1.0f; a.y += 1.0f; a.z += 1.0f; a.w += 1.0f;
@@ -147,55 +179,60 @@ __global__ void ln_mod_vec_kernel(const __nv_bfloat16* __restrict__ x, __nv_bflo
         s_sh[i] = __ldg(reinterpret_cast<const float4*>(shift) + i);
     }
     __syncthreads();
-    const int row = r0 + ((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
-    if (row >= r1) return;
-    const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)row * D);
-    float v[NV][8];
-    float s = 0.f;
+    int slot = 0;
+    for (int row = row0; row < r1; row += stride) {
+        issue((slot + kLnRing - 1) % kLnRing, row + (kLnRing - 1) * stride);
+        cp_async_wait<kLnRing - 1>();                      // this lane's copies of `row` have landed
+        const uint4* buf = my + slot * NV * 32;
+        float v[NV][8];
+        float sm = 0.f;
 #pragma unroll
-    for (int i = 0; i < NV; ++i) {
-        const uint4 u = __ldg(xr + i * 32 + lane);
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+        for (int i = 0; i < NV; ++i) {
+            const uint4 u = buf[i * 32 + lane];
+            const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[q]));
-            v[i][2 * q] = f.x;
-            v[i][2 * q + 1] = f.y;
-            s += f.x + f.y;
+            for (int q = 0; q < 4; ++q) {
+                const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[q]));
+                v[i][2 * q] = f.x;
+                v[i][2 * q + 1] = f.y;
+                sm += f.x + f.y;
+            }
         }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) sm += __shfl_xor_sync(0xffffffffu, sm, o);
+        const float mean = sm / (float)D;
+        float q2 = 0.f;
+#pragma unroll
+        for (int i = 0; i < NV; ++i)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const float dlt = v[i][e] - mean;
+                q2 += dlt * dlt;
+            }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) q2 += __shfl_xor_sync(0xffffffffu, q2, o);
+        const float rstd = 1.0f / sqrtf(q2 / (float)D + 1e-6f);
+        uint4* hr = reinterpret_cast<uint4*>(h + (size_t)(row - h_row_off) * D);
+#pragma unroll
+        for (int i = 0; i < NV; ++i) {
+            const int c4 = (i * 32 + lane) * 2;               // float4 index of column (i*32+lane)*8
+            const float4 sc0 = s_sc[c4], sc1 = s_sc[c4 + 1];
+            const float4 sh0 = s_sh[c4], sh1 = s_sh[c4 + 1];
+            const float sc[8] = {sc0.x, sc0.y, sc0.z, sc0.w, sc1.x, sc1.y, sc1.z, sc1.w};
+            const float sh[8] = {sh0.x, sh0.y, sh0.z, sh0.w, sh1.x, sh1.y, sh1.z, sh1.w};
+            uint32_t w[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float a = fmaf((v[i][2 * q] - mean) * rstd, sc[2 * q], sh[2 * q]);
+                const float b = fmaf((v[i][2 * q + 1] - mean) * rstd, sc[2 * q + 1], sh[2 * q + 1]);
+                __nv_bfloat162 hb = __floats2bfloat162_rn(a, b);
+                w[q] = *reinterpret_cast<uint32_t*>(&hb);
+            }
+            hr[i * 32 + lane] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        slot = slot + 1 == kLnRing ? 0 : slot + 1;
     }
-#pragma unroll
-    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    const float mean = s / (float)D;
-    float q2 = 0.f;
-#pragma unroll
-    for (int i = 0; i < NV; ++i)
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            const float dlt = v[i][e] - mean;
-            q2 += dlt * dlt;
-        }
-#pragma unroll
-    for (int o = 16; o; o >>= 1) q2 += __shfl_xor_sync(0xffffffffu, q2, o);
-    const float rstd = 1.0f / sqrtf(q2 / (float)D + 1e-6f);
-    uint4* hr = reinterpret_cast<uint4*>(h + (size_t)(row - h_row_off) * D);
-#pragma unroll
-    for (int i = 0; i < NV; ++i) {
-        const int c4 = (i * 32 + lane) * 2;                   // float4 index of column (i*32+lane)*8
-        const float4 sc0 = s_sc[c4], sc1 = s_sc[c4 + 1];
-        const float4 sh0 = s_sh[c4], sh1 = s_sh[c4 + 1];
-        const float sc[8] = {sc0.x, sc0.y, sc0.z, sc0.w, sc1.x, sc1.y, sc1.z, sc1.w};
-        const float sh[8] = {sh0.x, sh0.y, sh0.z, sh0.w, sh1.x, sh1.y, sh1.z, sh1.w};
-        uint32_t w[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const float a = fmaf((v[i][2 * q] - mean) * rstd, sc[2 * q], sh[2 * q]);
-            const float b = fmaf((v[i][2 * q + 1] - mean) * rstd, sc[2 * q + 1], sh[2 * q + 1]);
-            __nv_bfloat162 hb = __floats2bfloat162_rn(a, b);
-            w[q] = *reinterpret_cast<uint32_t*>(&hb);
-        }
-        hr[i * 32 + lane] = make_uint4(w[0], w[1], w[2], w[3]);
-    }
+    cp_async_wait<0>();                                    // no copy left in flight at exit
 }
 
 // Per-sample device pointers of a batch, passed by value.
@@ -396,7 +433,7 @@ inline unsigned blocks_for(long long n, int per) { return (unsigned)((n + per - 
 
 template <typename T>
 void launch_ln_mod(const void* x, void* h, int r0, int r1, int D, const float* shift, const float* scale,
-                   int h_row_off, cudaStream_t s) {
+                   int h_row_off, int num_sms, cudaStream_t s) {
     const int rows = r1 - r0;
     if (rows <= 0) return;
     const unsigned grid = blocks_for((long long)rows * 32, 256);
@@ -406,7 +443,16 @@ void launch_ln_mod(const void* x, void* h, int r0, int r1, int D, const float* s
         const bool vec_ok = D % 256 == 0 && ((uintptr_t)x & 15) == 0 && ((uintptr_t)h & 15) == 0 &&
                             ((uintptr_t)shift & 15) == 0 && ((uintptr_t)scale & 15) == 0;
         if (vec_ok && D == 3072) {
-            ln_mod_vec_kernel<12><<<grid, 256, 0, s>>>(xp, hp, r0, r1, D, shift, scale, h_row_off);
+            constexpr size_t ring_bytes = (size_t)kLnWarps * kLnRing * 12 * 32 * sizeof(uint4);
+            static bool attr = false;
+            if (!attr) {
+                cudaFuncSetAttribute(ln_mod_stream_kernel<12>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)ring_bytes);
+                attr = true;
+            }
+            const int blocks = (rows + kLnWarps - 1) / kLnWarps;
+            const unsigned g = (unsigned)(blocks < num_sms ? blocks : num_sms);
+            ln_mod_stream_kernel<12><<<g, kLnWarps * 32, ring_bytes, s>>>(xp, hp, r0, r1, D, shift, scale, h_row_off);
             return;
         }
     }
@@ -465,9 +511,9 @@ static void ln_mod(Ctx* c, const void* x, void* h, int r0, int r1, const float* 
     if (r1 <= r0) return;
     LaunchScope ls(c, WDC_K_NORM, s);
     if (c->cfg.dtype == WDC_BF16)
-        launch_ln_mod<__nv_bfloat16>(x, h, r0, r1, c->cfg.hidden, shift, scale, h_row_off, s);
+        launch_ln_mod<__nv_bfloat16>(x, h, r0, r1, c->cfg.hidden, shift, scale, h_row_off, c->num_sms, s);
     else
-        launch_ln_mod<float>(x, h, r0, r1, c->cfg.hidden, shift, scale, h_row_off, s);
+        launch_ln_mod<float>(x, h, r0, r1, c->cfg.hidden, shift, scale, h_row_off, c->num_sms, s);
 }
 
 // ---------------------------------------------------------------- lifetime
