@@ -425,9 +425,9 @@ wdc_status wdc_native_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* co
  * of the library is bracketed by two CUDA events recorded on its launch
  * stream.  wdc_profile_read synchronises the device and returns, per class,
  * the summed event time (ms) and the number of timed launches since the last
- * enable or read (which clears them).  Launches on the denoiser's internal
- * forked stream (the condition rows of a dual-stream model, which run beside
- * timed kernels) are not timed, so the per-class times do not overlap.
+ * enable or read (which clears them).  Every launch of the library is on the
+ * caller's stream (a dual-stream model's condition rows share their GEMM
+ * launches with the video rows), so the per-class times do not overlap.
  * Disabled by default; costs two cudaEventRecord calls per launch when on.
  * Not a method step (no counterpart in the paper). */
 enum wdc_kernel_class {

@@ -51,9 +51,7 @@ static cudaEvent_t next_event(Ctx* c, int cls) {
 
 LaunchScope::LaunchScope(Ctx* c_, int cls_, cudaStream_t s_) : c(c_), cls(cls_), s(s_) {
     c->launches++;
-    // launches on the denoiser's forked stream overlap timed main-stream
-    // kernels: counted in the total, not timed
-    if (c->prof && !(s_ != nullptr && s_ == c->untimed_stream)) {
+    if (c->prof) {
         // reserve both events of the pair up front so begin/end never misalign
         cudaEvent_t b = next_event(c, cls);
         cudaEvent_t e = b ? next_event(c, cls) : nullptr;

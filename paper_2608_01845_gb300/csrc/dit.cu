@@ -25,6 +25,8 @@ namespace wdc {
 // supported so the caller can report it.
 bool tc_gemm_supported(int M, int N, int K);
 wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, const Epi& e, cudaStream_t s);
+wdc_status tc_gemm_grouped(Ctx* c, const void* A0, const void* W0, int M0, const Epi& e0, const void* A1,
+                           const void* W1, int M1, const Epi& e1, int N, int K, cudaStream_t s);
 bool tc_attention_supported(int L, int d);
 wdc_status tc_attention(Ctx* c, const void* q, const void* k, const void* vt, int ldv, void* o, int H, int L, int d,
                         int Hs, int Lc, cudaStream_t s);
@@ -53,11 +55,6 @@ struct DiT {
     float *feat = nullptr, *h1 = nullptr, *temb = nullptr, *mods = nullptr;
     float* vb = nullptr;                  // [B, latent] velocities of a batched forward (B > 1)
     std::vector<void*> allocs;
-    // dual stream: the condition stream's row block runs on a second CUDA
-    // stream forked from and joined back into the caller's, so its small
-    // GEMMs fill the SMs the video GEMMs leave idle in their last wave
-    cudaStream_t aux = nullptr;
-    cudaEvent_t fork[2] = {}, join[2] = {};
     // set while a graph rollout captures the forward: the timestep comes from
     // device memory at replay time
     const float* t_src = nullptr;
@@ -484,6 +481,22 @@ static wdc_status gemm(Ctx* c, const void* A, const void* W, int M, int N, int K
 
 // H heads in all = nb samples x Hs heads; sample b's output rows follow the
 // batch's stream-major token layout (Lc condition tokens per sample).
+// Two GEMMs with the same N and K (the dual-stream block's video rows and
+// condition rows, each with its own weights and epilogue): one grouped
+// tcgen05 launch in bf16, two SIMT launches in the fp32 parity mode.
+static wdc_status gemm2(Ctx* c, const void* A0, const void* W0, int M0, const Epi& e0, const void* A1,
+                        const void* W1, int M1, const Epi& e1, int N, int K, cudaStream_t s) {
+    if (c->cfg.dtype != WDC_BF16) {
+        wdc_status st = gemm(c, A0, W0, M0, N, K, e0, s);
+        return st ? st : gemm(c, A1, W1, M1, N, K, e1, s);
+    }
+    if (!tc_gemm_supported(M0 > 0 ? M0 : 1, N, K))
+        return fail(c, WDC_ERR_UNSUPPORTED, "bf16 GEMM N=" + std::to_string(N) + " K=" + std::to_string(K) +
+                                                ": the tcgen05 GEMM needs N % 32 == 0 and K % 8 == 0");
+    LaunchScope ls(c, WDC_K_GEMM, s);
+    return tc_gemm_grouped(c, A0, W0, M0, e0, A1, W1, M1, e1, N, K, s);
+}
+
 // V^T rows have stride ldv (>= L).  bf16 runs on the tcgen05 kernel only;
 // the SIMT kernel serves the fp32 parity mode.
 static wdc_status attention(Ctx* c, const void* q, const void* k, const void* vt, int ldv, void* o, int H, int L,
@@ -591,15 +604,6 @@ wdc_status dit_create(Ctx* c) {
     if ((s = dalloc(c, (void**)&t->h1, (size_t)t->E * sizeof(float)))) return s;
     if ((s = dalloc(c, (void**)&t->temb, (size_t)t->E * sizeof(float)))) return s;
     if ((s = dalloc(c, (void**)&t->mods, t->mod_rows * sizeof(float)))) return s;
-    if (t->S == 2) {
-        if (cudaStreamCreateWithFlags(&t->aux, cudaStreamNonBlocking) != cudaSuccess)
-            return fail(c, WDC_ERR_CUDA, "DiT init: auxiliary stream");
-        c->untimed_stream = t->aux;
-        for (int i = 0; i < 2; ++i)
-            if (cudaEventCreateWithFlags(&t->fork[i], cudaEventDisableTiming) != cudaSuccess ||
-                cudaEventCreateWithFlags(&t->join[i], cudaEventDisableTiming) != cudaSuccess)
-                return fail(c, WDC_ERR_CUDA, "DiT init: stream events");
-    }
     const long long npe = (long long)t->Lv * t->D;
     LaunchScope ls(c, WDC_K_OTHER, 0);
     if (t->dtype == WDC_BF16)
@@ -614,12 +618,6 @@ wdc_status dit_create(Ctx* c) {
 void dit_destroy(Ctx* c) {
     if (!c->dit) return;
     for (void* p : c->dit->allocs) cudaFree(p);
-    for (int i = 0; i < 2; ++i) {
-        if (c->dit->fork[i]) cudaEventDestroy(c->dit->fork[i]);
-        if (c->dit->join[i]) cudaEventDestroy(c->dit->join[i]);
-    }
-    if (c->dit->aux) cudaStreamDestroy(c->dit->aux);
-    c->untimed_stream = nullptr;
     delete c->dit;
     c->dit = nullptr;
 }
@@ -789,62 +787,65 @@ static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, int nb
     if (t->S == 2) { r0[0] = nb * t->Lc; r1[0] = nb * t->L; r0[1] = 0; r1[1] = nb * t->Lc; }
     else { r0[0] = 0; r1[0] = nb * t->L; }
     wdc_status st;
-    // per-stream CUDA streams: the condition rows (dual stream) on t->aux,
-    // forked before and joined after each half of the block; every buffer
-    // they touch (h, q/k/vt, ao, m, x) is split by rows
-    cudaStream_t ss[2] = {s, t->S == 2 ? t->aux : s};
-    auto fork = [&](int i) -> wdc_status {
-        if (t->S < 2) return WDC_OK;
-        WDC_CUDA_TRY(c, cudaEventRecord(t->fork[i], s));
-        WDC_CUDA_TRY(c, cudaStreamWaitEvent(t->aux, t->fork[i], 0));
-        return WDC_OK;
+    // Each GEMM of the block is one launch: with dual-stream weights the
+    // video rows and the condition rows (each with its stream's weights and
+    // modulation) are the two problems of one grouped launch, so the
+    // condition rows' tiles fill the SMs the video tiles leave idle in their
+    // last wave.  The LayerNorms run per row range.
+    const int S = t->S;
+    const float* m6[2] = {mod, mod + (size_t)(S - 1) * 6 * D};
+    auto rows_of = [&](int sidx) { return r1[sidx] - r0[sidx]; };
+    auto at_row = [&](void* base, int sidx, int width) { return (char*)base + (size_t)r0[sidx] * width * es; };
+    auto lin_gemm = [&](const std::vector<Lin>& W, const void* A, int width, int N, Epi* e) -> wdc_status {
+        const Lin& w0 = W[layer * S];
+        if (S == 1) return gemm(c, at_row(const_cast<void*>(A), 0, width), w0.w, rows_of(0), N, width, e[0], s);
+        const Lin& w1 = W[layer * S + 1];
+        return gemm2(c, at_row(const_cast<void*>(A), 0, width), w0.w, rows_of(0), e[0],
+                     at_row(const_cast<void*>(A), 1, width), w1.w, rows_of(1), e[1], N, width, s);
     };
-    auto join = [&](int i) -> wdc_status {
-        if (t->S < 2) return WDC_OK;
-        WDC_CUDA_TRY(c, cudaEventRecord(t->join[i], t->aux));
-        WDC_CUDA_TRY(c, cudaStreamWaitEvent(s, t->join[i], 0));
-        return WDC_OK;
-    };
-    if ((st = fork(0))) return st;
-    for (int sidx = 0; sidx < t->S; ++sidx) {
-        const float* m6 = mod + (size_t)sidx * 6 * D;
-        cudaStream_t s = ss[sidx];
-        ln_mod(c, x, t->h, r0[sidx], r1[sidx], m6 + 0 * D, m6 + 1 * D, 0, s);
-        const Lin& w = t->qkv[layer * t->S + sidx];
-        Epi e{};
-        e.mode = kEpiQKV; e.bias = w.b; e.q = t->q; e.k = t->k; e.vt = t->vt;
-        e.L = t->L; e.H = t->H; e.d = t->d; e.D = D; e.row_off = r0[sidx]; e.nb = nb; e.Lc = t->Lc; e.ldv = t->ldv;
-        if ((st = gemm(c, (char*)t->h + (size_t)r0[sidx] * D * es, w.w, r1[sidx] - r0[sidx], 3 * D, D, e, s))) return st;
+    for (int sidx = 0; sidx < S; ++sidx) ln_mod(c, x, t->h, r0[sidx], r1[sidx], m6[sidx] + 0 * D, m6[sidx] + 1 * D, 0, s);
+    {
+        Epi e[2];
+        for (int sidx = 0; sidx < S; ++sidx) {
+            e[sidx] = Epi{};
+            e[sidx].mode = kEpiQKV; e[sidx].bias = t->qkv[layer * S + sidx].b;
+            e[sidx].q = t->q; e[sidx].k = t->k; e[sidx].vt = t->vt;
+            e[sidx].L = t->L; e[sidx].H = t->H; e[sidx].d = t->d; e[sidx].D = D; e[sidx].row_off = r0[sidx];
+            e[sidx].nb = nb; e[sidx].Lc = t->Lc; e[sidx].ldv = t->ldv;
+        }
+        if ((st = lin_gemm(t->qkv, t->h, D, 3 * D, e))) return st;
     }
-    if ((st = join(0))) return st;
     if ((st = attention(c, t->q, t->k, t->vt, t->ldv, t->ao, nb * t->H, t->L, t->d, t->H, t->Lc, s))) return st;
-    if ((st = fork(1))) return st;
-    for (int sidx = 0; sidx < t->S; ++sidx) {
-        const float* m6 = mod + (size_t)sidx * 6 * D;
-        cudaStream_t s = ss[sidx];
-        const int rows = r1[sidx] - r0[sidx];
-        char* xr = (char*)x + (size_t)r0[sidx] * D * es;
-        {
-            const Lin& w = t->o[layer * t->S + sidx];
-            Epi e{};
-            e.mode = kEpiResid; e.bias = w.b; e.out = xr; e.res = xr; e.ldo = D; e.gate = m6 + 2 * D;
-            if ((st = gemm(c, (char*)t->ao + (size_t)r0[sidx] * D * es, w.w, rows, D, D, e, s))) return st;
+    {
+        Epi e[2];
+        for (int sidx = 0; sidx < S; ++sidx) {
+            char* xr = at_row(x, sidx, D);
+            e[sidx] = Epi{};
+            e[sidx].mode = kEpiResid; e[sidx].bias = t->o[layer * S + sidx].b; e[sidx].out = xr; e[sidx].res = xr;
+            e[sidx].ldo = D; e[sidx].gate = m6[sidx] + 2 * D;
         }
-        ln_mod(c, x, t->h, r0[sidx], r1[sidx], m6 + 3 * D, m6 + 4 * D, 0, s);
-        {
-            const Lin& w = t->fc1[layer * t->S + sidx];
-            Epi e{};
-            e.mode = kEpiStore; e.bias = w.b; e.gelu = 1; e.out = (char*)t->m + (size_t)r0[sidx] * t->M * es; e.ldo = t->M;
-            if ((st = gemm(c, (char*)t->h + (size_t)r0[sidx] * D * es, w.w, rows, t->M, D, e, s))) return st;
-        }
-        {
-            const Lin& w = t->fc2[layer * t->S + sidx];
-            Epi e{};
-            e.mode = kEpiResid; e.bias = w.b; e.out = xr; e.res = xr; e.ldo = D; e.gate = m6 + 5 * D;
-            if ((st = gemm(c, (char*)t->m + (size_t)r0[sidx] * t->M * es, w.w, rows, D, t->M, e, s))) return st;
-        }
+        if ((st = lin_gemm(t->o, t->ao, D, D, e))) return st;
     }
-    if ((st = join(1))) return st;
+    for (int sidx = 0; sidx < S; ++sidx) ln_mod(c, x, t->h, r0[sidx], r1[sidx], m6[sidx] + 3 * D, m6[sidx] + 4 * D, 0, s);
+    {
+        Epi e[2];
+        for (int sidx = 0; sidx < S; ++sidx) {
+            e[sidx] = Epi{};
+            e[sidx].mode = kEpiStore; e[sidx].bias = t->fc1[layer * S + sidx].b; e[sidx].gelu = 1;
+            e[sidx].out = at_row(t->m, sidx, t->M); e[sidx].ldo = t->M;
+        }
+        if ((st = lin_gemm(t->fc1, t->h, D, t->M, e))) return st;
+    }
+    {
+        Epi e[2];
+        for (int sidx = 0; sidx < S; ++sidx) {
+            char* xr = at_row(x, sidx, D);
+            e[sidx] = Epi{};
+            e[sidx].mode = kEpiResid; e[sidx].bias = t->fc2[layer * S + sidx].b; e[sidx].out = xr; e[sidx].res = xr;
+            e[sidx].ldo = D; e[sidx].gate = m6[sidx] + 5 * D;
+        }
+        if ((st = lin_gemm(t->fc2, t->m, t->M, D, e))) return st;
+    }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("block: ") + cudaGetErrorString(e));
     return WDC_OK;

@@ -45,6 +45,11 @@ struct GemmArgs {
     int group_n;            // pair kernel: N tiles per raster group
     Epi e;
     unsigned* err;
+    // pair kernel, grouped launch: a second problem with the same N and K
+    // (its own A, W, M and epilogue) whose tiles follow the first problem's
+    int nprob;              // 1 or 2
+    int M1, m_pairs1;
+    Epi e1;
 };
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
@@ -318,8 +323,25 @@ __device__ __forceinline__ void pair_tile(const GemmArgs& g, int m_pairs, int ti
     n_blk = n_first + (r - m_blk * width);
 }
 
+// Tile `tile` of a (possibly grouped) pair launch: problem index, 256-row M
+// block and N block.  The first problem's tiles use the raster groups, the
+// second problem's follow in plain N-fastest order, so they fill the pairs
+// the first problem leaves idle in its last wave.
+__device__ __forceinline__ int grouped_tile(const GemmArgs& g, int m_pairs0, int tiles0, int tile, int& m_blk,
+                                            int& n_blk) {
+    if (tile < tiles0) {
+        pair_tile(g, m_pairs0, tile, m_blk, n_blk);
+        return 0;
+    }
+    const int r = tile - tiles0;
+    m_blk = r / g.n_tiles;
+    n_blk = r - m_blk * g.n_tiles;
+    return 1;
+}
+
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
                     const __grid_constant__ GemmArgs g) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -335,7 +357,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t rank = cluster_ctarank();
     const int cluster_id = blockIdx.x >> 1, n_clusters = gridDim.x >> 1;
     const int m_pairs = (g.m_tiles + 1) >> 1;  // 256-row tiles (m_tiles counts 128-row tiles)
-    const int num_tiles = m_pairs * g.n_tiles;
+    const int tiles0 = m_pairs * g.n_tiles;
+    const int num_tiles = tiles0 + (g.nprob > 1 ? g.m_pairs1 * g.n_tiles : 0);
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES2; ++s) {
             mbar_init(&full[s], 1);
@@ -352,6 +375,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (warp == 0 && lane == 0) {
         prefetch_tmap(&tmA);
         prefetch_tmap(&tmB);
+        if (g.nprob > 1) {
+            prefetch_tmap(&tmA1);
+            prefetch_tmap(&tmB1);
+        }
     }
     if (warp == 1) {
         tmem_alloc2(tmem_slot, TMEM2_COLS);
@@ -376,7 +403,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bool ok = true;
             for (int tile = cluster_id; tile < num_tiles && ok; tile += n_clusters) {
                 int mb, nb;
-                pair_tile(g, m_pairs, tile, mb, nb);
+                const int prob = grouped_tile(g, m_pairs, tiles0, tile, mb, nb);
+                const CUtensorMap* mA = prob ? &tmA1 : &tmA;
+                const CUtensorMap* mB = prob ? &tmB1 : &tmB;
                 const int m0 = mb * 256 + (int)rank * 128;
                 const int n0 = nb * BN + (int)rank * 128;
                 for (int kb = 0; kb < g.k_blocks; ++kb) {
@@ -384,8 +413,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * STAGE2_BYTES);
                     const uint32_t fb = mapa_shared(smem_u32(&full[stage]), 0);
                     uint8_t* sa = smem + stage * STAGE2_BYTES;
-                    tma_load_2d_pair(sa, &tmA, fb, kb * BK, m0);
-                    tma_load_2d_pair(sa + A2_BYTES, &tmB, fb, kb * BK, n0);
+                    tma_load_2d_pair(sa, mA, fb, kb * BK, m0);
+                    tma_load_2d_pair(sa + A2_BYTES, mB, fb, kb * BK, n0);
                     armed[stage] = true;
                     armed_phase[stage] = phase;
                     if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
@@ -443,7 +472,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         uint32_t acc_phase = 0;
         for (int tile = cluster_id; tile < num_tiles; tile += n_clusters) {
             int mb, n_blk;
-            pair_tile(g, m_pairs, tile, mb, n_blk);
+            const int prob = grouped_tile(g, m_pairs, tiles0, tile, mb, n_blk);
+            const int Mp = prob ? g.M1 : g.M;
             const int mrow = mb * 256 + (int)rank * 128;
             if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, g.err)) break;
             tc_fence_after();
@@ -455,7 +485,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 uint32_t r[32];
                 tmem_ld32(taddr + c0, r);
                 tmem_ld_wait();
-                if (m < g.M) epilogue_chunk(g.e, m, col0, r);
+                if (m < Mp) {
+                    // two direct calls (each reads its epilogue from the
+                    // kernel parameters; a selected reference would copy it)
+                    if (prob) epilogue_chunk(g.e1, m, col0, r);
+                    else epilogue_chunk(g.e, m, col0, r);
+                }
             }
             tc_fence_before();
             __syncwarp();
@@ -526,7 +561,9 @@ bool encode_tmap_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1
 
 bool tc_gemm_supported(int M, int N, int K) { return M > 0 && N > 0 && K > 0 && N % 32 == 0 && K % 8 == 0; }
 
-wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, const Epi& e, cudaStream_t s) {
+namespace {
+
+wdc_status check_operands(Ctx* c, const void* A, const void* W, const Epi& e) {
     if (((uintptr_t)A & 15) || ((uintptr_t)W & 15)) return fail(c, WDC_ERR_INVALID_ARG, "GEMM operands must be 16-byte aligned");
     if ((e.mode == kEpiStore || e.mode == kEpiResid) &&
         (e.ldo % 8 || ((uintptr_t)e.out & 15) || (e.res && ((uintptr_t)e.res & 15))))
@@ -534,76 +571,130 @@ wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, co
     if (e.bias && ((uintptr_t)e.bias & 15)) return fail(c, WDC_ERR_INVALID_ARG, "bias must be 16-byte aligned");
     if (e.gate && ((uintptr_t)e.gate & 15)) return fail(c, WDC_ERR_INVALID_ARG, "gate must be 16-byte aligned");
     if (e.mode == kEpiQKV && (e.D % 32 || e.d % 32)) return fail(c, WDC_ERR_UNSUPPORTED, "QKV epilogue needs d % 32 == 0");
+    return WDC_OK;
+}
+
+void set_attrs() {
     static bool attr_set = false;
     if (!attr_set) {
         cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
         cudaFuncSetAttribute(gemm_tc2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM2_BYTES);
         attr_set = true;
     }
-    const bool pair = M >= 256 && c->num_sms >= 2;
-    CUtensorMap ta, tb;
-    std::string why;
-    if (!encode_tmap_2d(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, BK, BM, &why) ||
-        !encode_tmap_2d(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, BK, pair ? BN / 2 : BN, &why))
-        return fail(c, WDC_ERR_CUDA, why);
-    GemmArgs g;
+}
+
+GemmArgs make_args(Ctx* c, int M, int N, int K, const Epi& e) {
+    GemmArgs g{};
     g.M = M;
     g.N = N;
     g.K = K;
     g.m_tiles = (M + BM - 1) / BM;
     g.n_tiles = (N + BN - 1) / BN;
     g.k_blocks = (K + BK - 1) / BK;
-    {
-        // raster groups: a W slab of at most ~40 MB per group (L2 is 126 MB,
-        // shared with the streamed A and the output), as few groups as that
-        // allows.  For deep K (> 4096) a 256-row slab of A is itself large
-        // and re-reading A per group costs more than it saves (measured on the
-        // 17776 x 3072 x 12288 MLP-down GEMM): plain N-fastest order there.
-        g.group_n = g.n_tiles;
-        if (K <= 4096) {
-            const double slab_per_tile = 256.0 * K * 2.0;
-            int gn = (int)(40.0e6 / slab_per_tile);
-            gn = gn < 1 ? 1 : (gn > g.n_tiles ? g.n_tiles : gn);
-            const int groups = (g.n_tiles + gn - 1) / gn;
-            g.group_n = (g.n_tiles + groups - 1) / groups;  // balance the groups
-        }
+    // raster groups: a W slab of at most ~40 MB per group (L2 is 126 MB,
+    // shared with the streamed A and the output), as few groups as that
+    // allows.  For deep K (> 4096) a 256-row slab of A is itself large
+    // and re-reading A per group costs more than it saves (measured on the
+    // 17776 x 3072 x 12288 MLP-down GEMM): plain N-fastest order there.
+    g.group_n = g.n_tiles;
+    if (K <= 4096) {
+        const double slab_per_tile = 256.0 * K * 2.0;
+        int gn = (int)(40.0e6 / slab_per_tile);
+        gn = gn < 1 ? 1 : (gn > g.n_tiles ? g.n_tiles : gn);
+        const int groups = (g.n_tiles + gn - 1) / gn;
+        g.group_n = (g.n_tiles + groups - 1) / groups;  // balance the groups
     }
     g.e = e;
     g.err = c->err;
-    if (pair) {
-        const int tiles = ((g.m_tiles + 1) / 2) * g.n_tiles;
-        cudaLaunchConfig_t cfg = {};
-        cfg.blockDim = dim3(kGemmThreads, 1, 1);
-        cfg.dynamicSmemBytes = SMEM2_BYTES;
-        cfg.stream = s;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = 2;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        // persistent grid: only as many pairs as can be resident at once
-        static int max_clusters = 0;
-        if (max_clusters == 0) {
-            cfg.gridDim = dim3(c->num_sms, 1, 1);
-            if (cudaOccupancyMaxActiveClusters(&max_clusters, gemm_tc2_kernel, &cfg) != cudaSuccess || max_clusters < 1) {
-                cudaGetLastError();
-                max_clusters = c->num_sms / 2;
-            }
+    g.nprob = 1;
+    return g;
+}
+
+// Pair-kernel launch: a persistent grid of as many CTA pairs as can be
+// resident, capped by the tile count.
+wdc_status launch_pair(Ctx* c, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& ta1,
+                       const CUtensorMap& tb1, const GemmArgs& g, cudaStream_t s) {
+    const int tiles = ((g.m_tiles + 1) / 2) * g.n_tiles + (g.nprob > 1 ? g.m_pairs1 * g.n_tiles : 0);
+    cudaLaunchConfig_t cfg = {};
+    cfg.blockDim = dim3(kGemmThreads, 1, 1);
+    cfg.dynamicSmemBytes = SMEM2_BYTES;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    static int max_clusters = 0;
+    if (max_clusters == 0) {
+        cfg.gridDim = dim3(c->num_sms, 1, 1);
+        if (cudaOccupancyMaxActiveClusters(&max_clusters, gemm_tc2_kernel, &cfg) != cudaSuccess || max_clusters < 1) {
+            cudaGetLastError();
+            max_clusters = c->num_sms / 2;
         }
-        int clusters = max_clusters < c->num_sms / 2 ? max_clusters : c->num_sms / 2;
-        if (tiles < clusters) clusters = tiles;
-        cfg.gridDim = dim3(2 * clusters, 1, 1);
-        cudaLaunchKernelEx(&cfg, gemm_tc2_kernel, ta, tb, g);
-    } else {
-        const int tiles = g.m_tiles * g.n_tiles;
-        const int grid = tiles < c->num_sms ? tiles : c->num_sms;
-        gemm_tc_kernel<<<grid, kGemmThreads, SMEM_BYTES, s>>>(ta, tb, g);
     }
+    int clusters = max_clusters < c->num_sms / 2 ? max_clusters : c->num_sms / 2;
+    if (tiles < clusters) clusters = tiles;
+    cfg.gridDim = dim3(2 * clusters, 1, 1);
+    cudaLaunchKernelEx(&cfg, gemm_tc2_kernel, ta, tb, ta1, tb1, g);
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(err));
     return WDC_OK;
+}
+
+}  // namespace
+
+wdc_status tc_gemm(Ctx* c, const void* A, const void* W, int M, int N, int K, const Epi& e, cudaStream_t s) {
+    wdc_status st = check_operands(c, A, W, e);
+    if (st) return st;
+    set_attrs();
+    const bool pair = M >= 256 && c->num_sms >= 2;
+    CUtensorMap ta, tb;
+    std::string why;
+    if (!encode_tmap_2d(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, BK, BM, &why) ||
+        !encode_tmap_2d(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, BK, pair ? BN / 2 : BN, &why))
+        return fail(c, WDC_ERR_CUDA, why);
+    const GemmArgs g = make_args(c, M, N, K, e);
+    if (pair) return launch_pair(c, ta, tb, ta, tb, g, s);
+    const int tiles = g.m_tiles * g.n_tiles;
+    const int grid = tiles < c->num_sms ? tiles : c->num_sms;
+    gemm_tc_kernel<<<grid, kGemmThreads, SMEM_BYTES, s>>>(ta, tb, g);
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(err));
+    return WDC_OK;
+}
+
+// Two GEMMs with the same N and K in one launch of the pair kernel (the
+// dual-stream blocks' video rows and condition rows): problem 1's tiles
+// follow problem 0's, filling the pairs problem 0 leaves idle in its last
+// wave.  When problem 0 is too short for the pair kernel the two run as two
+// launches on the stream.
+wdc_status tc_gemm_grouped(Ctx* c, const void* A0, const void* W0, int M0, const Epi& e0, const void* A1,
+                           const void* W1, int M1, const Epi& e1, int N, int K, cudaStream_t s) {
+    if (M1 <= 0) return tc_gemm(c, A0, W0, M0, N, K, e0, s);
+    if (M0 <= 0) return tc_gemm(c, A1, W1, M1, N, K, e1, s);
+    if (M0 < 256 || c->num_sms < 2) {
+        wdc_status st = tc_gemm(c, A0, W0, M0, N, K, e0, s);
+        return st ? st : tc_gemm(c, A1, W1, M1, N, K, e1, s);
+    }
+    wdc_status st = check_operands(c, A0, W0, e0);
+    if (!st) st = check_operands(c, A1, W1, e1);
+    if (st) return st;
+    set_attrs();
+    CUtensorMap ta, tb, ta1, tb1;
+    std::string why;
+    if (!encode_tmap_2d(&ta, A0, (uint64_t)K, (uint64_t)M0, (uint64_t)K * 2, BK, BM, &why) ||
+        !encode_tmap_2d(&tb, W0, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, BK, BN / 2, &why) ||
+        !encode_tmap_2d(&ta1, A1, (uint64_t)K, (uint64_t)M1, (uint64_t)K * 2, BK, BM, &why) ||
+        !encode_tmap_2d(&tb1, W1, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, BK, BN / 2, &why))
+        return fail(c, WDC_ERR_CUDA, why);
+    GemmArgs g = make_args(c, M0, N, K, e0);
+    g.nprob = 2;
+    g.M1 = M1;
+    g.m_pairs1 = (M1 + 255) / 256;
+    g.e1 = e1;
+    return launch_pair(c, ta, tb, ta1, tb1, g, s);
 }
 
 }  // namespace wdc

@@ -166,7 +166,6 @@ struct Ctx {
 
     // optional per-class event timing (wdc_profile_enable)
     bool prof = false;
-    cudaStream_t untimed_stream = nullptr;  // the denoiser's forked stream (dual stream): not profiled
     std::vector<cudaEvent_t> ev[WDC_K_COUNT];      // begin/end pairs
     size_t ev_used[WDC_K_COUNT] = {};
     unsigned long long cls_launches[WDC_K_COUNT] = {};

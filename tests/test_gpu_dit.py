@@ -285,10 +285,10 @@ def test_bf16_gemm_sampled_full_size_and_no_device_errors(M, N, K):
     assert ctx.device_errors() == 0
 
 
-def test_profiler_times_main_stream_launches_only():
-    """The event profiler times the main stream's launches; the condition
-    rows' kernels of a dual-stream model (forked stream, overlapping the timed
-    ones) count in the total launch number but are not timed."""
+def test_profiler_times_every_launch_and_dual_stream_gemms_are_grouped():
+    """The event profiler times every launch (all on the caller's stream); a
+    dual-stream block issues each of its four GEMMs as one grouped launch over
+    the video and the condition rows, and one LayerNorm launch per row range."""
     cfgd = dict(PARITY_MODEL, layers=1, dual_stream=1)
     ctx = _ctx(cfgd, wdc.BF16)
     ctx.init_weights(3, 0.02)
@@ -302,10 +302,9 @@ def test_profiler_times_main_stream_launches_only():
     ctx.dit_forward(z, 500.0, ct, v)
     prof = ctx.profile_read()
     ctx.profile_enable(False)
-    # main stream: condition and patch embeddings, the video rows' 4 block GEMMs, the final GEMM
+    # condition and patch embeddings, the block's 4 grouped GEMMs, the final GEMM
     assert prof["gemm"][1] == 7
     assert prof["attention"][1] == 1
-    assert prof["norm"][1] == 3                    # the video rows' two LayerNorms + the final one
-    # the forked stream adds the condition rows' 4 GEMMs and 2 LayerNorms
-    assert ctx.launches - n0 == sum(n for _, n in prof.values()) + 6
+    assert prof["norm"][1] == 5                    # 2 row ranges x 2 LayerNorms + the final one
+    assert ctx.launches - n0 == sum(n for _, n in prof.values())
     assert all(ms > 0 for ms, n in prof.values() if n)
