@@ -312,16 +312,45 @@ def skip_pass_gbps(torch, wdc, peaks, secant=False, n=SKIP_SWEEP_N, K=4, flush=T
             "frac_of_measured_copy": gbs / peaks["hbm_gbs"], "l2": "flushed" if flush else "resident"}
 
 
+def copy_ms(torch, nbytes, reps=10):
+    """A plain device copy (torch's copy_) moving `nbytes` in all (half read,
+    half written), L2 flushed before each, CUDA events, median of `reps`: the
+    bandwidth a copy itself reaches at that size (the measured peak is a 2 GB
+    copy; short copies pay their ramp and tail)."""
+    n = max(1, nbytes // 8)
+    a = torch.randn(n, device="cuda")
+    b = torch.empty_like(a)
+    buf = torch.empty(128 * 1024 * 1024, device="cuda")
+    for _ in range(3):
+        b.copy_(a)
+    ts = []
+    for _ in range(reps):
+        buf.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        b.copy_(a)
+        e1.record()
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    del a, b, buf
+    torch.cuda.empty_cache()
+    return statistics.median(ts)
+
+
 def skip_sweep(torch, wdc, peaks, workload_n):
     """The skipped-step kernel sweep: N in {2^20, 2^24, 2^26, 2^28} fp32
     elements x K in {2, 3, 4} bank records, L2 flushed before every launch;
-    plus 2^20 L2-resident and the workload's own latent size."""
+    plus 2^20 L2-resident and the workload's own latent size.  Each row also
+    gives a plain copy of the same byte count timed the same way, and the
+    pass's time against it."""
     rows = []
     for e in (20, 24, 26, 28):
         for K in (2, 3, 4):
             r = skip_pass_gbps(torch, wdc, peaks, n=1 << e, K=K)
+            cms = copy_ms(torch, r["bytes"])
             rows.append({"n": f"2^{e}", "K": K, "gbps": round(r["gbps"], 1), "ms": round(r["ms"], 5),
-                         "frac_of_measured_copy": round(r["frac_of_measured_copy"], 4)})
+                         "frac_of_measured_copy": round(r["frac_of_measured_copy"], 4),
+                         "same_bytes_copy_ms": round(cms, 5), "frac_of_same_bytes_copy": round(cms / r["ms"], 4)})
     r = skip_pass_gbps(torch, wdc, peaks, n=1 << 20, K=4, flush=False)
     rows.append({"n": "2^20", "K": 4, "l2": "resident", "gbps": round(r["gbps"], 1), "ms": round(r["ms"], 5),
                  "frac_of_measured_copy": round(r["frac_of_measured_copy"], 4)})
@@ -329,6 +358,7 @@ def skip_sweep(torch, wdc, peaks, workload_n):
     rows.append({"n": workload_n, "K": 4, "note": "the rollout's own latent", "gbps": round(r["gbps"], 1),
                  "ms": round(r["ms"], 5), "frac_of_measured_copy": round(r["frac_of_measured_copy"], 4)})
     return {"bytes_per_launch": "(K+1)*4*N", "timing": "CUDA events on the launching stream, mean of 10",
+            "same_bytes_copy": "torch copy_ of the same total bytes (half read, half written), median of 10",
             "rows": rows}
 
 

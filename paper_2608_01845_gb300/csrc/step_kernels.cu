@@ -214,23 +214,25 @@ __device__ __noinline__ void linear_readout(const PassArgs& a, const RecSummarie
     }
 }
 
-// Skip-pass head, Eq. 2-5 scalar part, in fp32 (every CTA computes it; it is
-// a few hundred cycles of latency, and no CTA has to wait for another).
+// Skip-pass head, Eq. 2-5 scalar part, in fp32 (every CTA computes it, so no
+// CTA has to wait for another).  The head and the controller tails are one
+// chain of dependent scalar steps per launch, so they use the fast division
+// and exponential intrinsics (a few ulp; the tolerances are 1e-5).
 template <int K>
 __device__ void skip_head(const PassArgs& a, const StateIn& S, const RecSummaries& rs, HeadShared& hs) {
     const int t = threadIdx.x;
     const float N = (float)a.n;
-    const float sc = sqrtf((float)kSketch / N);
+    const float sc = sqrtf(__fdividef((float)kSketch, N));
     const float eps_nu = a.prm.eps_nu;
     const bool no_cond = a.prm.flags & WDC_ABL_NO_COND;
     // s(phi_k): current-state summary (Eq. 2 through the linear sketch)
     if (t < kSummary) {
         float val;
         if (t < kSketch) {
-            val = sc * S.cur_S[t] / (sqrtf(S.cur_sumsq / N) + eps_nu);
+            val = __fdividef(sc * S.cur_S[t], sqrtf(__fdividef(S.cur_sumsq, N)) + eps_nu);
         } else if (t < 2 * kSketch) {
             const int b = t - kSketch;
-            val = sc * (S.cur_S[b] - S.anchor_S[b]) / (sqrtf(S.cur_sumsq_anchor / N) + eps_nu);
+            val = __fdividef(sc * (S.cur_S[b] - S.anchor_S[b]), sqrtf(__fdividef(S.cur_sumsq_anchor, N)) + eps_nu);
         } else if (t < kOffDepth) {
             val = no_cond ? 0.f : a.cam[t - kOffCam];
         } else if (t < kOffQ) {
@@ -246,14 +248,14 @@ __device__ void skip_head(const PassArgs& a, const StateIn& S, const RecSummarie
             } else if (j < 6) {
                 if (j - 3 < a.nsrc) val = -(float)a.T * S.dq[a.nsrc - 1 - (j - 3)];
             } else {
-                val = (float)a.nsrc / (float)a.prm.K;
+                val = __fdividef((float)a.nsrc, (float)a.prm.K);
             }
         }
         hs.phi[t] = val;
     }
     if (t == 0) {
         // Eq. 4: alpha = clip(|q_{t-1}-q_t| / (|q_{a-1}-q_a| + eps), alpha_min, alpha_max)
-        const float raw = fabsf(a.sk.dq) / (fabsf(S.q_a_dq) + a.prm.eps);
+        const float raw = __fdividef(fabsf(a.sk.dq), fabsf(S.q_a_dq) + a.prm.eps);
         hs.alpha = fminf(fmaxf(raw, a.prm.alpha_min), a.prm.alpha_max);
     }
     __syncthreads();
@@ -271,13 +273,13 @@ __device__ void skip_head(const PassArgs& a, const StateIn& S, const RecSummarie
     if (t == 0) {
         const float nphi = sqrtf(hs.red[K]);
         const bool filter = !(a.prm.flags & WDC_ABL_NO_SUPPORT);   // w/o support: N_t = whole bank
-        const float gq = a.prm.gamma_q, inv_tin = 1.0f / a.prm.tau_in;
+        const float gq = a.prm.gamma_q, inv_tin = __fdividef(1.0f, a.prm.tau_in);
         int nc = 0;
         float mx = -INFINITY;
         float ell[K > 0 ? K : 1];
 #pragma unroll
         for (int i = 0; i < K; ++i) {
-            const float s = (nphi == 0.f || S.n_in[i] == 0.f) ? 0.f : hs.red[i] / (nphi * S.n_in[i]);
+            const float s = (nphi == 0.f || S.n_in[i] == 0.f) ? 0.f : __fdividef(hs.red[i], nphi * S.n_in[i]);
             const float dq = a.sk.q_k - S.q_in[i];
             hs.sim_in[i] = s;
             const int c = !filter || ((s >= a.prm.sim_min) && (fabsf(dq) <= a.prm.q_gap_max));
@@ -288,11 +290,13 @@ __device__ void skip_head(const PassArgs& a, const StateIn& S, const RecSummarie
         float tot = 0.f;
 #pragma unroll
         for (int i = 0; i < K; ++i) {
-            hs.pi[i] = hs.compat[i] ? expf(ell[i] - mx) : 0.f;
+            hs.pi[i] = hs.compat[i] ? __expf(ell[i] - mx) : 0.f;
             tot += hs.pi[i];
         }
 #pragma unroll
-        for (int i = 0; i < K; ++i) hs.pi[i] = (nc > 0) ? hs.pi[i] / tot : 0.f;
+        const float inv_tot = nc > 0 ? __fdividef(1.0f, tot) : 0.f;
+#pragma unroll
+        for (int i = 0; i < K; ++i) hs.pi[i] *= inv_tot;
         hs.n_compat = nc;
         hs.supported = filter ? (nc >= a.prm.min_support) : 1;
     }
@@ -316,20 +320,20 @@ __device__ void skip_head(const PassArgs& a, const StateIn& S, const RecSummarie
     }
     if (t == 0) {
         const float nh = sqrtf(hs.red[K]);
-        const float inv_tau = 1.0f / a.prm.tau_obs;
+        const float inv_tau = __fdividef(1.0f, a.prm.tau_obs);
         float mx = -INFINITY;
         float e[K > 0 ? K : 1];
 #pragma unroll
         for (int i = 0; i < K; ++i) {
-            const float s = (nh == 0.f || S.n_out[i] == 0.f) ? 0.f : hs.red[i] / (nh * S.n_out[i]);
+            const float s = (nh == 0.f || S.n_out[i] == 0.f) ? 0.f : __fdividef(hs.red[i], nh * S.n_out[i]);
             hs.sim_out[i] = s;
             e[i] = s * inv_tau;
             mx = fmaxf(mx, e[i]);
         }
         float tot = 0.f;
 #pragma unroll
-        for (int i = 0; i < K; ++i) { e[i] = expf(e[i] - mx); tot += e[i]; }
-        const float inv = 1.0f / tot;
+        for (int i = 0; i < K; ++i) { e[i] = __expf(e[i] - mx); tot += e[i]; }
+        const float inv = __fdividef(1.0f, tot);
 #pragma unroll
         for (int i = 0; i < K; ++i) hs.kappa[i] = e[i] * inv;
     }
@@ -837,7 +841,7 @@ __device__ __forceinline__ void pass_body(const PassArgs& a_in) {
             const ParamsDev& p = a.prm;
             const float eps = p.eps;
             const StateIn& S = ps.S;
-            const float d_z = sqrtf(S.cur_sumsq_anchor / N) / (sqrtf(S.anchor_sumsq / N) + eps);
+            const float d_z = __fdividef(sqrtf(__fdividef(S.cur_sumsq_anchor, N)), sqrtf(__fdividef(S.anchor_sumsq, N)) + eps);
             const float d_age = (float)a.age;
             const float d_phase = fabsf(a.sk.q_next - S.q_a_out);
             float dc = 0.f, dd = 0.f, uc = 0.f, ud = 0.f;
@@ -922,10 +926,10 @@ __device__ __forceinline__ void pass_body(const PassArgs& a_in) {
         st->R = R;
         float d_cf = __int_as_float(0x7fc00000);    // NaN: no calibration this step
         if (a.zcf != nullptr && S.cand_k == a.k && S.cand_supported && S.cand_finite) {
-            d_cf = (fin[sc0 + 0] / N) / (fin[sc0 + 1] / N + eps);
+            d_cf = __fdividef(__fdividef(fin[sc0 + 0], N), __fdividef(fin[sc0 + 1], N) + eps);
             if (!(p.flags & WDC_ABL_NO_CALIB)) {
                 const float bd = p.beta_d;
-                const float v = bd * S.eta + (1.f - bd) * d_cf / (S.cand_p + eps);
+                const float v = bd * S.eta + (1.f - bd) * __fdividef(d_cf, S.cand_p + eps);
                 eta = fminf(fmaxf(v, p.eta_min), p.eta_max);
                 st->eta = eta;
             }
@@ -933,24 +937,24 @@ __device__ __forceinline__ void pass_body(const PassArgs& a_in) {
         st->out.d_cf = d_cf;
         st->out.R = R;
         st->out.eta = eta;
-        const float r = sqrtf(fin[sc0 + 4] / N) / (sqrtf(S.cur_sumsq / N) + eps);
+        const float r = __fdividef(sqrtf(__fdividef(fin[sc0 + 4], N)), sqrtf(__fdividef(S.cur_sumsq, N)) + eps);
         st->out.r = r;
         st->rec[a.ins_slot].r = r;
-        s_rms[0] = sqrtf(fin[sc0 + 2] / N);
-        s_rms[1] = sqrtf(fin[sc0 + 3] / N);
+        s_rms[0] = sqrtf(__fdividef(fin[sc0 + 2], N));
+        s_rms[1] = sqrtf(__fdividef(fin[sc0 + 3], N));
     }
     __syncthreads();
     DevRecord& rec = st->rec[a.ins_slot];
-    const float sc = sqrtf((float)kSketch / N);
+    const float sc = sqrtf(__fdividef((float)kSketch, N));
     const float eps_nu = a.prm.eps_nu;
     const bool no_cond = a.prm.flags & WDC_ABL_NO_COND;
     float so = 0.f, si = 0.f;
     if (t < kSummary) {
         if (t < kSketch) {
-            so = sc * fin[t] / (s_rms[0] + eps_nu);
+            so = __fdividef(sc * fin[t], s_rms[0] + eps_nu);
         } else if (t < 2 * kSketch) {
             const int b = t - kSketch;
-            so = sc * (fin[b] - ps.S.anchor_S[b]) / (s_rms[1] + eps_nu);
+            so = __fdividef(sc * (fin[b] - ps.S.anchor_S[b]), s_rms[1] + eps_nu);
         } else if (t < kOffDepth) {
             so = no_cond ? 0.f : a.cam[t - kOffCam];
         } else if (t < kOffQ) {
