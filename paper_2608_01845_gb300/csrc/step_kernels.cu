@@ -214,25 +214,38 @@ __device__ __noinline__ void linear_readout(const PassArgs& a, const RecSummarie
     }
 }
 
-// Skip-pass head, Eq. 2-5 scalar part, in fp32 (every CTA computes it, so no
-// CTA has to wait for another).  The head and the controller tails are one
-// chain of dependent scalar steps per launch, so they use the fast division
-// and exponential intrinsics (a few ulp; the tolerances are 1e-5).
+// Skip-pass head, Eq. 2-5 scalar part, in fp32, run by one warp of every CTA
+// (so no CTA waits for another): lane l owns the summary entries l, l+32, ...,
+// every dot product is a lane-local sum followed by a butterfly, and every
+// lane then holds the totals, so each lane evaluates the small softmaxes of
+// Eq. 3 and 5 itself and no block barrier is needed.  (Spread over 256
+// threads with block reductions, the same head took ~9k cycles, most of it in
+// barriers.)  The head and the controller tails are one chain of dependent
+// scalar steps per launch, so they use the fast division and exponential
+// intrinsics (a few ulp; the tolerances are 1e-5).  Writes hs.phi, hs.hat,
+// hs.alpha and, for K > 0, hs.sim_in/sim_out/compat/pi/kappa/n_compat/
+// supported; the caller synchronises the block afterwards.
 template <int K>
-__device__ void skip_head(const PassArgs& a, const StateIn& S, const RecSummaries& rs, HeadShared& hs) {
-    const int t = threadIdx.x;
+__device__ void skip_head_warp(const PassArgs& a, const StateIn& S, const RecSummaries& rs, HeadShared& hs) {
+    constexpr int J = kSummary / 32;                  // entries per lane
+    const int lane = threadIdx.x & 31;
     const float N = (float)a.n;
     const float sc = sqrtf(__fdividef((float)kSketch, N));
     const float eps_nu = a.prm.eps_nu;
     const bool no_cond = a.prm.flags & WDC_ABL_NO_COND;
+    const float inv_cur = __fdividef(sc, sqrtf(__fdividef(S.cur_sumsq, N)) + eps_nu);
+    const float inv_dz = __fdividef(sc, sqrtf(__fdividef(S.cur_sumsq_anchor, N)) + eps_nu);
     // s(phi_k): current-state summary (Eq. 2 through the linear sketch)
-    if (t < kSummary) {
+    float ph[J];
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+        const int t = lane + 32 * j;
         float val;
         if (t < kSketch) {
-            val = __fdividef(sc * S.cur_S[t], sqrtf(__fdividef(S.cur_sumsq, N)) + eps_nu);
+            val = S.cur_S[t] * inv_cur;
         } else if (t < 2 * kSketch) {
             const int b = t - kSketch;
-            val = __fdividef(sc * (S.cur_S[b] - S.anchor_S[b]), sqrtf(__fdividef(S.cur_sumsq_anchor, N)) + eps_nu);
+            val = (S.cur_S[b] - S.anchor_S[b]) * inv_dz;
         } else if (t < kOffDepth) {
             val = no_cond ? 0.f : a.cam[t - kOffCam];
         } else if (t < kOffQ) {
@@ -241,104 +254,106 @@ __device__ void skip_head(const PassArgs& a, const StateIn& S, const RecSummarie
             val = a.sk.q_k;
         } else {
             // h(H): [r_1..3, T*(q_in - q_out)_1..3, n_bank/K], newest record first
-            const int j = t - kOffH;
+            const int h = t - kOffH;
             val = 0.f;
-            if (j < 3) {
-                if (j < a.nsrc) val = S.r[a.nsrc - 1 - j];
-            } else if (j < 6) {
-                if (j - 3 < a.nsrc) val = -(float)a.T * S.dq[a.nsrc - 1 - (j - 3)];
+            if (h < 3) {
+                if (h < a.nsrc) val = S.r[a.nsrc - 1 - h];
+            } else if (h < 6) {
+                if (h - 3 < a.nsrc) val = -(float)a.T * S.dq[a.nsrc - 1 - (h - 3)];
             } else {
                 val = __fdividef((float)a.nsrc, (float)a.prm.K);
             }
         }
+        ph[j] = val;
         hs.phi[t] = val;
     }
-    if (t == 0) {
-        // Eq. 4: alpha = clip(|q_{t-1}-q_t| / (|q_{a-1}-q_a| + eps), alpha_min, alpha_max)
-        const float raw = __fdividef(fabsf(a.sk.dq), fabsf(S.q_a_dq) + a.prm.eps);
-        hs.alpha = fminf(fmaxf(raw, a.prm.alpha_min), a.prm.alpha_max);
-    }
-    __syncthreads();
-    if (K == 0) return;
-
-    // Eq. 3: similarities with the records' lifted inputs
-    {
-        float v[K + 1];
-        const float ph = (t < kSummary) ? hs.phi[t] : 0.f;
+    // Eq. 4: alpha = clip(|q_{t-1}-q_t| / (|q_{a-1}-q_a| + eps), alpha_min, alpha_max)
+    const float alpha =
+        fminf(fmaxf(__fdividef(fabsf(a.sk.dq), fabsf(S.q_a_dq) + a.prm.eps), a.prm.alpha_min), a.prm.alpha_max);
+    if (lane == 0) hs.alpha = alpha;
+    if constexpr (K > 0) {
+        // Eq. 3: similarities with the records' lifted inputs
+        float d[K + 1];
 #pragma unroll
-        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? ph * rs.s_in[i][t] : 0.f;
-        v[K] = ph * ph;
-        reduce256<K + 1>(v, hs.scratch, hs.red);
-    }
-    if (t == 0) {
-        const float nphi = sqrtf(hs.red[K]);
+        for (int i = 0; i <= K; ++i) d[i] = 0.f;
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            const int t = lane + 32 * j;
+#pragma unroll
+            for (int i = 0; i < K; ++i) d[i] = fmaf(ph[j], rs.s_in[i][t], d[i]);
+            d[K] = fmaf(ph[j], ph[j], d[K]);
+        }
+#pragma unroll
+        for (int i = 0; i <= K; ++i) d[i] = warp_sum_f(d[i]);
+        const float nphi = sqrtf(d[K]);
         const bool filter = !(a.prm.flags & WDC_ABL_NO_SUPPORT);   // w/o support: N_t = whole bank
         const float gq = a.prm.gamma_q, inv_tin = __fdividef(1.0f, a.prm.tau_in);
         int nc = 0;
-        float mx = -INFINITY;
-        float ell[K > 0 ? K : 1];
+        float mx = -INFINITY, ell[K], pi[K], sim[K];
+        bool compat[K];
 #pragma unroll
         for (int i = 0; i < K; ++i) {
-            const float s = (nphi == 0.f || S.n_in[i] == 0.f) ? 0.f : __fdividef(hs.red[i], nphi * S.n_in[i]);
+            sim[i] = (nphi == 0.f || S.n_in[i] == 0.f) ? 0.f : __fdividef(d[i], nphi * S.n_in[i]);
             const float dq = a.sk.q_k - S.q_in[i];
-            hs.sim_in[i] = s;
-            const int c = !filter || ((s >= a.prm.sim_min) && (fabsf(dq) <= a.prm.q_gap_max));
-            hs.compat[i] = c;
-            ell[i] = (s - gq * dq * dq) * inv_tin;
-            if (c) { ++nc; mx = fmaxf(mx, ell[i]); }
+            compat[i] = !filter || ((sim[i] >= a.prm.sim_min) && (fabsf(dq) <= a.prm.q_gap_max));
+            ell[i] = (sim[i] - gq * dq * dq) * inv_tin;
+            if (compat[i]) { ++nc; mx = fmaxf(mx, ell[i]); }
         }
         float tot = 0.f;
 #pragma unroll
         for (int i = 0; i < K; ++i) {
-            hs.pi[i] = hs.compat[i] ? __expf(ell[i] - mx) : 0.f;
-            tot += hs.pi[i];
+            pi[i] = compat[i] ? __expf(ell[i] - mx) : 0.f;
+            tot += pi[i];
         }
-#pragma unroll
         const float inv_tot = nc > 0 ? __fdividef(1.0f, tot) : 0.f;
 #pragma unroll
-        for (int i = 0; i < K; ++i) hs.pi[i] *= inv_tot;
-        hs.n_compat = nc;
-        hs.supported = filter ? (nc >= a.prm.min_support) : 1;
-    }
-    __syncthreads();
-    // Eq. 4 in summary space, then Eq. 5 similarities with the lifted outputs
-    {
-        float v[K + 1];
-        float hv = 0.f;
-        if (t < kSummary) {
+        for (int i = 0; i < K; ++i) pi[i] *= inv_tot;
+        // Eq. 4 in summary space, then Eq. 5 similarities with the lifted outputs
+        float e[K + 1];
+#pragma unroll
+        for (int i = 0; i <= K; ++i) e[i] = 0.f;
+#pragma unroll
+        for (int j = 0; j < J; ++j) {
+            const int t = lane + 32 * j;
             float acc = 0.f;
 #pragma unroll
             for (int i = 0; i < K; ++i)
-                if (hs.pi[i] != 0.f) acc = fmaf(hs.pi[i], rs.s_dphi[i][t], acc);
-            hv = fmaf(hs.alpha, acc, hs.phi[t]);
+                if (pi[i] != 0.f) acc = fmaf(pi[i], rs.s_dphi[i][t], acc);
+            const float hv = fmaf(alpha, acc, ph[j]);
             hs.hat[t] = hv;
+#pragma unroll
+            for (int i = 0; i < K; ++i) e[i] = fmaf(hv, rs.s_out[i][t], e[i]);
+            e[K] = fmaf(hv, hv, e[K]);
         }
 #pragma unroll
-        for (int i = 0; i < K; ++i) v[i] = (t < kSummary) ? hv * rs.s_out[i][t] : 0.f;
-        v[K] = hv * hv;
-        reduce256<K + 1>(v, hs.scratch, hs.red);
-    }
-    if (t == 0) {
-        const float nh = sqrtf(hs.red[K]);
+        for (int i = 0; i <= K; ++i) e[i] = warp_sum_f(e[i]);
+        const float nh = sqrtf(e[K]);
         const float inv_tau = __fdividef(1.0f, a.prm.tau_obs);
-        float mx = -INFINITY;
-        float e[K > 0 ? K : 1];
+        float so[K];
+        float mo = -INFINITY;
 #pragma unroll
         for (int i = 0; i < K; ++i) {
-            const float s = (nh == 0.f || S.n_out[i] == 0.f) ? 0.f : __fdividef(hs.red[i], nh * S.n_out[i]);
-            hs.sim_out[i] = s;
-            e[i] = s * inv_tau;
-            mx = fmaxf(mx, e[i]);
+            so[i] = (nh == 0.f || S.n_out[i] == 0.f) ? 0.f : __fdividef(e[i], nh * S.n_out[i]);
+            e[i] = so[i] * inv_tau;
+            mo = fmaxf(mo, e[i]);
         }
-        float tot = 0.f;
+        float to = 0.f;
 #pragma unroll
-        for (int i = 0; i < K; ++i) { e[i] = __expf(e[i] - mx); tot += e[i]; }
-        const float inv = __fdividef(1.0f, tot);
+        for (int i = 0; i < K; ++i) { e[i] = __expf(e[i] - mo); to += e[i]; }
+        const float inv = __fdividef(1.0f, to);
+        if (lane == 0) {
 #pragma unroll
-        for (int i = 0; i < K; ++i) hs.kappa[i] = e[i] * inv;
+            for (int i = 0; i < K; ++i) {
+                hs.sim_in[i] = sim[i];
+                hs.compat[i] = compat[i];
+                hs.pi[i] = pi[i];
+                hs.sim_out[i] = so[i];
+                hs.kappa[i] = e[i] * inv;
+            }
+            hs.n_compat = nc;
+            hs.supported = filter ? (nc >= a.prm.min_support) : 1;
+        }
     }
-    __syncthreads();
-    if (a.prm.flags & WDC_ABL_LINEAR_OBS) linear_readout<K>(a, rs, hs);
 }
 
 // Per-block scalar slots: the stream's five sums and the non-finite count.
@@ -462,12 +477,15 @@ __device__ __forceinline__ void pass_body(const PassArgs& a_in) {
     float kap[K > 0 ? K : 1];
     float alpha_f = 0.f;
     if (MODE == kModeSkip || MODE == kModeResidual) {
-        skip_head<K>(a, ps.S, ps.rs, hs);          // ends with a block barrier
+        if (warp == 0) skip_head_warp<K>(a, ps.S, ps.rs, hs);
+        __syncthreads();
+        if (a.prm.flags & WDC_ABL_LINEAR_OBS) linear_readout<K>(a, ps.rs, hs);
         do_stream = (K > 0) && hs.supported;
 #pragma unroll
         for (int i = 0; i < K; ++i) kap[i] = hs.kappa[i];
     } else if (MODE == kModeSecant) {
-        skip_head<0>(a, ps.S, ps.rs, hs);          // lift summary and alpha only: no retrieval
+        if (warp == 0) skip_head_warp<0>(a, ps.S, ps.rs, hs);   // lift summary and alpha only: no retrieval
+        __syncthreads();
         do_stream = a.nsrc > 0;
         alpha_f = hs.alpha;
     } else if (MODE == kModeObserve) {
