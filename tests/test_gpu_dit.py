@@ -308,3 +308,35 @@ def test_profiler_times_every_launch_and_dual_stream_gemms_are_grouped():
     assert prof["norm"][1] == 5                    # 2 row ranges x 2 LayerNorms + the final one
     assert ctx.launches - n0 == sum(n for _, n in prof.values())
     assert all(ms > 0 for ms, n in prof.values() if n)
+
+
+@pytest.mark.parametrize("dual", [0, 1])
+def test_bf16_block_hidden_3072_few_ragged_rows(dual):
+    """The D = 3072 kernels on a short ragged sequence: 5 condition + 272
+    video tokens (277 rows: not a multiple of the LayerNorm's 8 rows per
+    block nor of the attention's 128-row tiles; 272 video rows leave a
+    16-row tail in the second 256-row GEMM tile pair; with dual-stream
+    weights each GEMM is one grouped launch whose second problem has 5
+    rows), the whole block against the fp64 oracle on every row."""
+    cfgd = dict(layers=1, hidden=3072, heads=48, head_dim=64, mlp=12288, temb_dim=512, freq_dim=256, in_ch=16,
+                frames=1, height=32, width=34, patch=2, cond_tokens=5, cond_dim=3072, dual_stream=dual)
+    cfg = DiTConfig(**cfgd)
+    ctx = _ctx(cfgd, wdc.BF16)
+    S = 2 if dual else 1
+    names = [f"L0.s{s}.{n}" for s in range(S) for n in ["qkv.w", "qkv.b", "o.w", "o.b", "fc1.w", "fc1.b", "fc2.w",
+                                                         "fc2.b"]]
+    W = synth.dit_weights(cfgd, 9, std=0.02, bias_std=0.02, bf16=True, names=names)
+    ctx.set_weights(W)
+    L, D = 277, 3072
+    x = _bf(synth.normal(41, (L, D)))
+    mods = [synth.normal(42 + s, (6, D), 0.3) for s in range(S)]
+    for m in mods:
+        m[2] += 1.0
+        m[5] += 1.0
+    xt = _to_dev(x, torch.bfloat16)
+    ctx.dit_block_forward(0, xt, _to_dev(np.concatenate(mods, axis=0)))
+    torch.cuda.synchronize()
+    want = dit.block(x.astype(np.float64), W, cfg, 0, [m.astype(np.float64) for m in mods])
+    got = xt.float().cpu().numpy()
+    assert rel_l2(got - x, want - x) <= BF16_TOL
+    assert ctx.device_errors() == 0
