@@ -237,7 +237,10 @@ size_t wdc_latent_numel(const wdc_ctx* ctx);
 unsigned long long wdc_launch_count(const wdc_ctx* ctx);
 /* Synchronises the device and returns (then clears) the bits the kernels have
  * set in the context's error word: 1 = a bounded device-side wait timed out,
- * 4 = the two CTAs of a tensor-core pair saw different tensor-memory bases. */
+ * 4 = the two CTAs of a tensor-core pair saw different tensor-memory bases,
+ * 8 = a bf16 model's QKV projection produced a value of V beyond fp16's range
+ * (|v| > 65504), which was saturated to +-65504 when V^T was stored for the
+ * attention (NaN is kept). */
 wdc_status wdc_device_errors(wdc_ctx* ctx, unsigned* bits);
 /* Self-test of the bounded device-side waits (the paper has no counterpart):
  * one CTA waits on an mbarrier that nothing completes, through the same

@@ -812,6 +812,7 @@ static wdc_status run_block(Ctx* c, int layer, void* x, const float* mod, int nb
             e[sidx].q = t->q; e[sidx].k = t->k; e[sidx].vt = t->vt;
             e[sidx].L = t->L; e[sidx].H = t->H; e[sidx].d = t->d; e[sidx].D = D; e[sidx].row_off = r0[sidx];
             e[sidx].nb = nb; e[sidx].Lc = t->Lc; e[sidx].ldv = t->ldv;
+            e[sidx].err = c->err;
         }
         if ((st = lin_gemm(t->qkv, t->h, D, 3 * D, e))) return st;
     }

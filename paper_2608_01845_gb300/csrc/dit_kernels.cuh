@@ -14,10 +14,14 @@ template <> __device__ __forceinline__ float ld_act<float>(const float* p) { ret
 template <> __device__ __forceinline__ float ld_act<__nv_bfloat16>(const __nv_bfloat16* p) { return __bfloat162float(*p); }
 template <> __device__ __forceinline__ float ld_act<__half>(const __half* p) { return __half2float(*p); }
 
-// V^T of the bf16 model is stored in fp16 (10-bit mantissa, range +-65504,
-// saturated) so that the attention's PV product can take P in fp16.
-__device__ __forceinline__ __half to_vt_half(float v) {
-    return __float2half_rn(fminf(fmaxf(v, -65504.0f), 65504.0f));
+// V^T of the bf16 model is stored in fp16 (10-bit mantissa) so that the
+// attention's PV product can take P in fp16.  A value beyond fp16's range
+// (|v| > 65504, infinities included) is saturated to +-65504 and `sat` is
+// set, so that the caller can report it; NaN stays NaN.
+__device__ __forceinline__ __half to_vt_half(float v, bool& sat) {
+    const bool big = fabsf(v) > 65504.0f;
+    sat |= big;
+    return __float2half_rn(big ? copysignf(65504.0f, v) : v);
 }
 
 template <typename T> __device__ __forceinline__ T to_act(float v);
@@ -76,6 +80,7 @@ struct Epi {
     // of sample b = b*H + h
     void* q; void* k; void* vt;
     int L, H, d, D, row_off, nb, Lc, ldv;
+    unsigned* err;            // kEpiQKV: receives kErrVSaturated (may be null)
     // kEpiUnpatch: v fp32 [nb][C, F, Hh, Ww]; row m = (sample, f, h', w'),
     // column = (c, ph, pw)
     float* v;
@@ -107,8 +112,11 @@ __device__ __forceinline__ void epi_apply(const Epi& e, int m, int n, float acc)
                 reinterpret_cast<T*>(e.q)[(h * e.L + tok) * e.d + dd] = to_act<T>(x);
             else if (which == 1)
                 reinterpret_cast<T*>(e.k)[(h * e.L + tok) * e.d + dd] = to_act<T>(x);
-            else if constexpr (sizeof(T) == 2)
-                reinterpret_cast<__half*>(e.vt)[(h * e.d + dd) * e.ldv + tok] = to_vt_half(x);
+            else if constexpr (sizeof(T) == 2) {
+                bool sat = false;
+                reinterpret_cast<__half*>(e.vt)[(h * e.d + dd) * e.ldv + tok] = to_vt_half(x, sat);
+                if (sat && e.err) atomicOr(e.err, kErrVSaturated);
+            }
             else
                 reinterpret_cast<T*>(e.vt)[(h * e.d + dd) * e.ldv + tok] = to_act<T>(x);
             break;

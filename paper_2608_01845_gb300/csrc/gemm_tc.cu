@@ -145,8 +145,10 @@ __device__ __forceinline__ void epilogue_chunk(const Epi& e, int m, int col0, co
             }
         } else {
             __half* base = reinterpret_cast<__half*>(e.vt) + (h * e.d + dd0) * e.ldv + tok;
+            bool sat = false;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) base[(size_t)j * e.ldv] = to_vt_half(v[j]);
+            for (int j = 0; j < 32; ++j) base[(size_t)j * e.ldv] = to_vt_half(v[j], sat);
+            if (sat && e.err) atomicOr(e.err, kErrVSaturated);
         }
         return;
     }

@@ -23,7 +23,7 @@ constexpr int kOffQ = kOffDepth + 4;
 constexpr int kOffH = kOffQ + 1;
 
 // Error bits written by kernels into the context's device error word.
-enum : unsigned { kErrTimeout = 1u, kErrBounds = 2u, kErrTmem = 4u };
+enum : unsigned { kErrTimeout = 1u, kErrBounds = 2u, kErrTmem = 4u, kErrVSaturated = 8u };
 
 // ---------------------------------------------------------------- device state
 // Device state is fp32 throughout.  On GB300 an fp64 operation has a

@@ -247,7 +247,8 @@ class Context:
         self.params = params
 
     def device_errors(self):
-        """Error bits set by kernels since the last call (1 timeout, 4 TMEM pair mismatch)."""
+        """Error bits set by kernels since the last call (1 timeout, 4 TMEM pair
+        mismatch, 8 a bf16 model's V saturated to fp16's range)."""
         b = ctypes.c_uint()
         self._check(LIB.wdc_device_errors(self._h, ctypes.byref(b)), "device_errors")
         return b.value

@@ -340,3 +340,35 @@ def test_bf16_block_hidden_3072_few_ragged_rows(dual):
     got = xt.float().cpu().numpy()
     assert rel_l2(got - x, want - x) <= BF16_TOL
     assert ctx.device_errors() == 0
+
+
+def test_bf16_v_beyond_fp16_range_is_saturated_and_reported():
+    """V^T of a bf16 model is stored in fp16: a V value beyond +-65504 is
+    saturated and reported through bit 8 of the device error word; the same
+    block with ordinary weights reports nothing, and NaN input propagates
+    (it is not turned into a finite value)."""
+    cfgd = dict(PARITY_MODEL, layers=1)
+    names = [f"L0.s0.{n}" for n in ["qkv.w", "qkv.b", "o.w", "o.b", "fc1.w", "fc1.b", "fc2.w", "fc2.b"]]
+    W = synth.dit_weights(cfgd, 13, std=0.02, bf16=True, names=names)
+    L, D = 16 + 4 * 8 * 8, 256
+    x = _bf(synth.normal(51, (L, D)))
+    mod = _to_dev(synth.normal(52, (6, D), 0.3))
+    ctx = _ctx(cfgd, wdc.BF16)
+    ctx.set_weights(W)
+    ctx.dit_block_forward(0, _to_dev(x, torch.bfloat16), mod)
+    assert ctx.device_errors() == 0
+    big = dict(W)
+    big["L0.s0.qkv.w"] = W["L0.s0.qkv.w"].copy()
+    big["L0.s0.qkv.w"][2 * D:] *= 2.0 ** 24       # |V| ~ 1e6 > 65504
+    ctx.set_weights(big)
+    xt = _to_dev(x, torch.bfloat16)
+    ctx.dit_block_forward(0, xt, mod)
+    assert ctx.device_errors() == 8
+    assert torch.isfinite(xt.float()).all()
+    ctx.set_weights(W)
+    xn = x.copy()
+    xn[3, 5] = np.nan
+    xt = _to_dev(xn, torch.bfloat16)
+    ctx.dit_block_forward(0, xt, mod)
+    assert ctx.device_errors() == 0
+    assert torch.isnan(xt.float()).any()
