@@ -5,14 +5,13 @@
 // d = 64 or 128.
 //
 // One CTA per (head, 256 query rows), 12 warps in three warpgroups:
-//   warpgroup 0 (control, registers lowered to 40 / 72 per thread)
-//     warp 0    TMA producer: the two 128-row Q tiles once, then K / V^T tiles
-//               of 128 keys into a shared-memory ring (128-byte swizzle);
-//     warp 1(,2) MMA issuer(s): one thread per query tile (d = 64) or one
-//               thread for both (d = 128):
-//               S(t) = Q(t) K^T into TMEM (128 fp32 columns per tile) and
+//   warpgroup 0 (control, registers lowered to 40 per thread)
+//     warp 0    TMA producer: the two 128-row Q tiles once, then K / V^T
+//               tiles of BK keys into a shared-memory ring (128-byte swizzle);
+//     warps 1, 2 MMA issuers, one thread per query tile t:
+//               S(t) = Q(t) K^T into TMEM (BK fp32 columns) and
 //               O(t) += P(t) V into TMEM;
-//   warpgroups 1, 2 (softmax of query tile 0, 1; registers raised to 232 / 216)
+//   warpgroups 1, 2 (softmax of query tile 0, 1; registers raised to 232)
 //               one thread per query row = TMEM lane: exp2 numerators, row
 //               sums, O rescaling in TMEM when the exponent base moves, final
 //               1/l normalisation and the bf16 store.
@@ -30,17 +29,14 @@
 // the P word; row sums accumulate per 16 pairs in f16x2 and in fp32 beyond.
 // In fp16, x keeps 11 significant bits (error <= 2^-9 absolute for
 // |x| < 8, below the rounding of P itself where P matters) and P keeps 11
-// (bf16 would keep 8).  Two TMEM layouts:
-//   d = 64   per tile t: S (128 columns), P (64), O (64) = 256 columns, so P
-//            has its own columns: S(t) may be overwritten as soon as the
-//            softmax has loaded it, and the MMA of S(t, j+1) overlaps the
-//            softmax of tile j:
-//               S(t, j), PV(t, j-1)   (per issuer)
-//   d = 128  S (2 x 128) + O (2 x 128) fill TMEM, so P is written back over
-//            the first 64 columns of S(t); S(t, j+1) then follows PV(t, j):
-//               PV0(j-1), S0(j), PV1(j-1), S1(j)
-//            and the commit after S(t, j) also covers PV(t, j-1) (tcgen05 ops
-//            of one thread complete in order).
+// (bf16 would keep 8).
+// TMEM, per query tile t: S (BK columns), P (BK / 2) and O (d) side by side
+// -- d = 64 with BK = 128 keys per step, d = 128 with BK = 64, 256 and 224
+// columns a tile.  P has its own columns, so S(t) may be overwritten as soon
+// as the softmax has loaded it: each issuer runs
+//     S(t, j), PV(t, j-1)
+// and the MMA of S(t, j+1) overlaps the softmax of step j instead of
+// waiting behind PV(t, j).
 // Keys past L are masked (TMA zero-fills out-of-range K / V^T).  Every
 // mbarrier wait is bounded.
 #include "dit_kernels.cuh"
@@ -53,33 +49,33 @@ namespace wdc {
 namespace {
 
 constexpr int BQ = 128;        // query rows per tile (two tiles per CTA)
-constexpr int BKV = 128;       // keys per tile
 // Register split: launch allocation 168 per thread (65536 / 384 rounded
 // down to a multiple of 8); the control warpgroup hands registers to the two
-// softmax warpgroups (d = 64: 128 * 40 + 256 * 232 = 384 * 168; the single
-// d = 128 issuer, which drives both tiles, keeps 72: 128 * 72 + 256 * 216).
+// softmax warpgroups: 128 * 40 + 256 * 232 = 384 * 168.
 constexpr uint32_t kRegsLaunch = 168;
 
 template <int D>
 struct AttnCfg {
-    static constexpr bool P_SEP = D == 64;                  // P in its own TMEM columns, one issuer per tile
+    static constexpr int BK = D == 64 ? 128 : 64;           // keys per step
     static constexpr int THREADS = 384;                     // 3 warpgroups
-    static constexpr int ISSUERS = P_SEP ? 2 : 1;
+    static constexpr int ISSUERS = 2;                       // one MMA thread per query tile
     static constexpr int ATOMS = D / 64;                    // 128-byte atoms along d
     static constexpr uint32_t Q_TILE = BQ * D * 2;          // one query tile
-    static constexpr uint32_t K_TILE = BKV * D * 2;
-    static constexpr uint32_t V_TILE = D * BKV * 2;
-    static constexpr uint32_t STAGE = K_TILE + V_TILE;
-    static constexpr int STAGES = D == 64 ? 3 : 2;
+    static constexpr uint32_t K_TILE = BK * D * 2;
+    static constexpr uint32_t V_TILE = D * BK * 2;
+    static constexpr uint32_t STAGE = K_TILE + V_TILE;      // 32 KB for both head sizes
+    static constexpr int STAGES = D == 64 ? 3 : 5;
     static constexpr uint32_t SMEM = 2 * Q_TILE + STAGES * STAGE + 1024 + 256;
     static constexpr uint32_t TMEM_COLS = 512;
-    static constexpr uint32_t REGS_CONTROL = P_SEP ? 40 : 72;
-    static constexpr uint32_t REGS_SOFTMAX = P_SEP ? 232 : 216;
+    static constexpr uint32_t REGS_CONTROL = 40;
+    static constexpr uint32_t REGS_SOFTMAX = 232;
     static_assert(128 * REGS_CONTROL + 256 * REGS_SOFTMAX <= 384 * kRegsLaunch, "register split exceeds the launch");
+    static_assert(2 * (BK + BK / 2 + D) <= (int)TMEM_COLS, "S, P and O of two tiles exceed tensor memory");
+    static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
     // TMEM column of S, P and O of query tile t
-    __device__ static constexpr uint32_t s_col(int t) { return P_SEP ? 256u * t : 128u * t; }
-    __device__ static constexpr uint32_t p_col(int t) { return P_SEP ? 256u * t + 128u : 128u * t; }
-    __device__ static constexpr uint32_t o_col(int t) { return P_SEP ? 256u * t + 192u : 256u + (uint32_t)D * t; }
+    __device__ static constexpr uint32_t s_col(int t) { return (uint32_t)(BK + BK / 2 + D) * t; }
+    __device__ static constexpr uint32_t p_col(int t) { return s_col(t) + BK; }
+    __device__ static constexpr uint32_t o_col(int t) { return s_col(t) + BK + BK / 2; }
 };
 
 
@@ -146,6 +142,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
                    const __grid_constant__ CUtensorMap tv, const __grid_constant__ AttnArgs g) {
     using C = AttnCfg<D>;
+    constexpr int BKV = C::BK;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sq = smem;                                       // [2 tiles][ATOMS][128 x 128 B]
@@ -155,9 +152,9 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     uint64_t* kv_full = q_full + 1;
     uint64_t* kv_empty = kv_full + C::STAGES;
     uint64_t* s_full = kv_empty + C::STAGES;                  // [2]
-    uint64_t* s_free = s_full + 2;                            // [2] (separate P)
+    uint64_t* s_free = s_full + 2;                            // [2]
     uint64_t* p_full = s_free + 2;                            // [2]
-    uint64_t* p_free = p_full + 2;                            // [2] (separate P)
+    uint64_t* p_free = p_full + 2;                            // [2]
     uint64_t* o_final = p_free + 2;                           // [2]
     uint64_t* mma_done = o_final + 2;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
@@ -236,7 +233,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                 }
             }
         }
-      } else if (warp == 1 || (C::P_SEP && warp == 2)) {
+      } else if (warp == 1 || warp == 2) {
         if (lane == 0) {
             constexpr uint32_t idesc_s = idesc_bf16(BQ, BKV);
             constexpr uint32_t idesc_o = idesc_f16(BQ, D);       // P (fp16, TMEM) x V (fp16, shared memory)
@@ -244,7 +241,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
             bool ok = mbar_wait(q_full, 0, abort_flag, g.err);
             int stage = 0, prev = 0;
             uint32_t phase = 0;
-            // S(t) = Q(t) K^T into TMEM (128 fp32 columns)
+            // S(t) = Q(t) K^T into TMEM (BK fp32 columns)
             auto issue_s = [&](int t, int st) {
                 const uint32_t kb = smem_u32(skv + st * C::STAGE);
                 const uint32_t qb = sq0 + t * C::Q_TILE;
@@ -265,63 +262,34 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                               (acc || ks != 0) ? 1u : 0u);
                 }
             };
-            if constexpr (C::P_SEP) {
-                // this thread issues the MMAs of query tile t only; the other
-                // tile has its own issuer, so neither waits behind the other's
-                // softmax
-                const int t = warp - 1;
-                for (int j = 0; j < n_kv && ok; ++j) {
-                    if (!mbar_wait(&kv_full[stage], phase, abort_flag, g.err)) { ok = false; break; }
+            // this thread issues the MMAs of query tile t only; the other
+            // tile has its own issuer, so neither waits behind the other's
+            // softmax
+            const int t = warp - 1;
+            for (int j = 0; j < n_kv && ok; ++j) {
+                if (!mbar_wait(&kv_full[stage], phase, abort_flag, g.err)) { ok = false; break; }
+                tc_fence_after();
+                if (j > 0) {
+                    if (!mbar_wait(&s_free[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
                     tc_fence_after();
-                    if (j > 0) {
-                        if (!mbar_wait(&s_free[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
-                        tc_fence_after();
-                    }
-                    issue_s(t, stage);
-                    tc_commit(&s_full[t]);
-                    if (j > 0) {
-                        if (!mbar_wait(&p_full[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
-                        tc_fence_after();
-                        issue_pv(t, prev, j > 1);
-                        tc_commit(&p_free[t]);
-                        tc_commit(&kv_empty[prev]);
-                    }
-                    prev = stage;
-                    if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
                 }
-                if (ok && mbar_wait(&p_full[t], (n_kv - 1) & 1, abort_flag, g.err)) {
+                issue_s(t, stage);
+                tc_commit(&s_full[t]);
+                if (j > 0) {
+                    if (!mbar_wait(&p_full[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
                     tc_fence_after();
-                    issue_pv(t, prev, n_kv > 1);
+                    issue_pv(t, prev, j > 1);
+                    tc_commit(&p_free[t]);
                     tc_commit(&kv_empty[prev]);
-                    tc_commit(&o_final[t]);
                 }
-            } else {
-                // one issuer interleaving both tiles: PV0(j-1), S0(j), PV1(j-1), S1(j)
-                for (int j = 0; j < n_kv && ok; ++j) {
-                    if (!mbar_wait(&kv_full[stage], phase, abort_flag, g.err)) { ok = false; break; }
-                    tc_fence_after();
-                    for (int t = 0; t < 2; ++t) {
-                        if (j > 0) {
-                            if (!mbar_wait(&p_full[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
-                            tc_fence_after();
-                            issue_pv(t, prev, j > 1);
-                            if (t == 1) tc_commit(&kv_empty[prev]);
-                        }
-                        issue_s(t, stage);
-                        tc_commit(&s_full[t]);
-                    }
-                    prev = stage;
-                    if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
-                }
-                if (ok) {
-                    for (int t = 0; t < 2; ++t) {
-                        if (!mbar_wait(&p_full[t], (n_kv - 1) & 1, abort_flag, g.err)) break;
-                        tc_fence_after();
-                        issue_pv(t, prev, n_kv > 1);
-                        if (t == 1) tc_commit(&kv_empty[prev]);
-                        tc_commit(&o_final[t]);
-                    }
-                }
+                prev = stage;
+                if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
+            }
+            if (ok && mbar_wait(&p_full[t], (n_kv - 1) & 1, abort_flag, g.err)) {
+                tc_fence_after();
+                issue_pv(t, prev, n_kv > 1);
+                tc_commit(&kv_empty[prev]);
+                tc_commit(&o_final[t]);
             }
             tc_commit(mma_done);
             const unsigned long long t0 = globaltimer();
@@ -350,12 +318,10 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
 #pragma unroll
             for (int c = 0; c < BKV / 32; ++c) tmem_ld32(s_addr + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&s[c * 32]));
             tmem_ld_wait();
-            if constexpr (C::P_SEP) {
-                // S(t) is in registers: the MMA may compute S(t, j+1) now
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&s_free[t]);
-            }
+            // S(t) is in registers: the MMA may compute S(t, j+1) now
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s_free[t]);
             if (j == n_kv - 1 && last_valid < BKV) {
 #pragma unroll
                 for (int c = 0; c < BKV; ++c)
@@ -372,7 +338,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                     for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], s[c + i], s[c + 8 + i]);
                 return fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
             };
-            // numerators 2^(s * scale - base) into p (bf16 pairs); returns their sum
+            // numerators 2^(s * scale - base) into p (fp16 pairs); returns their sum
             uint32_t p[BKV / 2];
             auto numerators = [&](float base) {
                 uint32_t sum4[4];
@@ -387,40 +353,25 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
             float sum;
             // A numerator above 2^8 implies a row sum above 2^8 (so does a
             // non-finite one): only then take the tile max, move the base and
-            // recompute.  d = 64 runs the recompute as a second pass of the
-            // same code; d = 128 (higher register pressure around its single
-            // issuer's schedule) measured faster with a separate copy.
-            if constexpr (C::P_SEP) {
+            // recompute, as a second pass of the same code.
 #pragma unroll 1
-                for (int pass = 0;; ++pass) {
-                    sum = numerators(base);
-                    const bool redo = pass == 0 && !(sum <= 256.0f);
-                    if (!__any_sync(0xffffffffu, redo)) break;
-                    if (redo) base = fmaxf(base, tile_max() * g.scale_log2);
-                }
-            } else {
+            for (int pass = 0;; ++pass) {
                 sum = numerators(base);
-                const bool redo = !(sum <= 256.0f);
-                if (__any_sync(0xffffffffu, redo)) {
-                    if (redo) {
-                        base = fmaxf(base, tile_max() * g.scale_log2);
-                        sum = numerators(base);
-                    }
-                }
+                const bool redo = pass == 0 && !(sum <= 256.0f);
+                if (!__any_sync(0xffffffffu, redo)) break;
+                if (redo) base = fmaxf(base, tile_max() * g.scale_log2);
             }
             const bool moved = base != m_run;
             const float corr = ex2(m_run - base);     // 1 when the base stays; 0 before the first tile
             l_run = l_run * corr + sum;
             m_run = base;
-            if constexpr (C::P_SEP) {
-                // PV(t, j-1) must be done before P(t) is overwritten and O(t) rescaled
-                if (j > 0) {
-                    if (!mbar_wait(&p_free[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
-                    tc_fence_after();
-                }
+            // PV(t, j-1) must be done before P(t) is overwritten and O(t) rescaled
+            if (j > 0) {
+                if (!mbar_wait(&p_free[t], (j - 1) & 1, abort_flag, g.err)) { ok = false; break; }
+                tc_fence_after();
             }
             if (j > 0 && __any_sync(0xffffffffu, moved)) {
-                // PV(t, j-1) is complete (p_free, or the commit after S(t, j)): rescale O in place
+                // PV(t, j-1) is complete: rescale O in place
 #pragma unroll
                 for (int c = 0; c < D; c += 32) {
                     uint32_t o[32];
@@ -436,7 +387,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                     tmem_st16(o_addr + c + 16, hi);
                 }
             }
-            // P (64 columns of bf16 pairs)
+            // P (BK / 2 columns of fp16 pairs)
 #pragma unroll
             for (int c = 0; c < BKV / 2; c += 16) tmem_st16(p_addr + c, *reinterpret_cast<uint32_t(*)[16]>(&p[c]));
             tmem_st_wait();
@@ -489,6 +440,7 @@ template <int D, bool BATCH>
 wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, int ldv, void* o, int H, int L, int Hs,
                   int Lc, cudaStream_t s) {
     using Cf = AttnCfg<D>;
+    constexpr int BKV = Cf::BK;
     static bool attr = false;
     static bool regs_ok = false;
     if (!attr) {
