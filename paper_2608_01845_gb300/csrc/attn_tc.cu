@@ -85,6 +85,14 @@ struct AttnArgs {
     float scale_log2;
     __nv_bfloat16* o;
     unsigned* err;
+    // per sample: units_s = Hs * q_blocks units (head, 256-query block);
+    // those from n_full on are split over the key range into `split` CTAs
+    // each, which write unnormalised partials.  The split depends on the
+    // sample's own grid only, so a sample's attention is the same bits in a
+    // batched launch as alone.
+    int units_s, n_full, split;
+    float* part_o;            // [part slot][256 rows][d]
+    float* part_ml;           // [part slot][256 rows][base, row sum]
 };
 
 __device__ __forceinline__ float ex2(float x) {
@@ -161,9 +169,22 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int h = blockIdx.x / g.q_blocks;
-    const int q0 = (blockIdx.x % g.q_blocks) * (2 * BQ);
+    // unit (head, 256-query block) of this CTA: per sample, n_full whole
+    // units, then the key-range parts of the sample's last units (keys of
+    // steps j0 .. j0 + nj - 1)
+    const int n_split_s = g.units_s - g.n_full;
+    const int per_sample = g.n_full + n_split_s * g.split;
+    const int smp = blockIdx.x / per_sample, rem = blockIdx.x - smp * per_sample;
+    const bool is_part = rem >= g.n_full;
+    const int pidx = rem - g.n_full;                          // part CTA within the sample
+    const int unit = smp * g.units_s + (is_part ? g.n_full + pidx / g.split : rem);
+    const int part = is_part ? pidx % g.split : 0;
+    const int pslot = smp * n_split_s * g.split + pidx;       // workspace slot of a part CTA
+    const int h = unit / g.q_blocks;
+    const int q0 = (unit % g.q_blocks) * (2 * BQ);
     const int n_kv = g.n_kv;
+    const int j0 = is_part ? part * n_kv / g.split : 0;
+    const int nj = (is_part ? (part + 1) * n_kv / g.split : n_kv) - j0;
 
     if (threadIdx.x == 0) {
         mbar_init(q_full, 1);
@@ -210,7 +231,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
             bool armed[C::STAGES];
             uint32_t armed_phase[C::STAGES];
             for (int s = 0; s < C::STAGES; ++s) armed[s] = false;
-            for (int j = 0; j < n_kv; ++j) {
+            for (int j = j0; j < j0 + nj; ++j) {
                 if (!mbar_wait(&kv_empty[stage], phase ^ 1u, abort_flag, g.err)) break;
                 mbar_arrive_expect_tx(&kv_full[stage], C::STAGE);
                 uint8_t* sk = skv + stage * C::STAGE;
@@ -266,7 +287,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
             // tile has its own issuer, so neither waits behind the other's
             // softmax
             const int t = warp - 1;
-            for (int j = 0; j < n_kv && ok; ++j) {
+            for (int j = 0; j < nj && ok; ++j) {
                 if (!mbar_wait(&kv_full[stage], phase, abort_flag, g.err)) { ok = false; break; }
                 tc_fence_after();
                 if (j > 0) {
@@ -285,9 +306,9 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
                 prev = stage;
                 if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
             }
-            if (ok && mbar_wait(&p_full[t], (n_kv - 1) & 1, abort_flag, g.err)) {
+            if (ok && mbar_wait(&p_full[t], (nj - 1) & 1, abort_flag, g.err)) {
                 tc_fence_after();
-                issue_pv(t, prev, n_kv > 1);
+                issue_pv(t, prev, nj > 1);
                 tc_commit(&kv_empty[prev]);
                 tc_commit(&o_final[t]);
             }
@@ -308,10 +329,11 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
         const uint32_t p_addr = tmem + lane_base + C::p_col(t);
         const uint32_t o_addr = tmem + lane_base + C::o_col(t);
         const int last_valid = g.L - (n_kv - 1) * BKV;       // keys in the last tile
+        const int mask_step = (j0 + nj == n_kv && last_valid < BKV) ? nj - 1 : -1;   // this CTA's ragged step
         float m_run = -INFINITY, l_run = 0.f;
         const uint64_t scale2 = pair(g.scale_log2, g.scale_log2);
         bool ok = true;
-        for (int j = 0; j < n_kv; ++j) {
+        for (int j = 0; j < nj; ++j) {                  // j counts this CTA's steps
             if (!mbar_wait(&s_full[t], j & 1, abort_flag, g.err)) { ok = false; break; }
             tc_fence_after();
             float s[BKV];
@@ -322,7 +344,7 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&s_free[t]);
-            if (j == n_kv - 1 && last_valid < BKV) {
+            if (j == mask_step) {
 #pragma unroll
                 for (int c = 0; c < BKV; ++c)
                     if (c >= last_valid) s[c] = -INFINITY;
@@ -395,7 +417,24 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(&p_full[t]);
         }
-        if (ok && mbar_wait(&o_final[t], 0, abort_flag, g.err)) {
+        if (ok && is_part && mbar_wait(&o_final[t], 0, abort_flag, g.err)) {
+            // a part of a split unit: unnormalised O with its base and row
+            // sum, merged by the combine kernel
+            tc_fence_after();
+            const size_t prow = (size_t)pslot * (2 * BQ) + t * BQ + row;
+            float4* dst = reinterpret_cast<float4*>(g.part_o + prow * D);
+#pragma unroll
+            for (int c = 0; c < D; c += 32) {
+                uint32_t o[32];
+                tmem_ld32(o_addr + c, o);
+                tmem_ld_wait();
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    dst[c / 4 + q] = make_float4(__uint_as_float(o[4 * q]), __uint_as_float(o[4 * q + 1]),
+                                                 __uint_as_float(o[4 * q + 2]), __uint_as_float(o[4 * q + 3]));
+            }
+            reinterpret_cast<float2*>(g.part_ml)[prow] = make_float2(m_run, l_run);
+        } else if (ok && mbar_wait(&o_final[t], 0, abort_flag, g.err)) {
             tc_fence_after();
             const int tok = q0 + t * BQ + row;
             const float inv = 1.0f / l_run;
@@ -436,6 +475,65 @@ __global__ void __launch_bounds__(AttnCfg<D>::THREADS, 1)
     }
 }
 
+// Merges the key-range parts of each split unit: one warp per query row,
+// lane l owning columns l, l + 32, ...: O = sum_p 2^(m_p - m) O_p / l with
+// m = max_p m_p and l = sum_p 2^(m_p - m) l_p (bases in the log2 domain of
+// the numerators).
+template <int D, bool BATCH>
+__global__ void __launch_bounds__(256) attn_combine_kernel(const AttnArgs g, int n_split_units) {
+    const int w = (int)((blockIdx.x * 256u + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    if (w >= n_split_units * 2 * BQ) return;
+    const int ug = w / (2 * BQ), r = w - ug * (2 * BQ);      // split unit over all samples, row
+    const int n_split_s = g.units_s - g.n_full;
+    const int smp = ug / n_split_s, u = ug - smp * n_split_s;
+    const int unit = smp * g.units_s + g.n_full + u;
+    const int h = unit / g.q_blocks;
+    const int tok = (unit % g.q_blocks) * (2 * BQ) + r;
+    if (tok >= g.L) return;
+    const float2* ml = reinterpret_cast<const float2*>(g.part_ml);
+    const size_t slot0 = (size_t)ug * g.split;                // = smp * n_split_s * split + u * split
+    float m = -INFINITY;
+    for (int p = 0; p < g.split; ++p) m = fmaxf(m, ml[(slot0 + p) * (2 * BQ) + r].x);
+    float l = 0.f, acc[D / 32];
+#pragma unroll
+    for (int i = 0; i < D / 32; ++i) acc[i] = 0.f;
+    for (int p = 0; p < g.split; ++p) {
+        const size_t prow = (slot0 + p) * (2 * BQ) + r;
+        const float2 mp = ml[prow];
+        const float f = ex2(mp.x - m);
+        l = fmaf(mp.y, f, l);
+        const float* po = g.part_o + prow * D;
+#pragma unroll
+        for (int i = 0; i < D / 32; ++i) acc[i] = fmaf(f, po[lane + 32 * i], acc[i]);
+    }
+    size_t orow = (size_t)tok;
+    int hs = h;
+    if constexpr (BATCH) {
+        const int b = h / g.Hs;
+        hs = h - b * g.Hs;
+        orow = (size_t)batch_row(b, tok, g.nb, g.Lc, g.L);
+    }
+    const float inv = 1.0f / l;
+    __nv_bfloat16* dst = g.o + orow * g.Hs * D + (size_t)hs * D;
+#pragma unroll
+    for (int i = 0; i < D / 32; ++i) dst[lane + 32 * i] = __float2bfloat16_rn(acc[i] * inv);
+}
+
+// Units of a sample's last, partial round are split over the key range so
+// that its CTAs fill the SMs: r = units mod SMs leftover units, each in
+// min(8, SMs / r, steps) parts (none when the grid is whole rounds).
+int attn_split(int units, int num_sms, int n_kv, int& n_full) {
+    n_full = units;
+    const int r = units % num_sms;
+    if (r == 0) return 1;
+    int split = num_sms / r;
+    if (split > 8) split = 8;
+    if (split > n_kv) split = n_kv;
+    if (split < 2) return 1;
+    n_full = units - r;
+    return split;
+}
+
 template <int D, bool BATCH>
 wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, int ldv, void* o, int H, int L, int Hs,
                   int Lc, cudaStream_t s) {
@@ -473,9 +571,28 @@ wdc_status launch(Ctx* c, const void* q, const void* k, const void* vt, int ldv,
     g.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
     g.o = reinterpret_cast<__nv_bfloat16*>(o);
     g.err = c->err;
-    attn_tc_kernel<D, BATCH><<<H * g.q_blocks, Cf::THREADS, Cf::SMEM, s>>>(tq, tk, tv, g);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 attention launch: ") + cudaGetErrorString(e));
+    g.units_s = Hs * g.q_blocks;
+    g.split = attn_split(g.units_s, c->num_sms, g.n_kv, g.n_full);
+    // the workspace holds num_sms part CTAs per sample of the model's batch
+    if (!c->attn_part || g.nb > c->attn_part_samples) g.split = 1;
+    if (g.split == 1) g.n_full = g.units_s;
+    g.part_o = c->attn_part;
+    g.part_ml = c->attn_ml;
+    const int n_split = g.nb * (g.units_s - g.n_full);       // split units over all samples
+    {
+        LaunchScope ls(c, WDC_K_ATTN, s);
+        attn_tc_kernel<D, BATCH><<<g.nb * (g.n_full + (g.units_s - g.n_full) * g.split), Cf::THREADS, Cf::SMEM, s>>>(
+            tq, tk, tv, g);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("tcgen05 attention launch: ") + cudaGetErrorString(e));
+    }
+    if (n_split > 0) {
+        LaunchScope ls(c, WDC_K_OTHER, s);
+        const int threads = n_split * 2 * BQ * 32;
+        attn_combine_kernel<D, BATCH><<<(threads + 255) / 256, 256, 0, s>>>(g, n_split);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return fail(c, WDC_ERR_CUDA, std::string("attention combine launch: ") + cudaGetErrorString(e));
+    }
     return WDC_OK;
 }
 

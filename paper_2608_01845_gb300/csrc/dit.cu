@@ -504,8 +504,7 @@ static wdc_status attention(Ctx* c, const void* q, const void* k, const void* vt
     if (c->cfg.dtype == WDC_BF16) {
         if (!tc_attention_supported(L, d))
             return fail(c, WDC_ERR_UNSUPPORTED, "bf16 attention needs head_dim 64 or 128 and L > 0");
-        LaunchScope ls(c, WDC_K_ATTN, s);
-        return tc_attention(c, q, k, vt, ldv, o, H, L, d, Hs, Lc, s);
+        return tc_attention(c, q, k, vt, ldv, o, H, L, d, Hs, Lc, s);     // times its own launches
     }
     LaunchScope ls(c, WDC_K_ATTN, s);
     dim3 grid(blocks_for(L, 128), H);
@@ -604,6 +603,12 @@ wdc_status dit_create(Ctx* c) {
     if ((s = dalloc(c, (void**)&t->h1, (size_t)t->E * sizeof(float)))) return s;
     if ((s = dalloc(c, (void**)&t->temb, (size_t)t->E * sizeof(float)))) return s;
     if ((s = dalloc(c, (void**)&t->mods, t->mod_rows * sizeof(float)))) return s;
+    if (t->dtype == WDC_BF16) {
+        const size_t rows = (size_t)t->B * c->num_sms * 256;
+        if ((s = dalloc(c, (void**)&c->attn_part, rows * 128 * sizeof(float)))) return s;
+        if ((s = dalloc(c, (void**)&c->attn_ml, rows * 2 * sizeof(float)))) return s;
+        c->attn_part_samples = t->B;
+    }
     const long long npe = (long long)t->Lv * t->D;
     LaunchScope ls(c, WDC_K_OTHER, 0);
     if (t->dtype == WDC_BF16)
@@ -620,6 +625,9 @@ void dit_destroy(Ctx* c) {
     for (void* p : c->dit->allocs) cudaFree(p);
     delete c->dit;
     c->dit = nullptr;
+    c->attn_part = nullptr;
+    c->attn_ml = nullptr;
+    c->attn_part_samples = 0;
 }
 
 static uint16_t f32_to_bf16_bits(float f) {

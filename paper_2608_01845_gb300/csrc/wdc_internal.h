@@ -160,6 +160,12 @@ struct Ctx {
 
     // denoiser
     struct DiT* dit = nullptr;
+    // split-key attention partials of a sample's last round (bf16 models):
+    // per sample of the batch, unnormalised O rows [num_sms x 256][128] and
+    // (base, row sum) pairs
+    float* attn_part = nullptr;
+    float* attn_ml = nullptr;
+    int attn_part_samples = 0;
 
     // graph rollout (device-side control flow), built on first use
     GraphRollout* grollout = nullptr;
