@@ -463,7 +463,10 @@ wdc_status wdc_op_gemm(wdc_ctx* ctx, const void* A, const void* W, const float* 
  * stores V that way so that the PV product takes the probabilities in fp16),
  * with ldv = L rounded up to a multiple of 8 so that every V^T row starts on
  * a 16-byte boundary; the padding columns are never read.  Any L >= 1; d 64
- * or 128. */
+ * or 128.  A bf16 model may split the last (head, query block) units of the
+ * launch over the key range and merge them with a second kernel through a
+ * workspace the context owns, so two attention calls of one context must
+ * not run concurrently on different streams. */
 wdc_status wdc_op_attention(wdc_ctx* ctx, const void* q, const void* k, const void* vt, void* o,
                             int heads, int L, int d, wdc_stream stream);
 
