@@ -59,6 +59,13 @@ __device__ __forceinline__ float signed_term(uint32_t idx, uint32_t seed, float 
 
 // Butterfly sum over the 32 lanes (a fixed-order tree: every lane ends with
 // the same value).
+// Bulk prefetch of `bytes` (a multiple of 16, 16-byte aligned) into L2.
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+// Runs per warp whose bank reads are prefetched while warp 0 forms the head.
+constexpr int kPrefetchRuns = 4;
+
 __device__ __forceinline__ float warp_sum_f(float v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -476,6 +483,23 @@ __device__ __forceinline__ void pass_body(const PassArgs& a_in) {
     bool do_stream = true;
     float kap[K > 0 ? K : 1];
     float alpha_f = 0.f;
+    if constexpr ((MODE == kModeSkip || MODE == kModeResidual || MODE == kModeObserve) && K > 0) {
+        // while warp 0 forms the head, the other warps start the HBM reads of
+        // their first runs (into L2): lane i < K takes bank record i, lane K
+        // the anchor (observe / residual) or the current latent (residual)
+        if (warp != 0 && lane <= K) {
+            const float* src = lane < K ? a.src[lane] : (MODE == kModeSkip ? nullptr : a.anchor);
+            const long long gw = (long long)blockIdx.x * kWarps + warp;
+            const long long stride = (long long)gridDim.x * kWarps;
+            if (src) {
+                for (int it = 0; it < kPrefetchRuns; ++it) {
+                    const long long r = gw + it * stride;
+                    if (r >= full) break;
+                    prefetch_l2(src + r * kRun, kRun * 4);
+                }
+            }
+        }
+    }
     if (MODE == kModeSkip || MODE == kModeResidual) {
         if (warp == 0) skip_head_warp<K>(a, ps.S, ps.rs, hs);
         __syncthreads();
