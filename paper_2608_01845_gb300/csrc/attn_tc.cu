@@ -37,6 +37,11 @@
 //     S(t, j), PV(t, j-1)
 // and the MMA of S(t, j+1) overlaps the softmax of step j instead of
 // waiting behind PV(t, j).
+// Grid: one CTA per (head, 256-query) unit, one CTA per SM.  The units of a
+// sample's last, partial round are split over the key range instead: each
+// part runs the same pipeline over its steps and writes its unnormalised O,
+// exponent base and row sum to a workspace of the context, and
+// attn_combine_kernel merges the parts, so the round's CTAs fill the SMs.
 // Keys past L are masked (TMA zero-fills out-of-range K / V^T).  Every
 // mbarrier wait is bounded.
 #include "dit_kernels.cuh"
