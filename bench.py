@@ -42,6 +42,7 @@ WORKLOAD_5B = dict(
     layers=42, hidden=3072, heads=48, head_dim=64, mlp=12288, temb_dim=512, freq_dim=256,
     in_ch=16, frames=13, height=60, width=90, patch=2, cond_tokens=226, cond_dim=3072, dual_stream=0,
     T=50, tau_risk=0.1, target_exact=23, weight_seed=1234, input_seed=77,
+    paper_speedup=2.15,
 )
 # The HunyuanVoyager-13B-like cached rollout: 60 dual-stream layers (separate
 # condition-token weights, joint attention), 24 heads x 128, latent 16x13x64x64
@@ -52,6 +53,7 @@ WORKLOAD_13B = dict(
     layers=60, hidden=3072, heads=24, head_dim=128, mlp=12288, temb_dim=512, freq_dim=256,
     in_ch=16, frames=13, height=64, width=64, patch=2, cond_tokens=256, cond_dim=3072, dual_stream=1,
     T=50, tau_risk=0.8, target_exact=10, weight_seed=4321, input_seed=91,
+    paper_speedup=4.92,
 )
 WORKLOADS = {"5b": WORKLOAD_5B, "13b": WORKLOAD_13B}
 SKIP_SWEEP_N = 1 << 28          # fused skip pass measured at 2^28 fp32 elements, bank of 4
@@ -409,6 +411,26 @@ def surrogate_reading(flags):
     return "Eq. 5 as printed: sum_i kappa_i z_out_i"
 
 
+def native_speedup(torch, ctx, w, zT_d, cond, cached_steps_per_s):
+    """One uncached rollout (every step an exact forward, wdc_native_rollout)
+    on the same context and inputs, CUDA events: its steps/s and the cached
+    rollout's speedup over it, beside the paper's speedup for the model this
+    workload is shaped like (8x A6000, context only)."""
+    T = w["T"]
+    nat = torch.empty_like(zT_d)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    ctx.native_rollout(zT_d, cond, nat)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    del nat
+    native = T / (ms * 1e-3)
+    return {"steps_per_s": native, "ms_per_rollout": ms, "speedup_cached_vs_native": cached_steps_per_s / native,
+            "paper_speedup": w["paper_speedup"], "paper_hardware": "8x NVIDIA A6000 (context, not the target)"}
+
+
 def rollout_component(torch, wdc, w, peaks, reps=2):
     """One workload's cached rollout on its own context: steps/s over `reps`
     timed rollouts after one warm-up, the exact-step count, and the dominant
@@ -444,12 +466,13 @@ def rollout_component(torch, wdc, w, peaks, reps=2):
     else:
         avg = None
         achieved = None
+    native = native_speedup(torch, ctx, w, zT_d, cond, T / (ms * 1e-3))
     ctx.close()
     del zT_d, ct_d, out
     torch.cuda.empty_cache()
     res = {"workload": w["name"], "steps_per_s": T / (ms * 1e-3), "ms_per_rollout": ms, "exact_steps": exact,
            "tau_risk": w["tau_risk"], "dominant_kernel": dom,
-           "time_share": {k: v / sum(cls.values()) for k, v in cls.items()}}
+           "time_share": {k: v / sum(cls.values()) for k, v in cls.items()}, "native_rollout": native}
     if achieved is not None:
         res.update({"attention_avg_launch_ms": avg, "attention_tflops": achieved,
                     "attention_frac_of_measured_sustained": achieved / peaks["bf16_tflops_sustained"]})
@@ -659,6 +682,7 @@ def run_gpu(args, rank, world, local_rank):
         gt = time.perf_counter() - t0
         line["graph_rollout"] = {"steps_per_s": T / gt, "exact_steps": T - sum(dec_g),
                                  "note": "wdc_rollout_graph: no host synchronisation between steps"}
+        line["native_rollout"] = native_speedup(torch, ctx, w, zT_d, cond, T * args.steps / (ms * 1e-3))
 
     if args.ablation and rank == 0:
         # mechanics of the variant on the random-init model: final latent
