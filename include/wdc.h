@@ -381,7 +381,9 @@ wdc_status wdc_risk_update(wdc_ctx* ctx, int k, const wdc_cond* c, const float* 
  * each a wdc_surrogate_step and, on Exact, wdc_dit_forward + wdc_risk_update.
  * z_T and z_out may be device or host pointers (host ones are staged through
  * the context's buffers).  conds: n_cond == 1 (used for every step) or T
- * entries.  decisions (host int[T]) and trace (host wdc_step_info[T]) may be
+ * entries; their tokens may be device or host memory (host tokens are copied
+ * into a staging buffer the context keeps, grown on the first call that needs
+ * more; the call allocates device memory then).  decisions (host int[T]) and trace (host wdc_step_info[T]) may be
  * NULL.  Synchronises the stream once per step. */
 wdc_status wdc_rollout(wdc_ctx* ctx, const float* z_T, const wdc_cond* conds, int n_cond,
                        float* z_out, int* decisions, wdc_step_info* trace, wdc_stream stream);

@@ -377,6 +377,7 @@ void wdc_destroy(wdc_ctx* h) {
     cudaFree(c->cand[1]);
     cudaFree(c->vbuf);
     cudaFree(c->zstage);
+    cudaFree(c->cond_stage);
     for (int i = 0; i < kMaxBank; ++i) cudaFree(c->disp[i]);
     if (c->out_host) cudaFreeHost(c->out_host);
     if (c->st_host) cudaFreeHost(c->st_host);
@@ -791,22 +792,29 @@ static wdc_status rollout_impl(Ctx* c, const float* z_T, const wdc_cond* conds, 
     // condition tokens: device pointers are used directly, host ones staged
     const size_t cond_elems = (size_t)c->cfg.cond_tokens * c->cfg.cond_dim;
     std::vector<const float*> tok(n_cond, nullptr);
-    float* cstage = nullptr;
     for (int i = 0; i < n_cond; ++i) {
         if (cond_elems == 0) continue;
         if (!conds[i].tokens) return fail(c, WDC_ERR_INVALID_ARG, "condition tokens required");
         if (is_device_ptr(conds[i].tokens)) { tok[i] = conds[i].tokens; continue; }
-        if (!cstage) {
-            if (cudaMalloc((void**)&cstage, cond_elems * sizeof(float) * n_cond) != cudaSuccess) {
+        // host tokens go through the context's staging buffer, kept between
+        // calls and grown when a call needs more
+        const size_t need = cond_elems * sizeof(float) * n_cond;
+        if (c->cond_stage_bytes < need) {
+            WDC_CUDA_TRY(c, cudaStreamSynchronize(s));   // a failed earlier call may still read the old one
+            cudaFree(c->cond_stage);
+            c->cond_stage = nullptr;
+            c->cond_stage_bytes = 0;
+            if (cudaMalloc((void**)&c->cond_stage, need) != cudaSuccess) {
                 cudaGetLastError();
+                c->cond_stage = nullptr;
                 return fail(c, WDC_ERR_OOM, "condition staging");
             }
+            c->cond_stage_bytes = need;
         }
-        WDC_CUDA_TRY(c, cudaMemcpyAsync(cstage + cond_elems * i, conds[i].tokens, cond_elems * sizeof(float),
+        WDC_CUDA_TRY(c, cudaMemcpyAsync(c->cond_stage + cond_elems * i, conds[i].tokens, cond_elems * sizeof(float),
                                         cudaMemcpyHostToDevice, s));
-        tok[i] = cstage + cond_elems * i;
+        tok[i] = c->cond_stage + cond_elems * i;
     }
-    struct Free { float* p; ~Free() { if (p) { cudaStreamSynchronize(0); cudaFree(p); } } } guard{cstage};
 
     WDC_CUDA_TRY(c, cudaMemcpyAsync(c->cand[0], z_T, bytes, in_dev ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s));
     float* cur = c->cand[0];

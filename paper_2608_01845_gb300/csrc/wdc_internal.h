@@ -150,6 +150,8 @@ struct Ctx {
     float* cand[2] = {};               // rollout candidate buffers
     float* vbuf = nullptr;
     float* zstage = nullptr;           // host-pointer staging for rollouts
+    float* cond_stage = nullptr;       // host condition tokens staged for rollouts (grown on demand)
+    size_t cond_stage_bytes = 0;
     float* disp[kMaxBank] = {};        // secant / residual reading: z_out - z_in per bank slot
     const float* cur_latent = nullptr; // current latent of the step API (read by secant / residual)
 

@@ -121,6 +121,25 @@ def test_host_pointer_rollout_equals_device_rollout():
     assert torch.equal(host_out, dev_out.cpu())
 
 
+def test_host_condition_staging_grows_and_is_reused():
+    """Host condition tokens go through the context's staging buffer: one
+    condition, then one per step (the buffer grows), then one again; each
+    rollout equals the same rollout from device tokens bitwise."""
+    T = 10
+    op, cp, W, ctx, z0, ct, desc = _setup(T, tau_risk=0.5)
+    zT = torch.from_numpy(z0.ravel().copy()).cuda()
+    cts = [synth.cond_tokens(10 + k, 16, 256) for k in range(T)]
+    for tokens in ([ct], cts, [ct]):
+        dev = [wdc.make_cond(torch.from_numpy(x).cuda(), desc["cam"], desc["depth"]) for x in tokens]
+        host = [wdc.make_cond(torch.from_numpy(x.copy()).pin_memory(), desc["cam"], desc["depth"]) for x in tokens]
+        a = torch.empty_like(zT)
+        b = torch.empty_like(zT)
+        d1, _ = ctx.rollout(zT, dev, a)
+        d2, _ = ctx.rollout(zT, host, b)
+        assert d1 == d2
+        assert torch.equal(a, b)
+
+
 def test_age_convention_budget_on_gpu():
     gold = json.load(open(os.path.join(GOLDEN, "age_convention.json")))
     T = gold["T"]
