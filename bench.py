@@ -347,12 +347,41 @@ def copy_ms(torch, nbytes, reps=10):
     return statistics.median(ts)
 
 
-def skip_sweep(torch, wdc, peaks, workload_n):
+def oracle_step_gbps(n, K):
+    """The CPU oracle's surrogate step and anchor step at n latent elements
+    with a bank of K records (filled by K exact steps first), each timed once
+    on the host cores, as GB/s of the same algorithmic bytes as the GPU
+    passes: (K+1)*4n and 5*4n."""
+    from oracle import rollout as ro
+    from oracle import schedule as sch
+    from oracle.params import CacheParams
+    from paper_2608_01845_gb300 import synth
+    p = CacheParams(tau_risk=0.5, bank_capacity=K)
+    sig = sch.sigmas(50)
+    z = synth.latent(5, (n,))
+    v = synth.normal(6, (n,))
+    st = ro.CacheState.initial(z, sig, p)
+    for k in range(K):
+        zh, info = ro.surrogate_step(st, z, k, {}, sig, p)
+        z = ro.exact_step(st, z, v, zh, k, {}, sig, p, info)
+    t0 = time.perf_counter()
+    zh, info = ro.surrogate_step(st, z, K, {}, sig, p)
+    t_skip = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    ro.exact_step(st, z, v, zh, K, {}, sig, p, info)
+    t_anchor = time.perf_counter() - t0
+    return {"skip_gbps": (K + 1) * 4 * n / t_skip / 1e9, "anchor_gbps": 5 * 4 * n / t_anchor / 1e9,
+            "cores": os.cpu_count(), "kind": "oracle"}
+
+
+def skip_sweep(torch, wdc, peaks, workload_n, cpu=False):
     """The skipped-step kernel sweep: N in {2^20, 2^24, 2^26, 2^28} fp32
     elements x K in {2, 3, 4} bank records, L2 flushed before every launch;
     plus 2^20 L2-resident and the workload's own latent size.  Each row also
     gives a plain copy of the same byte count timed the same way, and the
-    pass's time against it."""
+    pass's time against it; with `cpu`, the 2^20 rows also give the CPU
+    oracle's surrogate and anchor steps (larger sizes take the oracle minutes
+    per bank fill)."""
     rows = []
     for e in (20, 24, 26, 28):
         for K in (2, 3, 4):
@@ -361,6 +390,9 @@ def skip_sweep(torch, wdc, peaks, workload_n):
             rows.append({"n": f"2^{e}", "K": K, "gbps": round(r["gbps"], 1), "ms": round(r["ms"], 5),
                          "frac_of_measured_copy": round(r["frac_of_measured_copy"], 4),
                          "same_bytes_copy_ms": round(cms, 5), "frac_of_same_bytes_copy": round(cms / r["ms"], 4)})
+            if cpu and e == 20:
+                rows[-1]["cpu_oracle"] = {k: (round(v, 4) if isinstance(v, float) else v)
+                                          for k, v in oracle_step_gbps(1 << e, K).items()}
     r = skip_pass_gbps(torch, wdc, peaks, n=1 << 20, K=4, flush=False)
     rows.append({"n": "2^20", "K": 4, "l2": "resident", "gbps": round(r["gbps"], 1), "ms": round(r["ms"], 5),
                  "frac_of_measured_copy": round(r["frac_of_measured_copy"], 4)})
@@ -713,7 +745,8 @@ def run_gpu(args, rank, world, local_rank):
         line["components"]["skip_pass"] = skip_pass_gbps(torch, wdc, peaks)
         line["components"]["secant_pass"] = skip_pass_gbps(torch, wdc, peaks, secant=True)
         line["components"]["skip_sweep"] = skip_sweep(torch, wdc, peaks,
-                                                      w["in_ch"] * w["frames"] * w["height"] * w["width"])
+                                                      w["in_ch"] * w["frames"] * w["height"] * w["width"],
+                                                      cpu=world == 1 and not args.no_cpu_baseline)
         line["components"]["peaks"] = {"hbm_gbs": peaks["hbm_gbs"], "bf16_tflops": peaks["bf16_tflops"],
                                        "source": peak_src}
         if world == 1 and not args.no_cpu_baseline:
