@@ -95,6 +95,61 @@ def test_skip_pass_full_size_64M():
     _check_skip(info, info_o, zh, zh_o, 4)
 
 
+@pytest.mark.parametrize("K", [2, 4])
+def test_skip_pass_2e28_sampled_and_reductions(K):
+    """The sweep's largest launch (2^28 elements, the bench's bank recipe and
+    launch): every output checked by what holds at any size.  The observation
+    (Eq. 5) on 2^20 sampled elements plus both ends equals sum_i kappa_i z_i
+    with the kernel's own kappa (fp64, 1e-6 of the terms' magnitude); kappa is
+    a softmax (non-negative, sums to 1); the statistics the next lift reads --
+    the sum of squares of z_hat and of z_hat - z_a, and the signed sketch of
+    z_hat -- equal fp64 sums of the kernel's z_hat (the sketch through the
+    oracle's sketch) within 1e-5."""
+    from oracle import summary as sm
+    n, T, k = 1 << 28, 50, 20
+    # every record compatible, as in the bench's sweep; a risk threshold no
+    # candidate reaches, so the pass commits the candidate's statistics
+    op, cp = params_for_both(bank_capacity=K, sim_min=-1.0, q_gap_max=1.0, tau_risk=1e9)
+    ctx = _ctx(n, cp, T)
+    bank = synth.drift_bank_device(n % 1000003 + K, n, K)
+    st = wdc.StateHost()
+    st.n_bank, st.R, st.eta = K, 0.1, 1.0
+    g = np.random.default_rng(0)
+    for i in range(K):
+        a = g.standard_normal(256)
+        for j in range(256):
+            st.rec[i].s_in[j] = a[j]
+            st.rec[i].s_out[j] = a[j] + 0.1
+            st.rec[i].s_dphi[j] = 0.1
+        st.rec[i].q_in = 0.6 + 0.02 * (K - i)
+        st.rec[i].q_out = st.rec[i].q_in - 0.02
+    st.q_a_in, st.q_a_out = st.rec[K - 1].q_in, st.rec[K - 1].q_out
+    zc = bank[-1] + 0.01
+    ctx.state_set(st, bank, zc)
+    zh = torch.empty(n, device="cuda")
+    info = ctx.surrogate_step(k, wdc.make_cond(), zh)
+    assert info.supported == 1 and info.finite == 1 and info.decision == 1
+    kap = np.array(list(info.kappa)[:K], dtype=np.float64)
+    assert np.all(kap >= 0.0) and abs(kap.sum() - 1.0) <= 1e-6
+    gen = torch.Generator(device="cuda").manual_seed(3)
+    idx = torch.cat([torch.arange(4096, device="cuda"), torch.arange(n - 4096, n, device="cuda"),
+                     torch.randint(0, n, (1 << 20,), device="cuda", generator=gen)])
+    terms = torch.stack([float(kap[i]) * bank[i][idx].double() for i in range(K)])
+    want = terms.sum(0)
+    scale = terms.abs().sum(0) + 1e-30
+    assert float(((zh[idx].double() - want).abs() / scale).max()) <= 1e-6
+    s = ctx.state_get()
+    zd = zh.double()
+    ss = float((zd * zd).sum())
+    assert abs(s.cur_sumsq - ss) <= 1e-5 * ss
+    d = zd - bank[-1].double()
+    sa = float((d * d).sum())
+    assert abs(s.cur_sumsq_anchor - sa) <= 1e-5 * sa
+    del zd, d
+    want_sk = sm.sketch(zh.cpu().numpy(), op.sketch_seed) / math.sqrt(120.0 / n)
+    assert rel_l2(np.array(s.cur_sketch), want_sk) <= 1e-5
+
+
 @pytest.mark.parametrize("n,K", [(128 * 1000 + 37, 1), (1 << 20, 4), (4096 * 3 + 128 * 5 + 64, 8)])
 def test_anchor_pass_parity(n, K):
     (ctx, op, cp, sig, z_k, st, st_o, cond, zh, zh_o, info, info_o, c, bank, zc) = _run_skip(n, K, 23 + K, -0.05)
