@@ -67,9 +67,15 @@ def _h(a):
     return np.asarray(a, dtype=np.float32).astype(np.float16).astype(np.float32)
 
 
-@pytest.mark.parametrize("M,N,K", [(300, 384, 320), (128, 256, 64), (1000, 768, 1024), (17, 64, 128)])
+@pytest.mark.parametrize("M,N,K", [(300, 384, 320), (128, 256, 64), (1000, 768, 1024), (17, 64, 128), (1, 32, 8),
+                                   (257, 32, 8)])
 @pytest.mark.parametrize("mode", ["store", "gelu", "resid"])
 def test_bf16_gemm_matches_oracle(M, N, K, mode):
+    """The tcgen05 GEMMs (one CTA per tile below 256 rows, CTA pairs from
+    256) with each fused epilogue, down to the smallest shapes they take: one
+    row, one 32-column chunk, one 8-element K step (one 64-wide K block,
+    zero-filled past K), and a pair grid whose second 256-row tile holds a
+    single row."""
     ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.BF16)
     A = _bf(synth.normal(1, (M, K)))
     W = _bf(synth.normal(2, (N, K), 0.05))
@@ -95,12 +101,14 @@ def test_bf16_gemm_matches_oracle(M, N, K, mode):
 
 
 @pytest.mark.parametrize("H,L,d", [(2, 1000, 64), (1, 1000, 128), (3, 264, 64), (1, 64, 128), (2, 4104, 64),
-                                   (1, 2056, 128), (2, 300, 64), (1, 129, 128), (1, 40, 64), (2, 400, 64)])
+                                   (1, 2056, 128), (2, 300, 64), (1, 129, 128), (1, 40, 64), (2, 400, 64),
+                                   (1, 1, 64), (2, 7, 128)])
 def test_bf16_attention_matches_oracle(H, L, d):
     """Every L runs the tcgen05 kernel, ragged against its 128-key steps and
     256-query CTAs (L = 40 and 400 leave the last CTA one partial query
-    tile); V^T rows are padded to a multiple of 8 tokens, and the padding
-    holds NaN to show it is never read."""
+    tile; L = 1 and 7 are a single ragged step, and at L = 1 the output is
+    the one value row); V^T rows are padded to a multiple of 8 tokens, and
+    the padding holds NaN to show it is never read."""
     ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.BF16)
     q = _bf(synth.normal(11, (H, L, d)))
     k = _bf(synth.normal(12, (H, L, d)))
