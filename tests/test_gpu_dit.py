@@ -102,13 +102,13 @@ def test_bf16_gemm_matches_oracle(M, N, K, mode):
 
 @pytest.mark.parametrize("H,L,d", [(2, 1000, 64), (1, 1000, 128), (3, 264, 64), (1, 64, 128), (2, 4104, 64),
                                    (1, 2056, 128), (2, 300, 64), (1, 129, 128), (1, 40, 64), (2, 400, 64),
-                                   (1, 1, 64), (2, 7, 128)])
+                                   (1, 1, 64), (2, 7, 128), (2, 100, 64)])
 def test_bf16_attention_matches_oracle(H, L, d):
     """Every L runs the tcgen05 kernel, ragged against its 128-key steps and
     256-query CTAs (L = 40 and 400 leave the last CTA one partial query
     tile; L = 1 and 7 are a single ragged step, and at L = 1 the output is
-    the one value row); V^T rows are padded to a multiple of 8 tokens, and
-    the padding holds NaN to show it is never read."""
+    the one value row); V^T rows are padded to a multiple of 8 tokens, and the padding
+    holds NaN to show it is never read."""
     ctx = _ctx(dict(PARITY_MODEL, layers=1), wdc.BF16)
     q = _bf(synth.normal(11, (H, L, d)))
     k = _bf(synth.normal(12, (H, L, d)))
