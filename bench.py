@@ -440,6 +440,8 @@ def surrogate_reading(flags):
         return "native latent secant (ablation)"
     if flags & 0x100:
         return "residual reading of Eq. 5: z_t + sum_i kappa_i (z_out_i - z_in_i)"
+    if flags & 0x40:
+        return "linear observation (ablation): sum_i beta_i z_out_i, beta the ridge readout of the lifted summary"
     return "Eq. 5 as printed: sum_i kappa_i z_out_i"
 
 
