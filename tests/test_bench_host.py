@@ -36,3 +36,26 @@ def test_traffic_is_reported_only_for_the_captured_source():
             assert got is None
         other = "13b" if e["bench_workload"] == "5b" else "5b"
         assert bench.traffic_for(path, other) is None
+
+
+def test_surrogate_reading_names_each_observation():
+    assert bench.surrogate_reading(0).startswith("Eq. 5 as printed")
+    assert bench.surrogate_reading(0x02).startswith("native latent secant")
+    assert bench.surrogate_reading(0x100).startswith("residual reading")
+    assert bench.surrogate_reading(0x40).startswith("linear observation")
+    # every ablation the bench offers maps to one reading
+    for v in bench.ABLATIONS.values():
+        assert bench.surrogate_reading(v["flags"])
+
+
+def test_oracle_step_rates_are_reported_per_host():
+    n, K = 4096, 2
+    r = bench.oracle_step_gbps(n, K)
+    assert r["kind"] == "oracle" and r["cores"] == os.cpu_count()
+    assert 0 < r["skip_gbps"] < 1e4 and 0 < r["anchor_gbps"] < 1e4
+
+
+def test_paper_speedups_sit_beside_the_right_workloads():
+    assert bench.WORKLOADS["5b"]["paper_speedup"] == 2.15     # Aether-5B, 47% exact calls
+    assert bench.WORKLOADS["13b"]["paper_speedup"] == 4.92    # HunyuanVoyager-13B, 20% exact calls
+    assert bench.WORKLOADS["5b"]["target_exact"] == 23 and bench.WORKLOADS["13b"]["target_exact"] == 10
