@@ -710,7 +710,7 @@ def run_gpu(args, rank, world, local_rank):
                    "h2d_bytes_per_step": zT.nbytes + ct.nbytes, "d2h_bytes_per_step": zT.nbytes,
                    "rollouts": e2e_reps,
                    "note": "without the per-launch event profiler the device-timed region runs for the roofline "
-                           "(two events per launch, about 0.5% of a rollout), so it can read slightly above value"}
+                           "(two events per launch, 0.2-0.4% of a rollout, measured), so it can read slightly above value"}
 
     # device-side control flow on the same workload (graph built by a first call)
     if rank == 0 and not args.ablation:
