@@ -745,7 +745,8 @@ def run_gpu(args, rank, world, local_rank):
         if not args.ablation and not args.no_extra_rollouts:
             other = "13b" if args.workload == "5b" else "5b"
             line["components"][f"rollout_{other}"] = rollout_component(torch, wdc, WORKLOADS[other], peaks)
-            line["components"]["rollout_cfg0"] = cfg0_component(torch, wdc, cpu=world == 1)
+            line["components"]["rollout_cfg0"] = cfg0_component(torch, wdc,
+                                                                cpu=world == 1 and not args.no_cpu_baseline)
         line["components"]["skip_pass"] = skip_pass_gbps(torch, wdc, peaks)
         line["components"]["secant_pass"] = skip_pass_gbps(torch, wdc, peaks, secant=True)
         line["components"]["skip_sweep"] = skip_sweep(torch, wdc, peaks,
